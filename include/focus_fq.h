@@ -1,0 +1,171 @@
+/*
+ * focus_fq.h -- C ABI of the FOCUS FP4 fake-quantizer for GB300 (sm_103a).
+ *
+ * FOCUS (Coupled-Relaxation and Dual-Granularity Scaling) learns the FP4
+ * quantization scale S^q separately from the stored, hardware-format
+ * dequantization scale S^dq.  Per block i of B contiguous elements along a
+ * row (B = 32 for MXFP4, 16 for NVFP4) and per sub-block k of b elements:
+ *
+ *   m_i      = max |x| over block i                              (Eq. 2-3)
+ *   S^dq_i   = MXFP4: 2^e_i, e_i from the E8M0 rule               (Eq. 3)
+ *              NVFP4: alpha * Q_E4M3(m_i / (alpha * 6))           (Eq. 2)
+ *   S^q_ik   = S^dq_i * c_i * c_i^k                               (Eq. 6, Eq. 8)
+ *   xbar     = Q_E2M1(x / S^q_ik),  y = xbar * S^dq_i             (Eq. 1, 7, 8)
+ *
+ * c_i is the per-block CRS coefficient (Sec. 3.3), c_i^k the per-sub-block
+ * DGS coefficient (Sec. 3.4).  The backward pass is the straight-through
+ * estimator the paper applies to every non-differentiable operation
+ * (Sec. 3.2).  The export writes what the deployed model keeps: FP4 codes and
+ * the dequantization scales (Fig. 3(d)).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All tensor pointers are DEVICE pointers owned by the caller.  The library
+ *   allocates nothing, keeps no pointer after a call returns and never
+ *   synchronises the host: work is enqueued on `stream` (NULL = the legacy
+ *   default stream) and completes asynchronously.
+ * - x, y, g and gx are row-major [rows, ld] arrays of desc->dtype; only the
+ *   first `cols` elements of each row are read or written.  They must be
+ *   16-byte aligned, and ld must be a multiple of 8 elements.
+ * - Coefficient arrays are dense fp32: crs / gcrs are [rows, cols/block] and
+ *   dgs / gdgs are [rows, cols/sub_block]; with coef_shared_rows = 1 both are
+ *   a single row ([cols/block], [cols/sub_block]) shared by all rows.  They
+ *   must be 16-byte aligned.  A NULL crs or dgs means "all coefficients 1".
+ * - Scale bytes are dense uint8 [rows, cols/block] (E8M0 biased exponent for
+ *   MXFP4, E4M3FN for NVFP4).  Codes are dense uint8 [rows, cols/2]: element
+ *   2t of a row in the low nibble of byte t, element 2t+1 in the high nibble;
+ *   a code is sign(1) | E2M1 magnitude index(3).  Codes must be 4-byte aligned.
+ * - Every call returns FOCUS_OK (0) or a negative focus_status_t.  Argument
+ *   errors are detected on the host before anything is launched; a launch
+ *   failure is reported as FOCUS_ERR_CUDA (cudaGetLastError is consumed).
+ * - Preconditions that are documented but not checked on the hot path: x and
+ *   g finite; coefficients finite and > 0; alpha finite and >= 0.  A
+ *   sub-block whose S^dq or S^q is zero or infinite is "dead": it yields
+ *   codes 0, values +0, input gradient +0 and no coefficient gradient.
+ * - Results are deterministic: no atomics, fixed reduction orders.
+ */
+#ifndef FOCUS_FQ_H
+#define FOCUS_FQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Opaque CUDA stream handle; identical to cudaStream_t. */
+typedef struct CUstream_st* focus_stream_t;
+
+typedef enum {
+    FOCUS_OK = 0,
+    FOCUS_ERR_INVALID_ARG = -1,   /* NULL where required, bad enum, ld < cols, ... */
+    FOCUS_ERR_UNSUPPORTED = -2,   /* block / sub-block / size outside what is built */
+    FOCUS_ERR_MISALIGNED = -3,    /* pointer or ld alignment rule broken */
+    FOCUS_ERR_WORKSPACE = -4,     /* workspace NULL or smaller than required */
+    FOCUS_ERR_CUDA = -5           /* the CUDA runtime reported an error */
+} focus_status_t;
+
+typedef enum { FOCUS_MXFP4 = 0, FOCUS_NVFP4 = 1 } focus_format_t;
+typedef enum { FOCUS_F32 = 0, FOCUS_BF16 = 1 } focus_dtype_t;
+typedef enum { FOCUS_STE_IDENTITY = 0, FOCUS_STE_CLIPPED = 1 } focus_ste_t;
+typedef enum { FOCUS_MX_CEIL = 0, FOCUS_MX_FLOOR = 1 } focus_mx_rule_t;
+
+/* Tensor and method descriptor (host memory, read during the call only).
+ *   rows, cols, ld    x is [rows, ld] row-major, blocks run along cols;
+ *                     cols % block == 0; rows * cols / 8 < 2^31.
+ *   dtype             focus_dtype_t of x, y, g and gx.
+ *   fmt               focus_format_t.
+ *   block             32 for FOCUS_MXFP4, 16 for FOCUS_NVFP4 (Sec. 3.1).
+ *   sub_block         DGS sub-block size b (Sec. 3.4): one of 2, 4, 8, 16,
+ *                     32 dividing block; b == block means K = 1 (CRS only).
+ *                     The paper uses 8 for both formats.
+ *   coef_shared_rows  0: coefficients per (row, block); 1: one set shared by
+ *                     all rows (channel-block coefficients of activations).
+ *   ste               focus_ste_t: IDENTITY passes the gradient through
+ *                     Q_E2M1 unchanged; CLIPPED zeroes it where |x/S^q| > 6.
+ *   mx_rule           focus_mx_rule_t, MXFP4 only: CEIL e = ceil(log2(m/6))
+ *                     (the paper's "typically ceiling", Eq. 3), or the OCP
+ *                     MX v1.0 rule e = floor(log2 m) - 2. */
+typedef struct {
+    int64_t rows;
+    int64_t cols;
+    int64_t ld;
+    int32_t dtype;
+    int32_t fmt;
+    int32_t block;
+    int32_t sub_block;
+    int32_t coef_shared_rows;
+    int32_t ste;
+    int32_t mx_rule;
+} focus_desc_t;
+
+/* Which workspace focus_workspace_bytes reports. */
+enum { FOCUS_WS_ALPHA = 0, FOCUS_WS_BWD = 1 };
+
+/* NVFP4 per-tensor scale, Eq. 2: alpha = max|x| / (M_FP4 * M_FP8)
+ * = fl(max|x| / 2688), written as one fp32 to *alpha_out (device).
+ * For weights the paper computes alpha once and freezes it (Sec. 3.2); for
+ * dynamically quantized activations it is recomputed on every call.
+ * ws: device scratch of at least focus_workspace_bytes(desc, FOCUS_WS_ALPHA)
+ * bytes, 16-byte aligned; its contents are overwritten.  desc->fmt, block and
+ * sub_block are not used. */
+int focus_nvfp4_alpha(const focus_desc_t* desc, const void* x, float* alpha_out,
+                      void* ws, size_t ws_bytes, focus_stream_t stream);
+
+/* Fake-quantization forward, Eq. 1-3 and 6-8: y = Q_E2M1(x / S^q) * S^dq.
+ * x      [rows, ld] input (read only).
+ * crs    CRS coefficients c_i, or NULL for 1 (Eq. 6-7).
+ * dgs    DGS coefficients c_i^k, or NULL for 1 (Eq. 8).
+ * alpha  NVFP4: device pointer to the fp32 per-tensor scale (required);
+ *        MXFP4: ignored (may be NULL).
+ * y      [rows, ld] output in dtype (may alias nothing else).
+ * scale_bytes  optional [rows, cols/block] output of the stored scale bytes. */
+int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
+                 const float* dgs, const float* alpha, void* y, uint8_t* scale_bytes,
+                 focus_stream_t stream);
+
+/* Straight-through-estimator backward (Sec. 3.2) of focus_fq_fwd.
+ * g      [rows, ld] upstream gradient dL/dy (dtype).
+ * gx     optional [rows, ld] output dL/dx = mask * fl(fl(g * S^dq) / S^q);
+ *        NULL skips it (frozen weights, Sec. 3.2).
+ * gcrs   optional dL/dc_i    = -sum_k T_ik * c_i^k / (c_i c_i^k)^2
+ * gdgs   optional dL/dc_i^k  = -T_ik * c_i / (c_i c_i^k)^2
+ *        with T_ik = sum over sub-block (i,k) of mask * g * x; in shared mode
+ *        both are also summed over rows.  They are written (not accumulated).
+ *        Requesting gcrs with crs == NULL gives the gradient at c_i = 1
+ *        (likewise gdgs with dgs == NULL).
+ * ws     device scratch of focus_workspace_bytes(desc, FOCUS_WS_BWD) bytes
+ *        (zero when coef_shared_rows == 0, in which case ws may be NULL).
+ * Coefficient gradients are computed with compensated (double-fp32)
+ * arithmetic and match an exact evaluation to about 1e-5 relative. */
+int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,
+                 const float* dgs, const float* alpha, const void* g, void* gx,
+                 float* gcrs, float* gdgs, void* ws, size_t ws_bytes,
+                 focus_stream_t stream);
+
+/* Export (Fig. 3(d)): the FP4 codes of Q_E2M1(x / S^q) and the scale bytes
+ * of S^dq -- what the deployed MXFP4 / NVFP4 model stores; S^q and the
+ * coefficients are not part of it.  NVFP4 also needs the caller's alpha.
+ * codes        [rows, cols/2] uint8 output (required).
+ * scale_bytes  [rows, cols/block] uint8 output (required). */
+int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
+               const float* dgs, const float* alpha, uint8_t* codes,
+               uint8_t* scale_bytes, focus_stream_t stream);
+
+/* Device scratch (bytes) that focus_nvfp4_alpha (which = FOCUS_WS_ALPHA) or
+ * focus_fq_bwd (which = FOCUS_WS_BWD) needs for this descriptor on the
+ * current device; 0 for an invalid descriptor. */
+size_t focus_workspace_bytes(const focus_desc_t* desc, int which);
+
+/* Static, NUL-terminated description of a status code. */
+const char* focus_status_string(int status);
+
+/* ABI version of this library (major * 100 + minor). */
+int focus_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FOCUS_FQ_H */

@@ -1,0 +1,240 @@
+"""CPU oracle for the FOCUS FP4 fake-quantizer -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The product path (the CUDA library
+under ``paper_2608_01847_gb300``) never imports it and shares no code with it.
+
+The arithmetic lives in ``focus_oracle.c`` (plain scalar C, binary32 forward,
+binary64 compensated gradient sums; see that file's header for the equations
+it follows: FOCUS Sec. 3.1 Eq. 1-3, Sec. 3.2 Eq. 4-5, Sec. 3.3 Eq. 6-7,
+Sec. 3.4 Eq. 8, Fig. 3(d)).  This module only builds it with gcc and marshals
+numpy arrays into it.
+
+Dtype codes: 0 = float32, 1 = bfloat16 (stored as uint16 bit patterns).
+Format codes: 0 = MXFP4 (block 32, E8M0), 1 = NVFP4 (block 16, E4M3 + alpha).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "focus_oracle.c")
+_LIB = os.path.join(_HERE, "_build", "libfocus_oracle.so")
+
+MXFP4, NVFP4 = 0, 1
+F32, BF16 = 0, 1
+STE_IDENTITY, STE_CLIPPED = 0, 1
+MX_CEIL, MX_FLOOR = 0, 1
+
+# -ffp-contract=off: no fused multiply-add may merge two binary32 roundings
+# (GCC contracts by default on aarch64); no fast-math so IEEE semantics hold.
+CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def build(force: bool = False) -> str:
+    """Compile focus_oracle.c into ``_build/libfocus_oracle.so`` (idempotent)."""
+    os.makedirs(os.path.dirname(_LIB), exist_ok=True)
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", *CFLAGS, _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        build()
+        L = ctypes.CDLL(_LIB)
+        i64, i32, p, f = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p, ctypes.c_float
+        L.focus_oracle_alpha.argtypes = [i32, i64, i64, i64, p, p]
+        L.focus_oracle_fwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32,
+                                       p, p, p, f, p, p, p]
+        L.focus_oracle_bwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32, i32,
+                                       p, p, p, f, p, p, p, p, p, p]
+        L.focus_oracle_dequant.argtypes = [i32, i32, i64, i64, i32, p, p, f, p]
+        L.focus_oracle_e2m1_code.argtypes = [f]
+        L.focus_oracle_e2m1_value.argtypes = [i32]
+        L.focus_oracle_e2m1_value.restype = f
+        L.focus_oracle_e4m3_decode.argtypes = [ctypes.c_uint8]
+        L.focus_oracle_e4m3_decode.restype = f
+        L.focus_oracle_e4m3_encode.argtypes = [f]
+        L.focus_oracle_e4m3_encode.restype = ctypes.c_uint8
+        L.focus_oracle_e8m0_exponent.argtypes = [f, i32]
+        L.focus_oracle_bf16_rne.argtypes = [f]
+        L.focus_oracle_bf16_rne.restype = ctypes.c_uint16
+        L.focus_oracle_e2m1_codes.argtypes = [p, i64, p]
+        L.focus_oracle_e4m3_encodes.argtypes = [p, i64, p]
+        L.focus_oracle_e8m0_exponents.argtypes = [p, i64, i32, p]
+        L.focus_oracle_bf16_rnes.argtypes = [p, i64, p]
+        _lib = L
+    return _lib
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def _check(rc):
+    if rc == -1:
+        raise OracleError("oracle: invalid argument")
+    if rc == -2:
+        raise OracleError("oracle: precondition violated (non-finite input or coefficient <= 0)")
+    if rc != 0:
+        raise OracleError(f"oracle: status {rc}")
+
+
+def _dtype_code(x: np.ndarray) -> int:
+    if x.dtype == np.float32:
+        return F32
+    if x.dtype == np.uint16:
+        return BF16
+    raise TypeError("oracle inputs are float32 or uint16 (bfloat16 bit patterns)")
+
+
+def _c32(a):
+    return None if a is None else np.ascontiguousarray(a, dtype=np.float32)
+
+
+def default_block(fmt: int) -> int:
+    return 32 if fmt == MXFP4 else 16
+
+
+# --------------------------------------------------------------------------
+# codecs, one value or a vector at a time
+# --------------------------------------------------------------------------
+def e2m1_codes(u) -> np.ndarray:
+    u = np.ascontiguousarray(u, dtype=np.float32)
+    out = np.empty(u.shape, np.uint8)
+    lib().focus_oracle_e2m1_codes(_ptr(u), u.size, _ptr(out))
+    return out
+
+
+def e2m1_value(code: int) -> float:
+    return lib().focus_oracle_e2m1_value(int(code))
+
+
+def e4m3_decode(byte: int) -> float:
+    return lib().focus_oracle_e4m3_decode(int(byte))
+
+
+def e4m3_encode(r) -> np.ndarray:
+    r = np.ascontiguousarray(r, dtype=np.float32)
+    out = np.empty(r.shape, np.uint8)
+    lib().focus_oracle_e4m3_encodes(_ptr(r), r.size, _ptr(out))
+    return out
+
+
+def e8m0_exponent(m, rule: int = MX_CEIL) -> np.ndarray:
+    m = np.ascontiguousarray(m, dtype=np.float32)
+    out = np.empty(m.shape, np.int32)
+    lib().focus_oracle_e8m0_exponents(_ptr(m), m.size, int(rule), _ptr(out))
+    return out
+
+
+def bf16_rne(f) -> np.ndarray:
+    f = np.ascontiguousarray(f, dtype=np.float32)
+    out = np.empty(f.shape, np.uint16)
+    lib().focus_oracle_bf16_rnes(_ptr(f), f.size, _ptr(out))
+    return out
+
+
+# --------------------------------------------------------------------------
+# tensor-level entry points
+# --------------------------------------------------------------------------
+def alpha(x: np.ndarray) -> float:
+    """NVFP4 per-tensor scale alpha = fl(max|x| / 2688) (Eq. 2)."""
+    x = np.ascontiguousarray(x)
+    rows, cols = x.shape
+    out = np.zeros(1, np.float32)
+    _check(lib().focus_oracle_alpha(_dtype_code(x), rows, cols, cols, _ptr(x), _ptr(out)))
+    return float(out[0])
+
+
+def fwd(x, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
+        mx_rule=MX_CEIL, want_y=True, want_scales=True, want_codes=False):
+    """Fake-quant forward / export (Eq. 1-8, Fig. 3(d)).
+
+    x: [rows, cols] float32 or uint16 (bf16 bits), contiguous.
+    Returns dict with 'y' (same dtype as x), 'scales' uint8 [rows, cols/block],
+    'codes' uint8 [rows, cols/2] (as requested)."""
+    x = np.ascontiguousarray(x)
+    rows, cols = x.shape
+    block = block or default_block(fmt)
+    crs, dgs = _c32(crs), _c32(dgs)
+    out = {}
+    y = np.empty_like(x) if want_y else None
+    sc = np.zeros((rows, cols // block), np.uint8) if want_scales else None
+    cd = np.zeros((rows, cols // 2), np.uint8) if want_codes else None
+    _check(lib().focus_oracle_fwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
+                                  int(bool(shared)), mx_rule, _ptr(x), _ptr(crs), _ptr(dgs),
+                                  float(alpha), _ptr(y), _ptr(sc), _ptr(cd)))
+    if want_y:
+        out["y"] = y
+    if want_scales:
+        out["scales"] = sc
+    if want_codes:
+        out["codes"] = cd
+    return out
+
+
+def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
+        ste=STE_IDENTITY, mx_rule=MX_CEIL, want_gx=True, want_gcrs=True, want_gdgs=True,
+        want_abs=False):
+    """STE backward (Sec. 3.2; Eq. 6-8): input gradient and coefficient gradients.
+
+    Returns dict with 'gx' (dtype of x), 'gcrs' float32 [rows or 1, cols/block],
+    'gdgs' float32 [rows or 1, cols/sub], and with want_abs the binary64
+    term-magnitude sums 'gcrs_abs', 'gdgs_abs' of the same shapes."""
+    x = np.ascontiguousarray(x)
+    g = np.ascontiguousarray(g)
+    assert g.dtype == x.dtype and g.shape == x.shape
+    rows, cols = x.shape
+    block = block or default_block(fmt)
+    crs, dgs = _c32(crs), _c32(dgs)
+    crow = 1 if shared else rows
+    gx = np.empty_like(x) if want_gx else None
+    gc = np.zeros((crow, cols // block), np.float32) if want_gcrs else None
+    gd = np.zeros((crow, cols // sub), np.float32) if want_gdgs else None
+    gca = np.zeros((crow, cols // block), np.float64) if (want_abs and want_gcrs) else None
+    gda = np.zeros((crow, cols // sub), np.float64) if (want_abs and want_gdgs) else None
+    _check(lib().focus_oracle_bwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
+                                  int(bool(shared)), ste, mx_rule, _ptr(x), _ptr(crs),
+                                  _ptr(dgs), float(alpha), _ptr(g), _ptr(gx), _ptr(gc),
+                                  _ptr(gd), _ptr(gca), _ptr(gda)))
+    out = {}
+    if want_gx:
+        out["gx"] = gx
+    if want_gcrs:
+        out["gcrs"] = gc
+        if want_abs:
+            out["gcrs_abs"] = gca
+    if want_gdgs:
+        out["gdgs"] = gd
+        if want_abs:
+            out["gdgs_abs"] = gda
+    return out
+
+
+def dequant(codes, scales, fmt, alpha=0.0, block=None, dtype=F32):
+    """Rebuild values from an export (codes + scale bytes [+ alpha])."""
+    codes = np.ascontiguousarray(codes, dtype=np.uint8)
+    scales = np.ascontiguousarray(scales, dtype=np.uint8)
+    rows = codes.shape[0]
+    cols = codes.shape[1] * 2
+    block = block or default_block(fmt)
+    y = np.empty((rows, cols), np.float32 if dtype == F32 else np.uint16)
+    _check(lib().focus_oracle_dequant(fmt, dtype, rows, cols, block, _ptr(codes),
+                                      _ptr(scales), float(alpha), _ptr(y)))
+    return y

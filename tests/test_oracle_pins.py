@@ -1,0 +1,492 @@
+"""Pins for the CPU oracle (no GPU).
+
+Each test ties the oracle to something other than itself: values worked by
+hand from the paper's definitions, library conversions (torch float8 /
+bfloat16), brute-force or independent numpy formulations, invariants the
+paper states, and finite differences of the STE surrogate.  A plausible slip
+in the oracle (dropped term, sign, index, transposed operand, off-by-one in an
+exponent rule, wrong tie rule) fails at least one of them.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2608_01847_gb300 import workloads as W
+
+
+def f32(a):
+    return np.asarray(a, dtype=np.float32)
+
+
+# ---------------------------------------------------------------------------
+# independent numpy restatements used only as pins
+# ---------------------------------------------------------------------------
+def e2m1_ref(u):
+    """E2M1 round-to-nearest-even by spacing: 0.5 below 2, 1 in [2,4), 2 from
+    4, saturated at 6; np.round rounds half to even, which on each spacing is
+    the even E2M1 code.  Returns signed float64 values."""
+    u = np.asarray(u, dtype=np.float64)
+    a = np.abs(u)
+    q = np.where(a < 2, np.round(a * 2) / 2, np.where(a < 4, np.round(a), 2 * np.round(a / 2)))
+    q = np.minimum(q, 6.0)
+    return np.copysign(q, u)
+
+
+GRID = np.array([0, 0.5, 1, 1.5, 2, 3, 4, 6], np.float64)
+
+
+def code_to_value(code):
+    code = np.asarray(code).astype(np.int64)
+    mag = GRID[code & 7]
+    return np.where(code & 8, -mag, mag)
+
+
+def e8m0_ceil_ref(m):
+    """Smallest e with fl(m/6) <= 2^e, clamped to [-127, 127]."""
+    m = f32(m)
+    t = (m / np.float32(6)).astype(np.float32)
+    out = np.full(m.shape, -127, np.int64)
+    nz = t > 0
+    out[nz] = np.ceil(np.log2(t[nz].astype(np.float64))).astype(np.int64)
+    return np.clip(out, -127, 127)
+
+
+def e8m0_floor_ref(m):
+    m = f32(m)
+    out = np.full(m.shape, -127, np.int64)
+    nz = m > 0
+    mant, ex = np.frexp(m[nz].astype(np.float64))   # m = mant * 2^ex, mant in [0.5,1)
+    out[nz] = (ex - 1) - 2
+    return np.clip(out, -127, 127)
+
+
+def torch_e4m3(r):
+    return torch.from_numpy(f32(r)).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+
+
+def torch_bf16_bits(f):
+    return torch.from_numpy(f32(f)).to(torch.bfloat16).view(torch.int16).numpy().astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# hand-worked blocks (computed by hand from Eq. 1-3, 6-7)
+# ---------------------------------------------------------------------------
+def test_hand_mxfp4_block_crs():
+    # m = 1.5 -> fl(1.5/6) = 0.25 = 2^-2 -> e = -2, E8M0 byte 125 (0x7D), S^dq = 0.25
+    x = np.zeros((1, 32), np.float32)
+    x[0, :4] = [0.7, -0.26, 0.13, 1.5]
+    out = O.fwd(x, O.MXFP4, want_codes=True)
+    assert out["scales"][0, 0] == 0x7D
+    # c = 1: u = [2.8, -1.04, 0.52, 6.0] -> codes [5, 0xA, 1, 7], y = [0.75, -0.25, 0.125, 1.5]
+    assert list(out["codes"][0, :2]) == [0xA5, 0x71]
+    assert np.all(out["codes"][0, 2:] == 0)
+    assert list(out["y"][0, :4]) == [0.75, -0.25, 0.125, 1.5]
+    assert np.all(out["y"][0, 4:] == 0)
+    # c = 1.25: S^q = 0.3125, u = [2.24, -0.832, 0.416, 4.8] -> codes [4, 0xA, 1, 6]
+    crs = np.array([[1.25]], np.float32)
+    out = O.fwd(x, O.MXFP4, crs=crs, want_codes=True)
+    assert out["scales"][0, 0] == 0x7D            # S^dq is unchanged by c
+    assert list(out["codes"][0, :2]) == [0xA4, 0x61]
+    assert list(out["y"][0, :4]) == [0.5, -0.25, 0.125, 1.0]
+    # STE backward with g = 1 on the first four: gx = fl(fl(1*0.25)/0.3125) = fl(0.8)
+    g = np.zeros_like(x)
+    g[0, :4] = 1
+    b = O.bwd(x, g, O.MXFP4, crs=crs)
+    assert np.all(b["gx"][0, :4] == np.float32(0.25) / np.float32(0.3125))
+    assert np.all(b["gx"][0, 4:] == 0)
+    # dL/dc = -(0.7 - 0.26 + 0.13 + 1.5) / 1.25^2 = -1.3248 (inputs as float32)
+    expect = -(float(np.float32(0.7)) + float(np.float32(-0.26)) + float(np.float32(0.13)) + 1.5) / 1.5625
+    assert b["gcrs"][0, 0] == pytest.approx(expect, rel=1e-7)
+    assert expect == pytest.approx(-1.3248, abs=1e-6)
+
+
+def test_hand_mxfp4_ties():
+    # S^q = 0.25 (m = 1.5): 0.625 -> u = 2.5 (tie 2|3 -> 2, code 4); 1.25 -> 5
+    # (tie 4|6 -> 4, code 6); 0.0625 -> 0.25 (tie 0|0.5 -> 0); -0.0625 -> -0 (0x8)
+    x = np.zeros((1, 32), np.float32)
+    x[0, :6] = [1.5, 0.625, 1.25, 0.0625, -0.0625, 0.1875]
+    out = O.fwd(x, O.MXFP4, want_codes=True)
+    codes = [(out["codes"][0, i // 2] >> (4 * (i % 2))) & 15 for i in range(6)]
+    # 0.1875 -> u = 0.75 (tie 0.5|1 -> 1.0, code 2)
+    assert codes == [7, 4, 6, 0, 8, 2]
+    y = out["y"][0, :6]
+    assert list(y) == [1.5, 0.5, 1.0, 0.0, 0.0, 0.25]
+    assert not np.signbit(y[3]) and np.signbit(y[4])   # -0 kept for the negative tie
+
+
+def test_hand_nvfp4_blocks():
+    # amax = 0.65625 = 21/32 and 2688 = 21 * 128 -> alpha = 2^-12 exactly
+    x = np.zeros((1, 32), np.float32)
+    x[0, 0] = 0.65625
+    x[0, 16] = 0.1
+    a = O.alpha(x)
+    assert a == 2.0 ** -12
+    out = O.fwd(x, O.NVFP4, alpha=a, want_codes=True)
+    # block 0: r = 0.65625 / (6 * 2^-12) = 448 -> E4M3 0x7E, S^dq = 448 * 2^-12
+    assert out["scales"][0, 0] == 0x7E
+    assert out["y"][0, 0] == np.float32(0.65625)
+    # block 1: r = fl(0.1 / (6 * 2^-12)) = 68.27 -> nearest E4M3 is 72 (0x69),
+    # S^dq = 72 * 2^-12 = 0.017578125, u = 0.1 / S^dq = 5.69 -> 6 (code 7)
+    assert out["scales"][0, 1] == 0x69
+    assert out["codes"][0, 8] & 15 == 7
+    assert out["y"][0, 16] == np.float32(6 * 0.017578125)
+
+
+def test_alpha_closed_form():
+    for k in (-20, -3, 0, 5):
+        x = np.zeros((3, 16), np.float32)
+        x[1, 7] = -2688.0 * 2.0 ** k
+        assert O.alpha(x) == 2.0 ** k
+    assert O.alpha(np.zeros((2, 16), np.float32)) == 0.0
+
+
+# ---------------------------------------------------------------------------
+# format codecs against libraries / brute force
+# ---------------------------------------------------------------------------
+def test_e4m3_decode_matches_torch():
+    b = np.arange(256, dtype=np.uint8)
+    ref = torch.from_numpy(b).view(torch.float8_e4m3fn).float().numpy()
+    ours = np.array([O.e4m3_decode(int(i)) for i in b], np.float32)
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(ours), nan) and nan.sum() == 2   # 0x7F, 0xFF
+    assert np.array_equal(ours[~nan].view(np.uint32), ref[~nan].view(np.uint32))
+
+
+def _near_boundaries(hi_max):
+    """Every float32 whose upper 16 bits are <= hi_max and whose lower 16 bits
+    are one of a few patterns around 0 and 0x8000: this hits every E4M3 (and
+    bf16) rounding midpoint and its neighbours one ulp away."""
+    hi = np.arange(0, hi_max + 1, dtype=np.uint32) << 16
+    lo = np.array([0x0000, 0x0001, 0x0002, 0x7FFF, 0x8000, 0x8001, 0xFFFE, 0xFFFF], np.uint32)
+    return (hi[:, None] | lo[None, :]).reshape(-1).view(np.float32)
+
+
+def test_e4m3_encode_matches_torch_rne():
+    r = _near_boundaries(0x43E7)                      # up to ~463.9 (midpoint 448|480 is 464)
+    r = r[np.isfinite(r) & (r < 464.0)]
+    rng = np.random.default_rng(7)
+    r = np.concatenate([r, rng.uniform(0, 463.9, 200000).astype(np.float32)])
+    assert np.array_equal(O.e4m3_encode(r), torch_e4m3(r))
+
+
+def test_e4m3_saturates():
+    big = f32([448.0, 464.0, 470.0, 1e4, 3e38, np.inf])
+    assert np.all(O.e4m3_encode(big) == 0x7E)
+
+
+def test_e2m1_matches_independent_rounding():
+    rng = np.random.default_rng(11)
+    mids = np.array([0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0, 6.0], np.float32)
+    near = np.concatenate([np.nextafter(mids, np.float32(0)), mids, np.nextafter(mids, np.float32(9))])
+    u = np.concatenate([rng.uniform(-8, 8, 400000).astype(np.float32),
+                        near, -near, f32([0.0, -0.0, 7.9, -100.0, 1e30])])
+    codes = O.e2m1_codes(u)
+    ref = e2m1_ref(u)
+    got = code_to_value(codes)
+    assert np.array_equal(got, ref)
+    # sign bit is the sign of u, also when the value rounds to zero
+    assert np.array_equal((codes >> 3).astype(bool), np.signbit(u))
+
+
+def test_e2m1_brute_force_grid():
+    """Tiny blocks: each code is the argmin over all 15 signed E2M1 values."""
+    vals = np.array(sorted(set(list(GRID) + list(-GRID))), np.float64)
+    rng = np.random.default_rng(3)
+    u = rng.uniform(-7, 7, 20000).astype(np.float32)
+    codes = O.e2m1_codes(u)
+    d = np.abs(u[:, None].astype(np.float64) - vals[None, :])
+    best = vals[np.argmin(d, axis=1)]
+    got = code_to_value(codes)
+    not_tie = np.sort(d, axis=1)[:, 1] > np.sort(d, axis=1)[:, 0]
+    assert np.array_equal(got[not_tie], best[not_tie])
+    assert np.all(np.abs(got - u) <= np.min(d, axis=1) + 0.0)
+
+
+def test_e8m0_ceil_and_floor_rules():
+    rng = np.random.default_rng(5)
+    pieces = []
+    for e in range(-150, 126):                        # around 6 * 2^e for every e
+        base = np.float32(6.0) * np.float32(2.0) ** np.float32(e) if e > -150 else np.float32(0)
+        if not np.isfinite(base) or base == 0:
+            continue
+        pieces.append(np.array([base, np.nextafter(base, np.float32(0)),
+                                np.nextafter(base, np.float32(np.inf))], np.float32))
+        pieces.append(np.float32(2.0) ** np.float32(e) * f32([1, 1.5, 1.9999999]))
+    subn = np.arange(1, 5000, dtype=np.uint32).view(np.float32)
+    rand = rng.integers(1, 0x7F800000, 2_000_000, dtype=np.uint32).view(np.float32)
+    m = np.concatenate(pieces + [subn, rand, f32([0.0, 3.4e38])])
+    m = m[np.isfinite(m) & (m >= 0)]
+    assert np.array_equal(O.e8m0_exponent(m, O.MX_CEIL), e8m0_ceil_ref(m))
+    assert np.array_equal(O.e8m0_exponent(m, O.MX_FLOOR), e8m0_floor_ref(m))
+
+
+def test_e8m0_ceil_never_saturates():
+    """Under the ceiling rule the block maximum never exceeds 6 * 2^e, so at
+    c = 1 no element saturates; and 2^e is the tightest such power."""
+    rng = np.random.default_rng(9)
+    m = rng.integers(0x00800000, 0x7F000000, 1_000_000, dtype=np.uint32).view(np.float32)
+    e = O.e8m0_exponent(m, O.MX_CEIL).astype(np.float64)
+    ok = e < 127
+    ratio = m[ok].astype(np.float64) / np.exp2(e[ok])
+    assert np.all(ratio <= 6.0)
+    inner = ok & (e > -127)
+    assert np.all(m[inner].astype(np.float64) / np.exp2(e[inner] - 1) > 6.0)
+
+
+def test_bf16_rne_matches_torch():
+    r = _near_boundaries(0xFFFF)
+    r = r[np.isfinite(r)]
+    rng = np.random.default_rng(13)
+    r = np.concatenate([r, rng.standard_normal(100000).astype(np.float32),
+                        f32([3.4e38, -3.4e38, 1e-45, -1e-45])])
+    assert np.array_equal(O.bf16_rne(r), torch_bf16_bits(r))
+
+
+# ---------------------------------------------------------------------------
+# invariants the paper states
+# ---------------------------------------------------------------------------
+def rtn_reference(x, fmt, alpha=0.0, block=None):
+    """Standard MXFP4 / NVFP4 round-to-nearest (Eq. 1-3), written in numpy
+    with torch's float8 conversion for E4M3: the c = 1 baseline."""
+    x = f32(x)
+    block = block or (32 if fmt == O.MXFP4 else 16)
+    rows, cols = x.shape
+    xb = x.reshape(rows, cols // block, block)
+    m = np.abs(xb).max(axis=2)
+    if fmt == O.MXFP4:
+        s = np.exp2(e8m0_ceil_ref(m)).astype(np.float32)
+    else:
+        den = np.float32(alpha) * np.float32(6)
+        with np.errstate(divide="ignore", invalid="ignore"):
+            r = (m / den).astype(np.float32)
+        r = np.where(m == 0, np.float32(0), np.minimum(r, np.float32(448)))
+        delta = torch.from_numpy(torch_e4m3(r)).view(torch.float8_e4m3fn).float().numpy()
+        s = (delta * np.float32(alpha)).astype(np.float32)
+    s3 = s[:, :, None]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        u = (xb / s3).astype(np.float32)
+    q = e2m1_ref(u).astype(np.float32)
+    y = (q * s3).astype(np.float32)
+    y = np.where(s3 == 0, np.float32(0), y)
+    return y.reshape(rows, cols)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_crs_at_one_equals_rtn(fmt):
+    """Starting from c = 1 the method is the baseline (Sec. 3.3): with all
+    coefficients 1 the fake-quant equals standard RTN bit for bit."""
+    w = W.WORKLOADS["w256x512_f32"]
+    x = W.draw_values(w, 64, 512, 42)
+    x[3, 16:32] = 0                                  # an all-zero block
+    x[5, :32] *= 1e-30                               # tiny values (subnormal scales)
+    block = 32 if fmt == O.MXFP4 else 16
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    ones_c = np.ones((64, 512 // block), np.float32)
+    ones_d = np.ones((64, 512 // 8), np.float32)
+    y = O.fwd(x, fmt, crs=ones_c, dgs=ones_d, alpha=a)["y"]
+    ref = rtn_reference(x, fmt, alpha=a)
+    assert np.array_equal(y.view(np.uint32), ref.view(np.uint32))
+    y0 = O.fwd(x, fmt, alpha=a)["y"]
+    assert np.array_equal(y0.view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_dgs_with_block_sized_subblocks_is_crs(fmt):
+    """Sub-block size equal to the block size reduces DGS to CRS (Sec. 3.4,
+    Table 5)."""
+    w = W.WORKLOADS["llama3_8b_block"]
+    x = W.to_bf16_bits(W.draw_values(w, 32, 256, 17))
+    g = W.to_bf16_bits(W.draw_grad(32, 256, 18))
+    block = 32 if fmt == O.MXFP4 else 16
+    coef = W.draw_coefs(w, 32 * 256 // block, 19).reshape(32, -1)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    f_c = O.fwd(x, fmt, crs=coef, alpha=a, sub=block, want_codes=True)
+    f_d = O.fwd(x, fmt, dgs=coef, alpha=a, sub=block, want_codes=True)
+    for k in ("y", "codes", "scales"):
+        assert np.array_equal(f_c[k], f_d[k])
+    b_c = O.bwd(x, g, fmt, crs=coef, alpha=a, sub=block)
+    b_d = O.bwd(x, g, fmt, dgs=coef, alpha=a, sub=block)
+    assert np.array_equal(b_c["gx"], b_d["gx"])
+    assert np.array_equal(b_c["gcrs"], b_d["gdgs"])
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_dequant_of_export_equals_forward(fmt, dtype):
+    """The deployed model (codes + scale bytes, Fig. 3(d)) reproduces the
+    fake-quantized forward output exactly."""
+    w = W.WORKLOADS["w256x512_f32"]
+    x = W.draw_values(w, 40, 512, 23)
+    x[1, :64] = 0
+    crs = W.draw_coefs(w, 40 * 512 // 32, 24).reshape(40, -1)
+    dgs = W.draw_coefs(w, 40 * 512 // 8, 25).reshape(40, -1)
+    if dtype == "bf16":
+        x = W.to_bf16_bits(x)
+    block = 32 if fmt == O.MXFP4 else 16
+    if fmt == O.NVFP4:
+        crs = W.draw_coefs(w, 40 * 512 // 16, 24).reshape(40, -1)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    out = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a, want_codes=True)
+    dq = O.dequant(out["codes"], out["scales"], fmt, alpha=a, block=block,
+                   dtype=O.F32 if dtype == "f32" else O.BF16)
+    assert np.array_equal(dq, out["y"])
+
+
+def test_mxfp4_input_gradient_is_g_at_c1():
+    """With c = 1 and a normal power-of-two S^dq, g * 2^e / 2^e is exact."""
+    w = W.WORKLOADS["w256x512_f32"]
+    x = W.draw_values(w, 16, 512, 31)
+    g = W.draw_grad(16, 512, 32)
+    b = O.bwd(x, g, O.MXFP4)
+    assert np.array_equal(b["gx"], g)
+
+
+# ---------------------------------------------------------------------------
+# gradients: finite differences of the STE surrogate, autograd restatement
+# ---------------------------------------------------------------------------
+def surrogate_loss(x, g, crs, dgs, sdq_mask, block, sub):
+    """Identity-STE surrogate: ytilde = (x / S^q) * S^dq = x / (c_i c_i^k) on
+    live sub-blocks, so L = sum g * x / (c_i c_i^k); evaluated in float64."""
+    rows, cols = x.shape
+    c = np.repeat(crs, block, axis=1)
+    d = np.repeat(dgs, sub, axis=1)
+    return float(np.sum(g * x / (c * d) * sdq_mask))
+
+
+@pytest.mark.parametrize("fmt,sub", [(O.MXFP4, 8), (O.MXFP4, 32), (O.NVFP4, 8), (O.NVFP4, 4)])
+def test_coefficient_gradients_finite_difference(fmt, sub):
+    rng = np.random.default_rng(100 + sub)
+    block = 32 if fmt == O.MXFP4 else 16
+    rows, cols = 3, 2 * block
+    x = rng.standard_normal((rows, cols)).astype(np.float32)
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    crs = rng.uniform(0.8, 1.2, (rows, cols // block)).astype(np.float32)
+    dgs = rng.uniform(0.8, 1.2, (rows, cols // sub)).astype(np.float32)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    b = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a, sub=sub)
+    x64, g64 = x.astype(np.float64), g.astype(np.float64)
+    c64, d64 = crs.astype(np.float64), dgs.astype(np.float64)
+    live = np.ones_like(x64)
+    for arr, grad in ((c64, b["gcrs"]), (d64, b["gdgs"])):
+        for idx in np.ndindex(arr.shape):
+            h = 1e-6 * arr[idx]
+            old = arr[idx]
+            arr[idx] = old + h
+            lp = surrogate_loss(x64, g64, c64, d64, live, block, sub)
+            arr[idx] = old - h
+            lm = surrogate_loss(x64, g64, c64, d64, live, block, sub)
+            arr[idx] = old
+            fd = (lp - lm) / (2 * h)
+            assert grad[idx] == pytest.approx(fd, rel=1e-6, abs=1e-9)
+
+
+def test_shared_row_gradients_sum_over_rows():
+    """Shared coefficients: the gradient is the per-row gradient summed over
+    rows (checked against the oracle's own per-row mode with broadcast
+    coefficients, and against finite differences)."""
+    rng = np.random.default_rng(77)
+    rows, cols, block, sub = 5, 64, 32, 8
+    x = rng.standard_normal((rows, cols)).astype(np.float32)
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    crs = rng.uniform(0.9, 1.1, (1, cols // block)).astype(np.float32)
+    dgs = rng.uniform(0.9, 1.1, (1, cols // sub)).astype(np.float32)
+    sh = O.bwd(x, g, O.MXFP4, crs=crs, dgs=dgs, shared=True)
+    pr = O.bwd(x, g, O.MXFP4, crs=np.repeat(crs, rows, 0), dgs=np.repeat(dgs, rows, 0))
+    assert np.array_equal(sh["gx"], pr["gx"])
+    np.testing.assert_allclose(sh["gcrs"][0], pr["gcrs"].astype(np.float64).sum(0), rtol=1e-6)
+    np.testing.assert_allclose(sh["gdgs"][0], pr["gdgs"].astype(np.float64).sum(0), rtol=1e-6)
+    fw = O.fwd(x, O.MXFP4, crs=crs, dgs=dgs, shared=True)
+    fw2 = O.fwd(x, O.MXFP4, crs=np.repeat(crs, rows, 0), dgs=np.repeat(dgs, rows, 0))
+    assert np.array_equal(fw["y"], fw2["y"])
+
+
+def torch_fake_quant(x, crs, dgs, sdq, block, sub):
+    """PyTorch autograd restatement of y = STE(Q(x / S^q)) * S^dq with
+    S^q = S^dq * (c * c^k): the straight-through trick u + (Q(u) - u).detach()."""
+    rows, cols = x.shape
+    c = crs.repeat_interleave(block, dim=1)
+    d = dgs.repeat_interleave(sub, dim=1)
+    s = sdq.repeat_interleave(block, dim=1)
+    s_q = s * (c * d)
+    u = x / s_q
+    q = torch.from_numpy(e2m1_ref(u.detach().numpy())).to(u.dtype)
+    return (u + (q - u).detach()) * s
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_autograd_restatement(fmt):
+    rng = np.random.default_rng(55)
+    block = 32 if fmt == O.MXFP4 else 16
+    sub = 8
+    rows, cols = 6, 4 * block
+    x = (rng.standard_normal((rows, cols)) * 0.02).astype(np.float32)
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    crs = rng.uniform(0.8, 1.2, (rows, cols // block)).astype(np.float32)
+    dgs = rng.uniform(0.8, 1.2, (rows, cols // sub)).astype(np.float32)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    ours = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a)
+    fw = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a)
+    # S^dq from the scale bytes, as the deployed model rebuilds it
+    sb = fw["scales"].astype(np.int64)
+    if fmt == O.MXFP4:
+        sdq = np.exp2(sb - 127).astype(np.float32)
+    else:
+        dl = torch.from_numpy(fw["scales"]).view(torch.float8_e4m3fn).float().numpy()
+        sdq = (dl * np.float32(a)).astype(np.float32)
+    # float32 autograd: forward values and input gradient bit-identical
+    xt = torch.from_numpy(x).requires_grad_(True)
+    ct = torch.from_numpy(crs).requires_grad_(True)
+    dt = torch.from_numpy(dgs).requires_grad_(True)
+    y = torch_fake_quant(xt, ct, dt, torch.from_numpy(sdq), block, sub)
+    y.backward(torch.from_numpy(g))
+    assert np.array_equal(y.detach().numpy(), fw["y"])
+    assert np.array_equal(xt.grad.numpy(), ours["gx"])
+    # float64 autograd for the coefficient gradients
+    x6 = torch.from_numpy(x.astype(np.float64))
+    c6 = torch.from_numpy(crs.astype(np.float64)).requires_grad_(True)
+    d6 = torch.from_numpy(dgs.astype(np.float64)).requires_grad_(True)
+    y6 = torch_fake_quant(x6, c6, d6, torch.from_numpy(sdq.astype(np.float64)), block, sub)
+    y6.backward(torch.from_numpy(g.astype(np.float64)))
+    np.testing.assert_allclose(ours["gcrs"], c6.grad.numpy(), rtol=1e-5, atol=1e-12)
+    np.testing.assert_allclose(ours["gdgs"], d6.grad.numpy(), rtol=1e-5, atol=1e-12)
+
+
+def test_clipped_ste_masks_saturated():
+    """Clipped STE: no gradient where |x / S^q| > 6 (only possible for c < 1
+    under the ceiling rule)."""
+    x = np.zeros((1, 32), np.float32)
+    x[0, :3] = [1.5, 1.45, 0.1]          # S^dq = 0.25
+    crs = np.array([[0.9]], np.float32)   # S^q = 0.225: 1.5/0.225 = 6.67, 1.45/.225 = 6.44
+    g = np.ones_like(x)
+    b = O.bwd(x, g, O.MXFP4, crs=crs, ste=O.STE_CLIPPED)
+    assert b["gx"][0, 0] == 0 and b["gx"][0, 1] == 0 and b["gx"][0, 2] != 0
+    bi = O.bwd(x, g, O.MXFP4, crs=crs, ste=O.STE_IDENTITY)
+    assert bi["gx"][0, 0] != 0
+    # only element 2 (x = 0.1) plus the zeros contribute: T = 0.1
+    assert b["gcrs"][0, 0] == pytest.approx(-float(np.float32(0.1)) / 0.81, rel=1e-6)
+
+
+def test_nvfp4_all_zero_tensor_is_dead():
+    x = np.zeros((4, 32), np.float32)
+    g = np.ones_like(x)
+    a = O.alpha(x)
+    assert a == 0.0
+    out = O.fwd(x, O.NVFP4, alpha=a, want_codes=True)
+    assert np.all(out["scales"] == 0) and np.all(out["codes"] == 0)
+    assert np.all(out["y"].view(np.uint32) == 0)
+    b = O.bwd(x, g, O.NVFP4, crs=np.ones((4, 2), np.float32), alpha=a)
+    assert np.all(b["gx"].view(np.uint32) == 0) and np.all(b["gcrs"] == 0)
+
+
+def test_oracle_rejects_bad_inputs():
+    x = np.ones((2, 32), np.float32)
+    with pytest.raises(O.OracleError):
+        O.fwd(x, O.MXFP4, crs=np.zeros((2, 1), np.float32))     # c must be > 0
+    x[0, 0] = np.nan
+    with pytest.raises(O.OracleError):
+        O.fwd(x, O.MXFP4)
+    with pytest.raises(O.OracleError):
+        O.fwd(np.ones((2, 30), np.float32), O.MXFP4)            # cols % block
