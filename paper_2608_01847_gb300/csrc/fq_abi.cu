@@ -1,0 +1,240 @@
+// fq_abi.cu -- the extern "C" entry points declared in include/focus_fq.h:
+// argument validation, launch parameters, scratch sizing, error mapping.
+// No allocation, no host synchronisation, no exception crosses the ABI.
+#include <cstdint>
+#include <cstring>
+
+#include "../../include/focus_fq.h"
+#include "fq_launch.h"
+
+#define FOCUS_API extern "C" __attribute__((visibility("default")))
+
+namespace focus {
+
+cudaError_t launch_bwd_mx(int dt, int sub, const KParams& p, cudaStream_t st);
+cudaError_t launch_bwd_nv(int dt, int sub, const KParams& p, cudaStream_t st);
+cudaError_t launch_bwd_shared_mx(int dt, int sub, const KParams& p, uint32_t ny, cudaStream_t st);
+cudaError_t launch_bwd_shared_nv(int dt, int sub, const KParams& p, uint32_t ny, cudaStream_t st);
+
+cudaError_t launch_bwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
+{
+    return fmt == 0 ? launch_bwd_mx(dt, sub, p, st) : launch_bwd_nv(dt, sub, p, st);
+}
+
+cudaError_t launch_bwd_shared(int fmt, int dt, int sub, const KParams& p, uint32_t ny,
+                              cudaStream_t st)
+{
+    return fmt == 0 ? launch_bwd_shared_mx(dt, sub, p, ny, st)
+                    : launch_bwd_shared_nv(dt, sub, p, ny, st);
+}
+
+namespace {
+
+constexpr int64_t kMaxChunks = (int64_t(1) << 31) - 1;
+
+bool misaligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; }
+
+// Shape checks common to every entry point; `method` adds the format,
+// block and sub-block rules (the alpha pass needs only the tensor shape).
+int check_desc(const focus_desc_t* d, bool method)
+{
+    if (!d) return FOCUS_ERR_INVALID_ARG;
+    if (d->rows < 0 || d->cols < 0 || d->ld < d->cols || d->ld < 0) return FOCUS_ERR_INVALID_ARG;
+    if (d->dtype != FOCUS_F32 && d->dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
+    if (d->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
+    if (d->ld % 8 != 0) return FOCUS_ERR_MISALIGNED;
+    if (d->rows > 0 && d->cols > 0 && d->rows > kMaxChunks / (d->cols / 8)) return FOCUS_ERR_UNSUPPORTED;
+    if (!method) return FOCUS_OK;
+    if (d->fmt != FOCUS_MXFP4 && d->fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;
+    if (d->ste != FOCUS_STE_IDENTITY && d->ste != FOCUS_STE_CLIPPED) return FOCUS_ERR_INVALID_ARG;
+    if (d->mx_rule != FOCUS_MX_CEIL && d->mx_rule != FOCUS_MX_FLOOR) return FOCUS_ERR_INVALID_ARG;
+    if (d->coef_shared_rows != 0 && d->coef_shared_rows != 1) return FOCUS_ERR_INVALID_ARG;
+    const int B = d->fmt == FOCUS_MXFP4 ? 32 : 16;
+    if (d->block != B) return FOCUS_ERR_UNSUPPORTED;
+    const int b = d->sub_block;
+    if (b != 2 && b != 4 && b != 8 && b != 16 && b != 32) return FOCUS_ERR_UNSUPPORTED;
+    if (b > B || B % b != 0) return FOCUS_ERR_UNSUPPORTED;
+    if (d->cols % B != 0) return FOCUS_ERR_INVALID_ARG;
+    return FOCUS_OK;
+}
+
+KParams make_params(const focus_desc_t* d)
+{
+    KParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.ld = static_cast<uint64_t>(d->ld);
+    p.cpr = static_cast<uint32_t>(d->cols / 8);
+    p.rows = static_cast<uint32_t>(d->rows);
+    p.n_chunks = static_cast<uint32_t>(d->rows * (d->cols / 8));
+    p.div_cpr = make_fastdiv(p.cpr > 0 ? p.cpr : 1u);
+    p.strided = d->ld != d->cols;
+    p.shared = d->coef_shared_rows;
+    p.ste = d->ste;
+    p.mx_rule = d->mx_rule;
+    return p;
+}
+
+int map_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA; }
+
+// Sub-block size the kernels run with: without DGS coefficients (and without
+// their gradient) every sub-block of a block shares S^q, so one sub-block per
+// block gives identical results.
+int effective_sub(const focus_desc_t* d, const float* dgs, const float* gdgs)
+{
+    return (dgs == nullptr && gdgs == nullptr) ? d->block : d->sub_block;
+}
+
+int check_coef_ptrs(const float* a, const float* b, const float* c, const float* e)
+{
+    if (misaligned(a, 16) || misaligned(b, 16) || misaligned(c, 16) || misaligned(e, 16))
+        return FOCUS_ERR_MISALIGNED;
+    return FOCUS_OK;
+}
+
+size_t bwd_ws_bytes(const focus_desc_t* d)
+{
+    if (!d->coef_shared_rows || d->rows == 0 || d->cols == 0) return 0;
+    const uint32_t cpr = static_cast<uint32_t>(d->cols / 8);
+    const uint32_t ny = shared_row_groups(static_cast<uint32_t>(d->rows), cpr, d->dtype);
+    return static_cast<size_t>(ny) * static_cast<size_t>(d->cols / d->sub_block) * 2 * sizeof(float);
+}
+
+}  // namespace
+}  // namespace focus
+
+using namespace focus;
+
+FOCUS_API int focus_version(void) { return 100; }
+
+FOCUS_API const char* focus_status_string(int status)
+{
+    switch (status) {
+    case FOCUS_OK: return "ok";
+    case FOCUS_ERR_INVALID_ARG: return "invalid argument";
+    case FOCUS_ERR_UNSUPPORTED: return "unsupported block / sub-block / size";
+    case FOCUS_ERR_MISALIGNED: return "misaligned pointer or leading dimension";
+    case FOCUS_ERR_WORKSPACE: return "workspace missing or too small";
+    case FOCUS_ERR_CUDA: return "CUDA runtime error";
+    default: return "unknown status";
+    }
+}
+
+FOCUS_API size_t focus_workspace_bytes(const focus_desc_t* desc, int which)
+{
+    if (which == FOCUS_WS_ALPHA) {
+        if (check_desc(desc, false) != FOCUS_OK) return 0;
+        const uint32_t n = static_cast<uint32_t>(desc->rows * (desc->cols / 8));
+        return static_cast<size_t>(alpha_grid(n)) * sizeof(float);
+    }
+    if (which == FOCUS_WS_BWD) {
+        if (check_desc(desc, true) != FOCUS_OK) return 0;
+        return bwd_ws_bytes(desc);
+    }
+    return 0;
+}
+
+FOCUS_API int focus_nvfp4_alpha(const focus_desc_t* desc, const void* x, float* alpha_out,
+                                void* ws, size_t ws_bytes, focus_stream_t stream)
+{
+    int rc = check_desc(desc, false);
+    if (rc) return rc;
+    const bool empty = desc->rows == 0 || desc->cols == 0;
+    if (!alpha_out || (!empty && !x)) return FOCUS_ERR_INVALID_ARG;
+    if (misaligned(x, 16) || misaligned(alpha_out, 4) || misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
+    KParams p = make_params(desc);
+    const size_t need = static_cast<size_t>(alpha_grid(p.n_chunks)) * sizeof(float);
+    if (!empty && (!ws || ws_bytes < need)) return FOCUS_ERR_WORKSPACE;
+    p.x = x;
+    p.ws = static_cast<float*>(ws);
+    return map_cuda(launch_alpha(desc->dtype, p, alpha_out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
+                           const float* dgs, const float* alpha, void* y, uint8_t* scale_bytes,
+                           focus_stream_t stream)
+{
+    int rc = check_desc(desc, true);
+    if (rc) return rc;
+    if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
+    if (!x || !y || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
+    if (misaligned(x, 16) || misaligned(y, 16) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
+    KParams p = make_params(desc);
+    p.x = x;
+    p.y = y;
+    p.crs = crs;
+    p.dgs = dgs;
+    p.alpha = alpha;
+    p.scales = scale_bytes;
+    return map_cuda(launch_fwd(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p,
+                               reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
+                         const float* dgs, const float* alpha, uint8_t* codes,
+                         uint8_t* scale_bytes, focus_stream_t stream)
+{
+    int rc = check_desc(desc, true);
+    if (rc) return rc;
+    if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
+    if (!x || !codes || !scale_bytes || (desc->fmt == FOCUS_NVFP4 && !alpha))
+        return FOCUS_ERR_INVALID_ARG;
+    if (misaligned(x, 16) || misaligned(codes, 4) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
+    KParams p = make_params(desc);
+    p.x = x;
+    p.crs = crs;
+    p.dgs = dgs;
+    p.alpha = alpha;
+    p.codes = codes;
+    p.scales = scale_bytes;
+    return map_cuda(launch_pack(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p,
+                                reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,
+                           const float* dgs, const float* alpha, const void* g, void* gx,
+                           float* gcrs, float* gdgs, void* ws, size_t ws_bytes,
+                           focus_stream_t stream)
+{
+    int rc = check_desc(desc, true);
+    if (rc) return rc;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const bool want_T = gcrs != nullptr || gdgs != nullptr;
+    if (misaligned(x, 16) || misaligned(g, 16) || misaligned(gx, 16) || misaligned(alpha, 4))
+        return FOCUS_ERR_MISALIGNED;
+    if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
+    if (desc->rows == 0 || desc->cols == 0) {
+        // shared-row gradients of an empty row set are sums over nothing: zero
+        if (desc->coef_shared_rows && desc->cols > 0) {
+            cudaError_t e = cudaSuccess;
+            if (gcrs) e = cudaMemsetAsync(gcrs, 0, sizeof(float) * (desc->cols / desc->block), st);
+            if (e == cudaSuccess && gdgs)
+                e = cudaMemsetAsync(gdgs, 0, sizeof(float) * (desc->cols / desc->sub_block), st);
+            return map_cuda(e);
+        }
+        return FOCUS_OK;
+    }
+    if (!x || !g || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
+    if (!gx && !want_T) return FOCUS_OK;
+    KParams p = make_params(desc);
+    p.x = x;
+    p.g = g;
+    p.gx = gx;
+    p.crs = crs;
+    p.dgs = dgs;
+    p.alpha = alpha;
+    p.gcrs = gcrs;
+    p.gdgs = gdgs;
+    const int sub = effective_sub(desc, dgs, gdgs);
+    if (desc->coef_shared_rows && want_T) {
+        const size_t need = bwd_ws_bytes(desc);
+        if (!ws || ws_bytes < need) return FOCUS_ERR_WORKSPACE;
+        if (misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
+        p.ws = static_cast<float*>(ws);
+        p.nsub = static_cast<uint32_t>(desc->cols / sub);
+        const uint32_t ny = shared_row_groups(p.rows, p.cpr, desc->dtype);
+        return map_cuda(launch_bwd_shared(desc->fmt, desc->dtype, sub, p, ny, st));
+    }
+    return map_cuda(launch_bwd(desc->fmt, desc->dtype, sub, p, st));
+}

@@ -1,0 +1,44 @@
+// Export (pack) kernels and the NVFP4 per-tensor alpha pass.
+#include "fq_launch.h"
+
+namespace focus {
+
+// One CTA: max of the per-CTA partial maxima, alpha = fl(amax / 2688) (Eq. 2).
+__global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* partials, uint32_t n,
+                                                               float* alpha_out)
+{
+    __shared__ float red[kThreads / 32];
+    float m = 0.0f;
+    for (uint32_t i = threadIdx.x; i < n; i += kThreads) m = fmaxf(m, partials[i]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        m = (threadIdx.x < kThreads / 32) ? red[threadIdx.x] : 0.0f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, o));
+        if (threadIdx.x == 0) *alpha_out = __fdiv_rn(m, 2688.0f);  // M_FP4 * M_FP8
+    }
+}
+
+cudaError_t launch_pack(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
+{
+    if (fmt == 0) return dt ? linear_by_sub<0, 1, kPack>(sub, p, st) : linear_by_sub<0, 0, kPack>(sub, p, st);
+    return dt ? linear_by_sub<1, 1, kPack>(sub, p, st) : linear_by_sub<1, 0, kPack>(sub, p, st);
+}
+
+cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_t st)
+{
+    const uint32_t grid = alpha_grid(p.n_chunks);
+    if (p.n_chunks > 0) {
+        if (dt) alpha_partial_kernel<1><<<grid, kThreads, 0, st>>>(p);
+        else alpha_partial_kernel<0><<<grid, kThreads, 0, st>>>(p);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    alpha_final_kernel<<<1, kThreads, 0, st>>>(p.ws, p.n_chunks > 0 ? grid : 0u, alpha_out);
+    return cudaGetLastError();
+}
+
+}  // namespace focus

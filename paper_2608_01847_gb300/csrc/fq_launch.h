@@ -1,0 +1,100 @@
+// fq_launch.h -- host-side launch helpers shared by the C-ABI layer and the
+// kernel instantiation units (internal; not part of the public ABI).
+#pragma once
+
+#include <algorithm>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "fq_kernels.cuh"
+
+namespace focus {
+
+// Streaming multiprocessors of the current device (cached per device id).
+inline int device_sms()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+    if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+// CTAs of the alpha pass and of the shared-row backward's row groups: a
+// fixed multiple of the SM count, so scratch sizes are a pure function of the
+// descriptor and the device.
+constexpr int kCtasPerSm = 8;
+
+inline uint32_t alpha_grid(uint32_t n_chunks)
+{
+    const uint32_t span = 4u * kThreads;
+    const uint64_t need = (static_cast<uint64_t>(n_chunks) + span - 1) / span;
+    const uint64_t cap = static_cast<uint64_t>(device_sms()) * kCtasPerSm;
+    return static_cast<uint32_t>(std::max<uint64_t>(1, std::min(need, cap)));
+}
+
+inline uint32_t shared_col_ctas(uint32_t cpr) { return (cpr + kThreads - 1) / kThreads; }
+
+inline uint32_t shared_row_groups(uint32_t rows, uint32_t cpr, int dtype)
+{
+    const uint32_t u = dtype == 1 ? 2u : 1u;
+    const uint64_t need = (static_cast<uint64_t>(rows) + u - 1) / u;
+    const uint64_t cap = std::max<uint64_t>(
+        1, static_cast<uint64_t>(device_sms()) * kCtasPerSm / shared_col_ctas(cpr));
+    return static_cast<uint32_t>(std::max<uint64_t>(1, std::min<uint64_t>({need, cap, 65535})));
+}
+
+// Grid of a grid-stride streaming kernel: enough CTAs for the work, at most
+// what is resident at once on the device.
+template <typename Kern>
+inline uint32_t stream_grid(Kern kern, int& occ_cache, uint32_t n_chunks, uint32_t span)
+{
+    if (occ_cache <= 0) {
+        int o = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, kern, kThreads, 0) != cudaSuccess || o <= 0) o = 1;
+        occ_cache = o;
+    }
+    const uint64_t need = (static_cast<uint64_t>(n_chunks) + span - 1) / span;
+    const uint64_t cap = static_cast<uint64_t>(device_sms()) * occ_cache;
+    return static_cast<uint32_t>(std::max<uint64_t>(1, std::min(need, cap)));
+}
+
+template <int FMT, int DT, int SUB, int MODE>
+cudaError_t run_linear(const KParams& p, cudaStream_t st)
+{
+    static int occ = 0;
+    auto kern = fq_linear_kernel<FMT, DT, SUB, MODE>;
+    const uint32_t grid = stream_grid(kern, occ, p.n_chunks, Unroll<DT, MODE>::U * kThreads);
+    kern<<<grid, kThreads, 0, st>>>(p);
+    return cudaGetLastError();
+}
+
+// Dispatch over the sub-block size for one (format, dtype, mode).
+template <int FMT, int DT, int MODE>
+cudaError_t linear_by_sub(int sub, const KParams& p, cudaStream_t st)
+{
+    switch (sub) {
+    case 2: return run_linear<FMT, DT, 2, MODE>(p, st);
+    case 4: return run_linear<FMT, DT, 4, MODE>(p, st);
+    case 8: return run_linear<FMT, DT, 8, MODE>(p, st);
+    case 16: return run_linear<FMT, DT, 16, MODE>(p, st);
+    case 32:
+        if constexpr (FMT == 0) return run_linear<FMT, DT, 32, MODE>(p, st);
+        break;
+    default: break;
+    }
+    return cudaErrorInvalidValue;
+}
+
+// Defined in the instantiation units.
+cudaError_t launch_fwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);
+cudaError_t launch_pack(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);
+cudaError_t launch_bwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);
+cudaError_t launch_bwd_shared(int fmt, int dt, int sub, const KParams& p, uint32_t ny,
+                              cudaStream_t st);
+cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_t st);
+
+}  // namespace focus

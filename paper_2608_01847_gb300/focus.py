@@ -1,0 +1,187 @@
+"""Python binding of libfocus_fq.so -- argument marshalling only.
+
+Every function here has the name of the C entry point it calls (see
+include/focus_fq.h for the semantics, layouts and error codes) and does no
+arithmetic of its own: it turns torch CUDA tensors into device pointers, the
+current torch stream into a cudaStream_t, allocates missing outputs with
+torch (PyTorch is the device-memory provider), and raises FocusError on a
+non-zero status.  There is no fallback: without the built library every call
+raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_build", "libfocus_fq.so")
+
+FOCUS_MXFP4, FOCUS_NVFP4 = 0, 1
+FOCUS_F32, FOCUS_BF16 = 0, 1
+FOCUS_STE_IDENTITY, FOCUS_STE_CLIPPED = 0, 1
+FOCUS_MX_CEIL, FOCUS_MX_FLOOR = 0, 1
+FOCUS_WS_ALPHA, FOCUS_WS_BWD = 0, 1
+
+STATUS = {0: "FOCUS_OK", -1: "FOCUS_ERR_INVALID_ARG", -2: "FOCUS_ERR_UNSUPPORTED",
+          -3: "FOCUS_ERR_MISALIGNED", -4: "FOCUS_ERR_WORKSPACE", -5: "FOCUS_ERR_CUDA"}
+
+ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_fq_fwd", "focus_fq_bwd", "focus_pack",
+                "focus_workspace_bytes", "focus_status_string", "focus_version")
+
+
+class FocusError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = _lib.focus_status_string(status).decode() if _lib is not None else str(status)
+        super().__init__(f"{where}: {STATUS.get(status, status)} ({msg})")
+
+
+class focus_desc_t(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int64), ("cols", ctypes.c_int64), ("ld", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("fmt", ctypes.c_int32), ("block", ctypes.c_int32),
+                ("sub_block", ctypes.c_int32), ("coef_shared_rows", ctypes.c_int32),
+                ("ste", ctypes.c_int32), ("mx_rule", ctypes.c_int32)]
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load the in-tree library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(LIB_PATH)
+        P, D, SZ = ctypes.c_void_p, ctypes.POINTER(focus_desc_t), ctypes.c_size_t
+        L.focus_nvfp4_alpha.argtypes = [D, P, P, P, SZ, P]
+        L.focus_fq_fwd.argtypes = [D, P, P, P, P, P, P, P]
+        L.focus_fq_bwd.argtypes = [D, P, P, P, P, P, P, P, P, P, SZ, P]
+        L.focus_pack.argtypes = [D, P, P, P, P, P, P, P]
+        L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
+        L.focus_workspace_bytes.restype = SZ
+        L.focus_status_string.argtypes = [ctypes.c_int]
+        L.focus_status_string.restype = ctypes.c_char_p
+        L.focus_version.restype = ctypes.c_int
+        for n in ("focus_nvfp4_alpha", "focus_fq_fwd", "focus_fq_bwd", "focus_pack"):
+            getattr(L, n).restype = ctypes.c_int
+        _lib = L
+    return _lib
+
+
+def block_of(fmt: int) -> int:
+    return 32 if fmt == FOCUS_MXFP4 else 16
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return FOCUS_F32
+    if t.dtype == torch.bfloat16:
+        return FOCUS_BF16
+    raise TypeError(f"unsupported dtype {t.dtype} (float32 or bfloat16)")
+
+
+def make_desc(x: torch.Tensor, fmt: int = FOCUS_MXFP4, sub_block: int = 8, shared: bool = False,
+              ste: int = FOCUS_STE_IDENTITY, mx_rule: int = FOCUS_MX_CEIL,
+              block: Optional[int] = None) -> focus_desc_t:
+    if x.dim() != 2 or (x.shape[0] > 1 and x.shape[1] > 0 and x.stride(1) != 1):
+        raise ValueError("x must be a 2-D tensor with unit stride along columns")
+    rows, cols = x.shape
+    ld = x.stride(0) if rows > 1 else cols
+    return focus_desc_t(rows, cols, ld, _dtype_code(x), fmt, block or block_of(fmt),
+                        sub_block, int(bool(shared)), ste, mx_rule)
+
+
+def _p(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _check(rc: int, where: str):
+    if rc != 0:
+        raise FocusError(rc, where)
+
+
+def focus_workspace_bytes(desc: focus_desc_t, which: int) -> int:
+    return int(lib().focus_workspace_bytes(ctypes.byref(desc), which))
+
+
+def _workspace(desc, which, device, ws):
+    n = focus_workspace_bytes(desc, which)
+    if ws is None:
+        ws = torch.empty(max(n, 16), dtype=torch.uint8, device=device)
+    return ws, ws.numel() * ws.element_size()
+
+
+def focus_nvfp4_alpha(x: torch.Tensor, alpha_out: Optional[torch.Tensor] = None,
+                      ws: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Per-tensor NVFP4 scale alpha = max|x| / 2688 (Eq. 2) as a [1] fp32 tensor."""
+    desc = make_desc(x, FOCUS_NVFP4)
+    if alpha_out is None:
+        alpha_out = torch.empty(1, dtype=torch.float32, device=x.device)
+    ws, nb = _workspace(desc, FOCUS_WS_ALPHA, x.device, ws)
+    _check(lib().focus_nvfp4_alpha(ctypes.byref(desc), _p(x), _p(alpha_out), _p(ws), nb,
+                                   _stream(x.device)), "focus_nvfp4_alpha")
+    return alpha_out
+
+
+def focus_fq_fwd(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
+                 mx_rule=FOCUS_MX_CEIL, y=None, scale_bytes=None, want_scales=False):
+    """y = Q_E2M1(x / S^q) * S^dq (Eq. 1-8); returns y, or (y, scale_bytes)."""
+    desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
+    if y is None:
+        y = torch.empty_like(x)
+    if scale_bytes is None and want_scales:
+        scale_bytes = torch.empty((x.shape[0], x.shape[1] // block_of(fmt)), dtype=torch.uint8,
+                                  device=x.device)
+    _check(lib().focus_fq_fwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(y),
+                              _p(scale_bytes), _stream(x.device)), "focus_fq_fwd")
+    return (y, scale_bytes) if (want_scales or scale_bytes is not None) else y
+
+
+def focus_fq_bwd(x, g, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
+                 ste=FOCUS_STE_IDENTITY, mx_rule=FOCUS_MX_CEIL, want_gx=True, want_gcrs=None,
+                 want_gdgs=None, gx=None, gcrs=None, gdgs=None, ws=None):
+    """STE backward (Sec. 3.2): returns (gx, gcrs, gdgs); an unrequested output is None.
+    By default gcrs / gdgs are produced when crs / dgs are given."""
+    desc = make_desc(x, fmt, sub_block, shared, ste, mx_rule)
+    rows, cols = x.shape
+    crow = 1 if shared else rows
+    want_gcrs = (crs is not None) if want_gcrs is None else want_gcrs
+    want_gdgs = (dgs is not None) if want_gdgs is None else want_gdgs
+    if gx is None and want_gx:
+        gx = torch.empty_like(x)
+    if gcrs is None and want_gcrs:
+        gcrs = torch.empty((crow, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
+    if gdgs is None and want_gdgs:
+        gdgs = torch.empty((crow, cols // sub_block), dtype=torch.float32, device=x.device)
+    ws, nb = _workspace(desc, FOCUS_WS_BWD, x.device, ws)
+    _check(lib().focus_fq_bwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(g),
+                              _p(gx), _p(gcrs), _p(gdgs), _p(ws), nb, _stream(x.device)),
+           "focus_fq_bwd")
+    return gx, gcrs, gdgs
+
+
+def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
+               mx_rule=FOCUS_MX_CEIL, codes=None, scale_bytes=None):
+    """Export (Fig. 3(d)): returns (codes [rows, cols/2] uint8, scale bytes [rows, cols/B])."""
+    desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
+    rows, cols = x.shape
+    if codes is None:
+        codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device=x.device)
+    if scale_bytes is None:
+        scale_bytes = torch.empty((rows, cols // block_of(fmt)), dtype=torch.uint8, device=x.device)
+    _check(lib().focus_pack(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(codes),
+                            _p(scale_bytes), _stream(x.device)), "focus_pack")
+    return codes, scale_bytes
+
+
+def focus_version() -> int:
+    return int(lib().focus_version())

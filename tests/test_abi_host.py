@@ -1,0 +1,140 @@
+"""Host-side checks of the C ABI (no GPU needed).
+
+The library must build for sm_103a, load, and export every entry point that
+include/focus_fq.h declares -- and nothing else.  Argument errors must be
+reported with the documented status before anything reaches the GPU, so the
+calls below use placeholder pointer values that are never dereferenced.
+"""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2608_01847_gb300 import build as B
+from paper_2608_01847_gb300 import focus as F
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "focus_fq.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    B.build()
+    return F.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(focus_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_abi():
+    assert declared_functions() == sorted(F.ENTRY_POINTS)
+
+
+def test_exports_exactly_the_declared_symbols(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", B.LIB], capture_output=True, text=True,
+                         check=True).stdout
+    exported = sorted({ln.split()[-1] for ln in out.splitlines()
+                       if ln.split() and ln.split()[-2] in ("T", "W")
+                       and not ln.split()[-1].startswith("_")})
+    assert exported == declared_functions()
+
+
+def test_version_and_status_strings(L):
+    assert F.focus_version() == 100
+    for code in (0, -1, -2, -3, -4, -5):
+        assert L.focus_status_string(code)
+    assert L.focus_status_string(42) == b"unknown status"
+
+
+def _desc(rows=4, cols=64, ld=None, dtype=1, fmt=0, block=None, sub=8, shared=0, ste=0, rule=0):
+    return F.focus_desc_t(rows, cols, cols if ld is None else ld, dtype, fmt,
+                          block if block is not None else (32 if fmt == 0 else 16), sub, shared,
+                          ste, rule)
+
+
+P = ctypes.c_void_p
+ALIGNED = P(0x100000)       # placeholder device addresses: never dereferenced
+ALIGNED2 = P(0x200000)
+ODD = P(0x100008)           # 8-byte aligned only
+
+
+def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None):
+    return L.focus_fq_fwd(ctypes.byref(d) if d is not None else None, x, crs, dgs, alpha, y, sb, None)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(block=64), -2), (dict(fmt=1, block=32), -2), (dict(sub=3), -2), (dict(sub=32, fmt=1), -2),
+    (dict(sub=64), -2), (dict(cols=48), -1), (dict(ld=60), -1), (dict(ld=68), -3),
+    (dict(dtype=2), -1), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
+    (dict(shared=2), -1), (dict(rows=-1), -1), (dict(rows=1 << 40, cols=1 << 20), -2),
+])
+def test_descriptor_rejections(L, kw, status):
+    assert fwd(L, _desc(**kw)) == status
+
+
+def test_null_and_alignment_rejections(L):
+    assert fwd(L, None) == -1
+    assert fwd(L, _desc(), x=None) == -1
+    assert fwd(L, _desc(), y=None) == -1
+    assert fwd(L, _desc(fmt=1), alpha=None) == -1                 # NVFP4 needs alpha
+    assert fwd(L, _desc(), x=ODD) == -3
+    assert fwd(L, _desc(), y=ODD) == -3
+    assert fwd(L, _desc(), crs=ODD) == -3
+    assert fwd(L, _desc(rows=0)) == 0                             # empty: nothing to do
+    d = _desc()
+    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, None, ALIGNED2, None) == -1
+    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, P(0x100002), ALIGNED2, None) == -3
+    g = ALIGNED2
+    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, g, None, None, None, 0,
+                          None) == -1                             # g missing
+    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, g, ODD, None, None, None, 0,
+                          None) == -3                             # gx misaligned
+    assert L.focus_nvfp4_alpha(ctypes.byref(d), ALIGNED, None, ALIGNED2, 1 << 20, None) == -1
+
+
+def test_shared_backward_needs_workspace(L):
+    d = _desc(rows=64, cols=256, shared=1)
+    need = L.focus_workspace_bytes(ctypes.byref(d), F.FOCUS_WS_BWD)
+    assert need > 0
+    gc = ALIGNED2
+    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, ALIGNED2, None, gc, None,
+                        None, 0, None)
+    assert rc == -4
+    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, ALIGNED2, None, gc, None,
+                        ALIGNED, need - 1, None)
+    assert rc == -4
+    assert L.focus_nvfp4_alpha(ctypes.byref(d), ALIGNED, ALIGNED2, None, 0, None) == -4
+
+
+def test_workspace_queries(L):
+    d = _desc(rows=64, cols=256, shared=0)
+    assert L.focus_workspace_bytes(ctypes.byref(d), F.FOCUS_WS_BWD) == 0
+    assert L.focus_workspace_bytes(ctypes.byref(d), F.FOCUS_WS_ALPHA) >= 4
+    assert L.focus_workspace_bytes(ctypes.byref(d), 7) == 0
+    assert L.focus_workspace_bytes(None, 0) == 0
+
+
+def test_fastdiv_magic_numbers():
+    """The invariant-divisor reciprocal used for row / column indices
+    (Granlund-Montgomery) divides exactly for every 32-bit numerator."""
+    import numpy as np
+    rng = np.random.default_rng(0)
+    for d in [1, 2, 3, 7, 64, 320, 1216, 3584, 4096, 65535, 1 << 20, (1 << 28) + 3]:
+        l = 0
+        while (1 << l) < d:
+            l += 1
+        m = ((1 << 32) * ((1 << l) - d)) // d + 1
+        assert m < (1 << 32)
+        n = np.concatenate([rng.integers(0, 1 << 32, 200000, dtype=np.uint64),
+                            np.array([0, 1, d - 1, d, d + 1, (1 << 32) - 1], np.uint64)])
+        n = n[n < (1 << 32)]
+        t = (n * np.uint64(m)) >> np.uint64(32)
+        q = (t + n) >> np.uint64(l)
+        assert np.array_equal(q, n // np.uint64(d)), d
