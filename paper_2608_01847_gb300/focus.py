@@ -96,6 +96,28 @@ def make_desc(x: torch.Tensor, fmt: int = FOCUS_MXFP4, sub_block: int = 8, share
                         sub_block, int(bool(shared)), ste, mx_rule)
 
 
+def _like_x(x: torch.Tensor) -> torch.Tensor:
+    """An output with x's exact shape and row pitch (the ABI's [rows, ld] layout)."""
+    return torch.empty_strided(tuple(x.shape), tuple(x.stride()), dtype=x.dtype, device=x.device)
+
+
+def _same_layout(x: torch.Tensor, t: Optional[torch.Tensor], name: str):
+    if t is None:
+        return
+    if t.shape != x.shape or t.dtype != x.dtype or t.device != x.device or (
+            x.shape[0] > 1 and t.stride() != x.stride()):
+        raise ValueError(f"{name} must have x's shape, dtype, device and strides "
+                         f"(got {tuple(t.shape)} {t.dtype} stride {t.stride()}, "
+                         f"x is {tuple(x.shape)} {x.dtype} stride {x.stride()})")
+
+
+def _dense(t: Optional[torch.Tensor], n: int, dtype, name: str):
+    if t is None:
+        return
+    if not t.is_contiguous() or t.numel() != n or t.dtype != dtype:
+        raise ValueError(f"{name} must be a contiguous {dtype} tensor of {n} elements")
+
+
 def _p(t: Optional[torch.Tensor]):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
@@ -107,6 +129,14 @@ def _stream(device) -> ctypes.c_void_p:
 def _check(rc: int, where: str):
     if rc != 0:
         raise FocusError(rc, where)
+
+
+def _check_coefs(x, fmt, sub_block, shared, c, d):
+    rows, cols = x.shape
+    crow = 1 if shared else rows
+    _dense(c, crow * (cols // block_of(fmt)), torch.float32, "block coefficients")
+    _dense(d, crow * (cols // sub_block) if sub_block else 0, torch.float32,
+           "sub-block coefficients")
 
 
 def focus_workspace_bytes(desc: focus_desc_t, which: int) -> int:
@@ -136,11 +166,14 @@ def focus_fq_fwd(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=
                  mx_rule=FOCUS_MX_CEIL, y=None, scale_bytes=None, want_scales=False):
     """y = Q_E2M1(x / S^q) * S^dq (Eq. 1-8); returns y, or (y, scale_bytes)."""
     desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
+    _check_coefs(x, fmt, sub_block, shared, crs, dgs)
     if y is None:
-        y = torch.empty_like(x)
+        y = _like_x(x)
+    _same_layout(x, y, "y")
     if scale_bytes is None and want_scales:
         scale_bytes = torch.empty((x.shape[0], x.shape[1] // block_of(fmt)), dtype=torch.uint8,
                                   device=x.device)
+    _dense(scale_bytes, x.shape[0] * (x.shape[1] // block_of(fmt)), torch.uint8, "scale_bytes")
     _check(lib().focus_fq_fwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(y),
                               _p(scale_bytes), _stream(x.device)), "focus_fq_fwd")
     return (y, scale_bytes) if (want_scales or scale_bytes is not None) else y
@@ -156,12 +189,16 @@ def focus_fq_bwd(x, g, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shar
     crow = 1 if shared else rows
     want_gcrs = (crs is not None) if want_gcrs is None else want_gcrs
     want_gdgs = (dgs is not None) if want_gdgs is None else want_gdgs
+    _check_coefs(x, fmt, sub_block, shared, crs, dgs)
+    _same_layout(x, g, "g")
     if gx is None and want_gx:
-        gx = torch.empty_like(x)
+        gx = _like_x(x)
+    _same_layout(x, gx, "gx")
     if gcrs is None and want_gcrs:
         gcrs = torch.empty((crow, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
     if gdgs is None and want_gdgs:
         gdgs = torch.empty((crow, cols // sub_block), dtype=torch.float32, device=x.device)
+    _check_coefs(x, fmt, sub_block, shared, gcrs, gdgs)
     ws, nb = _workspace(desc, FOCUS_WS_BWD, x.device, ws)
     _check(lib().focus_fq_bwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(g),
                               _p(gx), _p(gcrs), _p(gdgs), _p(ws), nb, _stream(x.device)),
@@ -178,6 +215,9 @@ def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=Fa
         codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device=x.device)
     if scale_bytes is None:
         scale_bytes = torch.empty((rows, cols // block_of(fmt)), dtype=torch.uint8, device=x.device)
+    _check_coefs(x, fmt, sub_block, shared, crs, dgs)
+    _dense(codes, rows * cols // 2, torch.uint8, "codes")
+    _dense(scale_bytes, rows * cols // block_of(fmt), torch.uint8, "scale_bytes")
     _check(lib().focus_pack(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(codes),
                             _p(scale_bytes), _stream(x.device)), "focus_pack")
     return codes, scale_bytes
