@@ -113,6 +113,27 @@ enum { FOCUS_WS_ALPHA = 0, FOCUS_WS_BWD = 1 };
 int focus_nvfp4_alpha(const focus_desc_t* desc, const void* x, float* alpha_out,
                       void* ws, size_t ws_bytes, focus_stream_t stream);
 
+/* focus_nvfp4_alpha for callers that cannot allocate device memory.  The
+ * paper has no counterpart: this is a deployment aid of this library.
+ * Computes exactly what focus_nvfp4_alpha computes, but takes no workspace:
+ * the per-CTA partial maxima live in a 16 KiB array inside the library's own
+ * device memory (4096 fp32 slots, held by every GPU that loads the library
+ * until the process exits).  Meant for code that is handed only its input
+ * and output buffers -- e.g. a plugin inside a host application that owns
+ * every device allocation -- or that must never call cudaMalloc on its hot
+ * path because that call can synchronise the device.  It calls no
+ * allocating routine.
+ * - The first call on a device looks up the array's device address (with
+ *   that device current) and caches it; make that first call before any
+ *   stream capture.
+ * - Every call on a device shares the one array, so calls that overlap on
+ *   the GPU (e.g. on two streams at once) race and may return wrong values;
+ *   serialise them.  Nothing in the array needs clearing between calls.
+ * - Returns FOCUS_ERR_WORKSPACE if the pass would need more than 4096
+ *   partial slots (a GPU with more than 512 SMs). */
+int focus_nvfp4_alpha_noalloc(const focus_desc_t* desc, const void* x, float* alpha_out,
+                              focus_stream_t stream);
+
 /* Fake-quantization forward, Eq. 1-3 and 6-8: y = Q_E2M1(x / S^q) * S^dq.
  * x      [rows, ld] input (read only).
  * crs    CRS coefficients c_i, or NULL for 1 (Eq. 6-7).

@@ -28,7 +28,7 @@ FOCUS_WS_ALPHA, FOCUS_WS_BWD = 0, 1
 STATUS = {0: "FOCUS_OK", -1: "FOCUS_ERR_INVALID_ARG", -2: "FOCUS_ERR_UNSUPPORTED",
           -3: "FOCUS_ERR_MISALIGNED", -4: "FOCUS_ERR_WORKSPACE", -5: "FOCUS_ERR_CUDA"}
 
-ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_fq_fwd", "focus_fq_bwd", "focus_pack",
+ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd", "focus_pack",
                 "focus_workspace_bytes", "focus_status_string", "focus_version")
 
 
@@ -59,6 +59,7 @@ def lib() -> ctypes.CDLL:
         L = ctypes.CDLL(LIB_PATH)
         P, D, SZ = ctypes.c_void_p, ctypes.POINTER(focus_desc_t), ctypes.c_size_t
         L.focus_nvfp4_alpha.argtypes = [D, P, P, P, SZ, P]
+        L.focus_nvfp4_alpha_noalloc.argtypes = [D, P, P, P]
         L.focus_fq_fwd.argtypes = [D, P, P, P, P, P, P, P]
         L.focus_fq_bwd.argtypes = [D, P, P, P, P, P, P, P, P, P, SZ, P]
         L.focus_pack.argtypes = [D, P, P, P, P, P, P, P]
@@ -67,7 +68,7 @@ def lib() -> ctypes.CDLL:
         L.focus_status_string.argtypes = [ctypes.c_int]
         L.focus_status_string.restype = ctypes.c_char_p
         L.focus_version.restype = ctypes.c_int
-        for n in ("focus_nvfp4_alpha", "focus_fq_fwd", "focus_fq_bwd", "focus_pack"):
+        for n in ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd", "focus_pack"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -159,6 +160,16 @@ def focus_nvfp4_alpha(x: torch.Tensor, alpha_out: Optional[torch.Tensor] = None,
     ws, nb = _workspace(desc, FOCUS_WS_ALPHA, x.device, ws)
     _check(lib().focus_nvfp4_alpha(ctypes.byref(desc), _p(x), _p(alpha_out), _p(ws), nb,
                                    _stream(x.device)), "focus_nvfp4_alpha")
+    return alpha_out
+
+
+def focus_nvfp4_alpha_noalloc(x: torch.Tensor, alpha_out: torch.Tensor) -> torch.Tensor:
+    """focus_nvfp4_alpha without a workspace, for callers that cannot allocate
+    device memory: the partials live in the library's static device array.
+    alpha_out must be given (a [1] fp32 CUDA tensor); nothing is allocated."""
+    desc = make_desc(x, FOCUS_NVFP4)
+    _check(lib().focus_nvfp4_alpha_noalloc(ctypes.byref(desc), _p(x), _p(alpha_out),
+                                           _stream(x.device)), "focus_nvfp4_alpha_noalloc")
     return alpha_out
 
 
