@@ -343,10 +343,10 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
 /* STE backward (Sec. 3.2: STE on all non-differentiable ops; Eq. 6-8)  */
 /* ------------------------------------------------------------------ */
 /* With y = Q(x / S^q) * S^dq and the STE taking dQ(u)/du = mask (1, or
- * [|u| <= 6] in the clipped variant):
- *   gx      = mask ? fl(fl(g * S^dq) / S^q) : +0   (the order autograd takes:
- *             the product's backward first, then the quotient's)
- *   dy/dc_eff = -mask * x / c_eff^2               (S^dq cancels)
+ * [|u| <= 6] in the clipped variant), dy/dx = mask * S^dq / S^q:
+ *   rho     = fl(S^dq / S^q)           (once per sub-block)
+ *   gx      = mask ? fl(g * rho) : +0
+ *   dy/dc_eff = -mask * x / c_eff^2    (S^dq cancels)
  * With T_ik = sum over sub-block (i,k) of mask*g*x and c_eff = c_i * c_i^k
  * taken exactly (binary64):
  *   dL/dc_i^k = -T_ik * c_i / c_eff^2
@@ -399,6 +399,9 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                 float c_eff = c * d;
                 float s_q = s_dq * c_eff;
                 int dead = (s_dq == 0.0f) || (s_q == 0.0f) || isinf(s_q);
+                /* the STE derivative of y = Q(x / S^q) * S^dq w.r.t. x is the
+                 * scale ratio S^dq / S^q, rounded once for the sub-block */
+                float rho = dead ? 0.0f : s_dq / s_q;
                 ksum_t T = zero, Ta = zero;
                 for (int e = 0; e < sub; e++) {
                     int64_t col = j * block + (int64_t)k * sub + e;
@@ -412,8 +415,7 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                             mask = fabsf(u) <= 6.0f;
                         }
                         if (mask) {
-                            float t = gv * s_dq;
-                            gxv = t / s_q;
+                            gxv = gv * rho;
                             double p = (double)gv * (double)xv;   /* exact */
                             ksum_add(&T, p);
                             ksum_add(&Ta, fabs(p));

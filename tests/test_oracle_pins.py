@@ -91,11 +91,11 @@ def test_hand_mxfp4_block_crs():
     assert out["scales"][0, 0] == 0x7D            # S^dq is unchanged by c
     assert list(out["codes"][0, :2]) == [0xA4, 0x61]
     assert list(out["y"][0, :4]) == [0.5, -0.25, 0.125, 1.0]
-    # STE backward with g = 1 on the first four: gx = fl(fl(1*0.25)/0.3125) = fl(0.8)
+    # STE backward with g = 1 on the first four: gx = g * fl(S^dq / S^q) = fl(0.25 / 0.3125)
     g = np.zeros_like(x)
     g[0, :4] = 1
     b = O.bwd(x, g, O.MXFP4, crs=crs)
-    assert np.all(b["gx"][0, :4] == np.float32(0.25) / np.float32(0.3125))
+    assert np.all(b["gx"][0, :4] == np.float32(0.8))
     assert np.all(b["gx"][0, 4:] == 0)
     # dL/dc = -(0.7 - 0.26 + 0.13 + 1.5) / 1.25^2 = -1.3248 (inputs as float32)
     expect = -(float(np.float32(0.7)) + float(np.float32(-0.26)) + float(np.float32(0.13)) + 1.5) / 1.5625
@@ -335,13 +335,34 @@ def test_dequant_of_export_equals_forward(fmt, dtype):
     assert np.array_equal(dq, out["y"])
 
 
-def test_mxfp4_input_gradient_is_g_at_c1():
-    """With c = 1 and a normal power-of-two S^dq, g * 2^e / 2^e is exact."""
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_input_gradient_at_c1_is_g(fmt):
+    """At c = 1 the two scales coincide, S^dq / S^q = 1, and the STE passes
+    the gradient through unchanged (live blocks)."""
     w = W.WORKLOADS["w256x512_f32"]
     x = W.draw_values(w, 16, 512, 31)
     g = W.draw_grad(16, 512, 32)
-    b = O.bwd(x, g, O.MXFP4)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    b = O.bwd(x, g, fmt, alpha=a)
     assert np.array_equal(b["gx"], g)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_input_gradient_is_g_over_c(fmt):
+    """dy/dx of the relaxed surrogate is S^dq / S^q = 1 / (c_i c_i^k): the
+    input gradient equals g / c_eff up to the roundings of S^q, of the ratio
+    and of the product, i.e. within 2^-22 relative."""
+    rng = np.random.default_rng(41)
+    block = 32 if fmt == O.MXFP4 else 16
+    x = (rng.standard_normal((8, 4 * block)) * 0.02).astype(np.float32)
+    g = rng.standard_normal(x.shape).astype(np.float32)
+    crs = rng.uniform(0.8, 1.2, (8, 4)).astype(np.float32)
+    dgs = rng.uniform(0.8, 1.2, (8, 4 * block // 8)).astype(np.float32)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    b = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a)
+    ceff = np.repeat(crs.astype(np.float64), block, 1) * np.repeat(dgs.astype(np.float64), 8, 1)
+    expect = g.astype(np.float64) / ceff
+    np.testing.assert_allclose(b["gx"].astype(np.float64), expect, rtol=2.0 ** -22, atol=0)
 
 
 # ---------------------------------------------------------------------------
@@ -416,6 +437,18 @@ def torch_fake_quant(x, crs, dgs, sdq, block, sub):
     return (u + (q - u).detach()) * s
 
 
+def torch_ste_ratio(x, crs, dgs, sdq, block, sub):
+    """The same forward written as y = x * rho + (Q(x / S^q) * S^dq - x * rho).detach()
+    with the scale ratio rho = S^dq / S^q: autograd's input gradient is g * rho."""
+    c = crs.repeat_interleave(block, dim=1)
+    d = dgs.repeat_interleave(sub, dim=1)
+    s = sdq.repeat_interleave(block, dim=1)
+    s_q = s * (c * d)
+    rho = (s / s_q).detach()
+    q = torch.from_numpy(e2m1_ref((x / s_q).detach().numpy())).to(x.dtype)
+    return x * rho + (q * s - x * rho).detach()
+
+
 @pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
 def test_autograd_restatement(fmt):
     rng = np.random.default_rng(55)
@@ -441,9 +474,12 @@ def test_autograd_restatement(fmt):
     ct = torch.from_numpy(crs).requires_grad_(True)
     dt = torch.from_numpy(dgs).requires_grad_(True)
     y = torch_fake_quant(xt, ct, dt, torch.from_numpy(sdq), block, sub)
-    y.backward(torch.from_numpy(g))
     assert np.array_equal(y.detach().numpy(), fw["y"])
-    assert np.array_equal(xt.grad.numpy(), ours["gx"])
+    x2 = torch.from_numpy(x).requires_grad_(True)
+    y2 = torch_ste_ratio(x2, ct, dt, torch.from_numpy(sdq), block, sub)
+    y2.backward(torch.from_numpy(g))
+    assert np.array_equal(y2.detach().numpy(), fw["y"])
+    assert np.array_equal(x2.grad.numpy(), ours["gx"])
     # float64 autograd for the coefficient gradients
     x6 = torch.from_numpy(x.astype(np.float64))
     c6 = torch.from_numpy(crs.astype(np.float64)).requires_grad_(True)
