@@ -154,17 +154,86 @@ __device__ __forceinline__ float exp2_int(int e)
                        : __uint_as_float(0x00400000u);
 }
 
-// NVFP4 block scale (Eq. 2): Delta = Q_E4M3(m / fl(alpha * 6)),
-// S^dq = fl(Delta * alpha); an all-zero block has Delta = 0.
-__device__ __forceinline__ float nv_scale(float m, float alpha, uint32_t& byte)
+// ---------------------------------------------------------------------------
+// Deciding on an IEEE quotient without dividing.
+//
+// Several steps use a quotient q = fl(a / b) (IEEE division, round to
+// nearest) only through a monotone rounding of it: its E2M1 code, the
+// clipping test |q| <= 6, its E4M3 code, the E8M0 ceiling exponent.  With r
+// within a few ulps of 1/b (rcp.approx.f32 is within 1 ulp), the products
+//   a * fl(r * (1 - 2^-18))  and  a * fl(r * (1 + 2^-18))
+// bracket q strictly (their relative distance to a/b is at least
+// 2^-18 - 2^-21 > 2^-24, the most fl(a/b) can move).  A monotone rounding
+// that agrees on both brackets therefore agrees on q; only when the brackets
+// straddle a decision boundary is the exact quotient computed.  The estimate
+// needs b and 1/b normal: exponent field of b in [2, 252].
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float rcp_approx(float b)
 {
-    if (m == 0.0f) {
-        byte = 0u;
-        return 0.0f;
-    }
-    const float den = __fmul_rn(alpha, 6.0f);
-    byte = e4m3_encode(__fdiv_rn(m, den));
+    float r;
+    asm("rcp.approx.f32 %0, %1;" : "=f"(r) : "f"(b));
+    return r;
+}
+
+constexpr float kBracketLo = 1.0f - 0x1p-18f;
+constexpr float kBracketHi = 1.0f + 0x1p-18f;
+
+__device__ __forceinline__ bool recip_ok(float b)
+{
+    const uint32_t E = __float_as_uint(b) >> 23;
+    return (E >= 2u) && (E <= 252u);
+}
+
+struct Bracket {
+    float lo, hi;  // bracketing multipliers for 1/b
+    bool ok;
+};
+
+__device__ __forceinline__ Bracket make_bracket(float b)
+{
+    const float r = rcp_approx(b);
+    return {__fmul_rn(r, kBracketLo), __fmul_rn(r, kBracketHi), recip_ok(b)};
+}
+
+// True when q' may sit within 16 encodings of a value whose encoding has its
+// low LOWBITS bits clear (used for the E8M0 power-of-two test, where q' is
+// within a few encodings of q).
+template <int LOWBITS>
+__device__ __forceinline__ bool near_threshold(float qp)
+{
+    constexpr uint32_t mask = (1u << LOWBITS) - 1u;
+    return ((__float_as_uint(qp) + 16u) & mask) < 32u;
+}
+
+// NVFP4 block scale (Eq. 2): Delta = Q_E4M3(m / den), den = fl(alpha * 6),
+// S^dq = fl(Delta * alpha); an all-zero block has Delta = 0.  `bd` brackets
+// 1/den (uniform over the tensor): both brackets are converted with one
+// cvt, and the exact quotient is needed only when their E4M3 codes differ.
+__device__ __forceinline__ float nv_scale(float m, float alpha, float den, const Bracket& bd,
+                                          uint32_t& byte)
+{
+    uint16_t h;
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;"
+        : "=h"(h)
+        : "f"(__fmul_rn(m, bd.hi)), "f"(__fmul_rn(m, bd.lo)));
+    byte = h & 0xffu;
+    if (!bd.ok || (h >> 8) != byte) byte = e4m3_encode(__fdiv_rn(m, den));
+    if (m == 0.0f) byte = 0u;
     return __fmul_rn(e4m3_decode(byte), alpha);
+}
+
+// MXFP4 ceiling exponent with the quotient m / 6 estimated (see above):
+// only whether fl(m/6) is a power of two, and its binade, matter.
+__device__ __forceinline__ int mx_exponent_fast(float m, int rule)
+{
+    if (rule == 0) {
+        const float t = __fmul_rn(m, 1.0f / 6.0f);
+        const uint32_t b = __float_as_uint(t);
+        const uint32_t E = b >> 23;
+        if (E >= 2u && E <= 252u && !near_threshold<23>(t))
+            return min(max(static_cast<int>(E) - 126, -127), 127);  // not a power of two
+    }
+    return mx_exponent(m, rule);
 }
 
 // ---------------------------------------------------------------------------
@@ -207,10 +276,10 @@ __device__ __forceinline__ void sum2_add(df& acc, float p)
     acc.l = __fadd_rn(acc.l, s.l);
 }
 
-// (a.h + a.l) / b to about 2^-46 relative (b > 0, finite).
-__device__ __forceinline__ df df_div_f(df a, float b)
+// (a.h + a.l) / b to about 2^-44 relative, given r within a few ulps of 1/b
+// (b > 0, normal): one correction step on the FMA residual.
+__device__ __forceinline__ df df_div_f(df a, float b, float r)
 {
-    const float r = __frcp_rn(b);
     const float q1 = __fmul_rn(a.h, r);
     const float rem = __fmaf_rn(-q1, b, a.h);
     const float q2 = __fmul_rn(__fadd_rn(rem, a.l), r);

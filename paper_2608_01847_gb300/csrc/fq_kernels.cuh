@@ -13,10 +13,10 @@
 //   m      = block absmax                       (Eq. 2-3)
 //   S^dq   = 2^e (E8M0) or fl(alpha * E4M3)     (Eq. 2-3)
 //   c_eff  = fl(c_i * c_i^k),  S^q = fl(S^dq * c_eff)   (Eq. 6, 8)
-//   u      = fl(x / S^q) (IEEE division), code = Q_E2M1(u)  (Eq. 1, 7, 8)
+//   u      = fl(x / S^q) (IEEE quotient), code = Q_E2M1(u)   (Eq. 1, 7, 8)
 //   y      = fl(E2M1(code) * S^dq)               (Eq. 1, 7, 8)
 // and the STE backward (Sec. 3.2):
-//   gx     = mask * fl(fl(g * S^dq) / S^q)
+//   gx     = mask * fl(g * rho),  rho = fl(S^dq / S^q) once per sub-block
 //   T_ik   = sum of mask * g * x over the sub-block (compensated, Sum2)
 //   dL/dc_i^k = -T_ik / (c_i (c_i^k)^2),  dL/dc_i = -(sum_k T_ik / c_i^k) / c_i^2
 #pragma once
@@ -63,18 +63,36 @@ struct Geo {
     static_assert(SUB >= 2 && SUB <= B && B % SUB == 0, "sub-block must divide the block");
 };
 
-// Block absmax over the LPB lanes of a block, then the hardware scale.
+// Per-tensor constants of the block-scale step: NVFP4's alpha, fl(alpha * 6)
+// and the bracket of its reciprocal.
+struct TensorScale {
+    float alpha;
+    float den;
+    Bracket bd;
+};
+
 template <int FMT>
-__device__ __forceinline__ float block_scale(float m, float alpha, int mx_rule, uint32_t& byte)
+__device__ __forceinline__ TensorScale tensor_scale(const float* alpha_ptr)
+{
+    TensorScale t;
+    t.alpha = (FMT == 1) ? __ldg(alpha_ptr) : 0.0f;
+    t.den = __fmul_rn(t.alpha, 6.0f);
+    t.bd = make_bracket(t.den);
+    return t;
+}
+
+template <int FMT>
+__device__ __forceinline__ float block_scale(float m, const TensorScale& ts, int mx_rule,
+                                             uint32_t& byte)
 {
 #pragma unroll
     for (int o = 1; o < (FMT == 0 ? 4 : 2); o <<= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, o));
     if (FMT == 0) {
-        const int e = mx_exponent(m, mx_rule);
+        const int e = mx_exponent_fast(m, mx_rule);
         byte = static_cast<uint32_t>(e + 127);
         return exp2_int(e);
     }
-    return nv_scale(m, alpha, byte);
+    return nv_scale(m, ts.alpha, ts.den, ts.bd, byte);
 }
 
 __device__ __forceinline__ float chunk_absmax(const float (&v)[8])
@@ -98,29 +116,129 @@ __device__ __forceinline__ void relaxed_scales(float sdq, float c, const float (
     }
 }
 
-// STE backward of one chunk: input gradient and per-sub-block Sum2 of mask*g*x.
-template <int DT, int NS>
-__device__ __forceinline__ void bwd_chunk(const float (&v)[8], const float (&gv)[8], float sdq,
-                                          const float (&sq)[NS], const bool (&dead)[NS],
-                                          int ste, bool want_gx, bool want_T, float (&gxo)[8],
-                                          df (&T)[NS])
+// Nibble mask of the live sub-blocks of a chunk (4 bits per element).
+template <int NS>
+__device__ __forceinline__ uint32_t live_nibbles(const bool (&dead)[NS])
 {
     constexpr int EPS = 8 / NS;
+    constexpr uint32_t sub_mask = EPS == 8 ? 0xffffffffu : ((1u << (4 * EPS)) - 1u);
+    uint32_t m = 0u;
 #pragma unroll
-    for (int t = 0; t < NS; ++t) T[t] = {0.0f, 0.0f};
+    for (int t = 0; t < NS; ++t) m |= dead[t] ? 0u : (sub_mask << (4 * EPS * t));
+    return m;
+}
+
+// E2M1 codes (Eq. 1) of u = fl(x / S^q) for the eight elements of a chunk,
+// exact: both brackets of every quotient (see make_bracket) are converted,
+// and when the two code words differ on a live element the quotients are
+// recomputed by IEEE division.  Dead sub-blocks get code 0.
+template <int NS>
+__device__ __forceinline__ uint32_t chunk_codes(const float (&v)[8], const float (&sq)[NS],
+                                                const bool (&dead)[NS])
+{
+    constexpr int EPS = 8 / NS;
+    Bracket br[NS];
+    bool ok = true;
+#pragma unroll
+    for (int t = 0; t < NS; ++t) {
+        br[t] = make_bracket(sq[t]);
+        ok = ok & (dead[t] | br[t].ok);
+    }
+    float lo[8], hi[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        lo[e] = __fmul_rn(v[e], br[e / EPS].lo);
+        hi[e] = __fmul_rn(v[e], br[e / EPS].hi);
+    }
+    const uint32_t live = live_nibbles<NS>(dead);
+    uint32_t c = e2m1_pack8(lo);
+    if (!ok | (((c ^ e2m1_pack8(hi)) & live) != 0u)) {
+        float u[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) u[e] = __fdiv_rn(v[e], sq[e / EPS]);
+        c = e2m1_pack8(u);
+    }
+    return c & live;
+}
+
+// Clipping mask of the STE (|fl(x / S^q)| <= 6, live sub-blocks only),
+// decided on the brackets and exactly when they straddle 6.
+template <int NS>
+__device__ __forceinline__ void chunk_clip_mask(const float (&v)[8], const float (&sq)[NS],
+                                                const bool (&dead)[NS], bool (&live)[8])
+{
+    constexpr int EPS = 8 / NS;
+    Bracket br[NS];
+#pragma unroll
+    for (int t = 0; t < NS; ++t) br[t] = make_bracket(sq[t]);
+    bool ambiguous = false;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
         const int t = e / EPS;
-        bool live = !dead[t];
-        if (ste == 1) live = live && (fabsf(__fdiv_rn(v[e], sq[t])) <= 6.0f);
-        if (want_gx) gxo[e] = live ? __fdiv_rn(__fmul_rn(gv[e], sdq), sq[t]) : 0.0f;
+        const float lo = fabsf(__fmul_rn(v[e], br[t].lo));
+        const float hi = fabsf(__fmul_rn(v[e], br[t].hi));
+        live[e] = !dead[t] & (hi <= 6.0f);
+        ambiguous = ambiguous | (!dead[t] & (!br[t].ok | ((lo <= 6.0f) != (hi <= 6.0f))));
+    }
+    if (ambiguous) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            live[e] = !dead[e / EPS] & (fabsf(__fdiv_rn(v[e], sq[e / EPS])) <= 6.0f);
+    }
+}
+
+// STE backward of one chunk: input gradient g * rho (rho = S^dq / S^q of the
+// sub-block, Sec. 3.2; rho = 0 on dead sub-blocks, and the +0 addend turns
+// -0 into +0) and the per-sub-block Sum2 of mask*g*x.
+template <int DT, int NS>
+__device__ __forceinline__ void bwd_chunk(const float (&v)[8], const float (&gv)[8],
+                                          const float (&sq)[NS], const float (&rho)[NS],
+                                          const bool (&dead)[NS], int ste, bool want_gx,
+                                          bool want_T, float (&gxo)[8], df (&T)[NS])
+{
+    constexpr int EPS = 8 / NS;
+    if (ste == 1) {
+        bool live[8];
+        chunk_clip_mask<NS>(v, sq, dead, live);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int t = e / EPS;
+            if (want_gx) gxo[e] = live[e] ? __fmul_rn(gv[e], rho[t]) : 0.0f;
+            if (want_T) {
+                const float a = live[e] ? gv[e] : 0.0f;
+                const float p = __fmul_rn(a, v[e]);  // exact for bf16 inputs
+                if (e % EPS == 0) T[t] = {p, 0.0f};
+                else sum2_add(T[t], p);
+                if (DT == 0) T[t].l = __fadd_rn(T[t].l, __fmaf_rn(a, v[e], -p));
+            }
+        }
+        return;
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const int t = e / EPS;
+        if (want_gx) gxo[e] = __fmaf_rn(gv[e], rho[t], 0.0f);
         if (want_T) {
-            const float a = live ? gv[e] : 0.0f;
-            const float p = __fmul_rn(a, v[e]);  // exact for bf16 inputs
-            sum2_add(T[t], p);
-            if (DT == 0) T[t].l = __fadd_rn(T[t].l, __fmaf_rn(a, v[e], -p));
+            const float p = __fmul_rn(gv[e], v[e]);  // exact for bf16 inputs
+            if (e % EPS == 0) T[t] = {p, 0.0f};
+            else sum2_add(T[t], p);
+            if (DT == 0) T[t].l = __fadd_rn(T[t].l, __fmaf_rn(gv[e], v[e], -p));
         }
     }
+    if (want_T) {
+#pragma unroll
+        for (int t = 0; t < NS; ++t)
+            if (dead[t]) T[t] = {0.0f, 0.0f};
+    }
+}
+
+// Scale ratio rho = fl(S^dq / S^q) per sub-block (0 for dead sub-blocks).
+template <int NS>
+__device__ __forceinline__ void scale_ratios(float sdq, const float (&sq)[NS], const bool (&dead)[NS],
+                                             float (&rho)[NS])
+{
+#pragma unroll
+    for (int t = 0; t < NS; ++t) rho[t] = dead[t] ? 0.0f : __fdiv_rn(sdq, sq[t]);
 }
 
 // ---------------------------------------------------------------------------
@@ -137,7 +255,7 @@ __global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
     using G = Geo<FMT, SUB>;
     constexpr int U = Unroll<DT, MODE>::U;
     constexpr int NS = G::NS;
-    const float alpha = (FMT == 1) ? __ldg(p.alpha) : 0.0f;
+    const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = (MODE == kBwd) && p.gx != nullptr;
     const bool want_T = (MODE == kBwd) && (p.gcrs != nullptr || p.gdgs != nullptr);
     const uint32_t span = U * kThreads;
@@ -186,19 +304,13 @@ __global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
             float v[8];
             unpack_chunk<DT>(xr[j], v);
             uint32_t sbyte;
-            const float sdq = block_scale<FMT>(chunk_absmax(v), alpha, p.mx_rule, sbyte);
+            const float sdq = block_scale<FMT>(chunk_absmax(v), ts, p.mx_rule, sbyte);
             float sq[NS];
             bool dead[NS];
             relaxed_scales<NS>(sdq, cv[j], dv[j], sq, dead);
 
             if (MODE != kBwd) {
-                float u[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int t = e / G::EPS;
-                    u[e] = dead[t] ? 0.0f : __fdiv_rn(v[e], sq[t]);
-                }
-                const uint32_t codes = e2m1_pack8(u);
+                const uint32_t codes = chunk_codes<NS>(v, sq, dead);
                 if (valid) {
                     if (MODE == kFwd) {
                         float q[8];
@@ -216,21 +328,26 @@ __global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
                 float gv[8];
                 unpack_chunk<DT>(gr[MODE == kBwd ? j : 0], gv);
                 float gxo[8];
+                float rho[NS];
                 df T[NS];
-                bwd_chunk<DT, NS>(v, gv, sdq, sq, dead, p.ste, want_gx, want_T, gxo, T);
+                if (want_gx) scale_ratios<NS>(sdq, sq, dead, rho);
+                bwd_chunk<DT, NS>(v, gv, sq, rho, dead, p.ste, want_gx, want_T, gxo, T);
                 if (want_gx && valid) store_chunk<DT>(p.gx, off[j], gxo);
                 if (want_T) {
                     // sub-blocks wider than a chunk: combine their lanes
 #pragma unroll
                     for (int o = 1; o < G::LPS; o <<= 1) T[0] = df_add(T[0], shfl_xor_df(T[0], o));
                     const float c = cv[j];
+                    const float rc = rcp_approx(c);
                     df Q = {0.0f, 0.0f};
                     float gd[NS];
 #pragma unroll
                     for (int t = 0; t < NS; ++t) {
-                        const df qk = df_div_f(T[t], dv[j][t]);  // T_ik / c_i^k
-                        gd[t] = -__fmul_rn(df_to_f(qk), __frcp_rn(__fmul_rn(c, dv[j][t])));
-                        if (G::LPS == 1 || (s % G::LPS) == 0) Q = df_add(Q, qk);
+                        const float d = dv[j][t];
+                        const float rd = rcp_approx(d);
+                        const df qk = df_div_f(T[t], d, rd);  // T_ik / c_i^k
+                        gd[t] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
+                        if (G::LPS == 1 || (s % G::LPS) == 0) Q = (t == 0) ? qk : df_add(Q, qk);
                     }
 #pragma unroll
                     for (int o = G::LPS; o < G::LPB; o <<= 1) Q = df_add(Q, shfl_xor_df(Q, o));
@@ -240,7 +357,7 @@ __global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
                             else if ((s % G::LPS) == 0) p.gdgs[s / G::LPS] = gd[0];
                         }
                         if (p.gcrs && (s % G::LPB) == 0)
-                            p.gcrs[s / G::LPB] = -df_to_f(df_div_f(df_div_f(Q, c), c));
+                            p.gcrs[s / G::LPB] = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
                     }
                 }
             }
@@ -262,7 +379,7 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
     using G = Geo<FMT, SUB>;
     constexpr int NS = G::NS;
     constexpr int U = DT == 1 ? 2 : 1;
-    const float alpha = (FMT == 1) ? __ldg(p.alpha) : 0.0f;
+    const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = p.gx != nullptr;
     const bool want_T = p.gcrs != nullptr || p.gdgs != nullptr;
     const uint32_t cc = blockIdx.x * kThreads + threadIdx.x;
@@ -305,13 +422,15 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
             unpack_chunk<DT>(xr[j], v);
             unpack_chunk<DT>(gr[j], gv);
             uint32_t sbyte;
-            const float sdq = block_scale<FMT>(chunk_absmax(v), alpha, p.mx_rule, sbyte);
+            const float sdq = block_scale<FMT>(chunk_absmax(v), ts, p.mx_rule, sbyte);
             float sq[NS];
             bool dead[NS];
             relaxed_scales<NS>(sdq, c, d, sq, dead);
             float gxo[8];
+            float rho[NS];
             df T[NS];
-            bwd_chunk<DT, NS>(v, gv, sdq, sq, dead, p.ste, want_gx, want_T, gxo, T);
+            if (want_gx) scale_ratios<NS>(sdq, sq, dead, rho);
+            bwd_chunk<DT, NS>(v, gv, sq, rho, dead, p.ste, want_gx, want_T, gxo, T);
             if (want_gx && valid) store_chunk<DT>(p.gx, off[j], gxo);
             if (want_T) {
 #pragma unroll
@@ -371,14 +490,16 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams
     }
     if (threadIdx.x != 0) return;
     const float c = p.crs ? __ldg(p.crs + j) : 1.0f;
+    const float rc = rcp_approx(c);
     df Q = {0.0f, 0.0f};
     for (int k = 0; k < K; ++k) {
         const float d = p.dgs ? __ldg(p.dgs + j * K + k) : 1.0f;
-        const df qk = df_div_f(df{res_h[k], res_l[k]}, d);
-        if (p.gdgs) p.gdgs[j * K + k] = -__fmul_rn(df_to_f(qk), __frcp_rn(__fmul_rn(c, d)));
+        const float rd = rcp_approx(d);
+        const df qk = df_div_f(df{res_h[k], res_l[k]}, d, rd);
+        if (p.gdgs) p.gdgs[j * K + k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
         Q = df_add(Q, qk);
     }
-    if (p.gcrs) p.gcrs[j] = -df_to_f(df_div_f(df_div_f(Q, c), c));
+    if (p.gcrs) p.gcrs[j] = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
 }
 
 // ---------------------------------------------------------------------------

@@ -1,0 +1,99 @@
+"""Run one kernel of the fake-quantizer on one tensor of a workload, for
+profiler captures (ncu) of a single launch on a case of known size.
+
+  python -m paper_2608_01847_gb300.profile_case --phase bwd --workload qwen3_4b_layer \
+      --tensor gate_proj --fmt nvfp4 --launches 3
+
+Draws the tensor on the GPU (seeded, same recipe as the benchmark), runs the
+phase `--launches` times and prints the CUDA-event time per launch and the
+algorithmic bytes it moves.  Not a benchmark: the numbers it prints are for
+orientation only.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def bytes_per_elem(phase, fmt, sub, shared, gx=True):
+    B = 32 if fmt == "mxfp4" else 16
+    coef = 0.0 if shared else 4 / B + 4 / sub
+    return {"alpha": 2.0, "fwd": 4 + coef, "pack": 2 + coef + 0.5 + 1 / B,
+            "bwd": 4 + (2 if gx else 0) + 2 * coef}[phase]
+
+
+def main():
+    import torch
+
+    from paper_2608_01847_gb300 import build as B
+    from paper_2608_01847_gb300 import focus as F
+    from paper_2608_01847_gb300 import workloads as W
+
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--phase", choices=["alpha", "fwd", "bwd", "pack"], default="bwd")
+    ap.add_argument("--workload", default="qwen3_4b_layer")
+    ap.add_argument("--tensor", default="gate_proj")
+    ap.add_argument("--fmt", choices=["mxfp4", "nvfp4"], default="nvfp4")
+    ap.add_argument("--sub", type=int, default=8)
+    ap.add_argument("--shared", action="store_true")
+    ap.add_argument("--no-gx", action="store_true")
+    ap.add_argument("--launches", type=int, default=3)
+    a = ap.parse_args()
+
+    B.build()
+    F.lib()
+    w = W.WORKLOADS[a.workload]
+    idx = [t.name for t in w.tensors].index(a.tensor)
+    fmt = F.FOCUS_MXFP4 if a.fmt == "mxfp4" else F.FOCUS_NVFP4
+    blk = F.block_of(fmt)
+    x, g = W.device_tensor(w, idx, "cuda")
+    crs, dgs = W.device_coefs(w, idx, blk, a.sub, "cuda", shared=a.shared)
+    alpha = F.focus_nvfp4_alpha(x)
+    y = torch.empty_like(x)
+    gx = None if a.no_gx else torch.empty_like(x)
+    gc, gd = torch.empty_like(crs), torch.empty_like(dgs)
+    rows, cols = x.shape
+    codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device="cuda")
+    sb = torch.empty((rows, cols // blk), dtype=torch.uint8, device="cuda")
+    desc = F.make_desc(x, fmt, a.sub, a.shared)
+    ws = torch.empty(max(16, F.focus_workspace_bytes(desc, F.FOCUS_WS_BWD),
+                         F.focus_workspace_bytes(desc, F.FOCUS_WS_ALPHA)),
+                     dtype=torch.uint8, device="cuda")
+
+    def run():
+        if a.phase == "alpha":
+            F.focus_nvfp4_alpha(x, alpha, ws)
+        elif a.phase == "fwd":
+            F.focus_fq_fwd(x, fmt, crs, dgs, alpha, sub_block=a.sub, shared=a.shared, y=y)
+        elif a.phase == "pack":
+            F.focus_pack(x, fmt, crs, dgs, alpha, sub_block=a.sub, shared=a.shared, codes=codes,
+                         scale_bytes=sb)
+        else:
+            F.focus_fq_bwd(x, g, fmt, crs, dgs, alpha, sub_block=a.sub, shared=a.shared, gx=gx,
+                           want_gx=not a.no_gx, gcrs=gc, gdgs=gd, ws=ws)
+
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(a.launches):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        run()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    n = rows * cols
+    bpe = bytes_per_elem(a.phase, a.fmt, a.sub, a.shared, not a.no_gx)
+    print(json.dumps({"phase": a.phase, "tensor": f"{a.workload}/{a.tensor}", "shape": [rows, cols],
+                      "fmt": a.fmt, "sub": a.sub, "shared": a.shared, "ms": times,
+                      "algorithmic_bytes": n * bpe,
+                      "gbs_last": n * bpe / (times[-1] * 1e-3) / 1e9}))
+
+
+if __name__ == "__main__":
+    main()
