@@ -6,7 +6,9 @@ alpha), per-block CRS and per-sub-block (8) DGS coefficients:
   alpha (per tensor)  ->  fake-quant forward  ->  STE backward (input
   gradient + both coefficient gradients)  ->  export pack,
 each phase over all 7 tensors before the next (as a calibration step runs
-all forwards, then all backwards), inputs resident in HBM.  `value` is the
+all forwards, then all backwards), inputs resident in HBM.  Each phase is
+captured once as a CUDA graph (its 7 tensors on parallel branches) and a
+step replays the four graphs in order.  `value` is the
 algorithmic bytes of the step (per-element figures below) over the step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
@@ -159,6 +161,31 @@ PHASES = [("alpha", phase_alpha), ("fwd", phase_fwd), ("bwd", phase_bwd), ("pack
 LAUNCHES_PER_TENSOR = {"alpha": 2, "fwd": 1, "bwd": 1, "pack": 1}
 
 
+class PhaseGraph:
+    """One phase (alpha, fwd, bwd or pack over all 7 tensors) captured as a
+    CUDA graph whose 7 tensors run on parallel branches (one stream each), so
+    small tensors fill the GPU alongside large ones."""
+
+    def __init__(self, fn, layers, device):
+        import torch
+        self.graph = torch.cuda.CUDAGraph()
+        side = [torch.cuda.Stream(device) for _ in layers]
+        cap = torch.cuda.Stream(device)
+        cap.wait_stream(torch.cuda.current_stream(device))
+        with torch.cuda.graph(self.graph, stream=cap):
+            main = torch.cuda.current_stream(device)
+            for L, st in zip(layers, side):
+                st.wait_stream(main)
+                with torch.cuda.stream(st):
+                    fn([L])
+            for st in side:
+                main.wait_stream(st)
+        torch.cuda.current_stream(device).wait_stream(cap)
+
+    def replay(self):
+        self.graph.replay()
+
+
 def gpu_arm(args, rank, world, device):
     import torch
     import torch.distributed as dist
@@ -172,13 +199,15 @@ def gpu_arm(args, rank, world, device):
     stream = torch.cuda.current_stream(device)
     torch.cuda.synchronize(device)
 
-    def step(ev=None):
-        for k, (name, fn) in enumerate(PHASES):
-            if ev is not None:
-                ev[name][0].record(stream)
-            fn(layers)
-            if ev is not None:
-                ev[name][1].record(stream)
+    # eager warm-up (resolves launch configurations), then capture one step
+    for name, fn in PHASES:
+        fn(layers)
+    torch.cuda.synchronize(device)
+    graphs = [(name, PhaseGraph(fn, layers, device)) for name, fn in PHASES]
+
+    def step():
+        for _, gph in graphs:
+            gph.replay()
 
     for _ in range(args.warmup):
         step()
@@ -189,22 +218,27 @@ def gpu_arm(args, rank, world, device):
             dist.barrier()
         torch.cuda.synchronize(device)
 
-    # ---- device-resident timing: whole steps + per-phase events ----
+    # ---- device-resident timing: K graph replays; per-phase events ----
     phase_ms = {n: 0.0 for n, _ in PHASES}
     with ClockSampler(device.index if device.index is not None else 0) as clk:
         barrier()
         start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for n, _ in PHASES} for _ in range(args.steps)]
         start.record(stream)
         for k in range(args.steps):
-            step(evs[k])
+            step()
         end.record(stream)
         barrier()
     total_ms = start.elapsed_time(end)
-    for ev in evs:
-        for n, _ in PHASES:
-            phase_ms[n] += ev[n][0].elapsed_time(ev[n][1])
+    # phase split: each phase graph replayed on its own, timed the same way
+    n_split = max(1, min(args.steps, 100))
+    for name, gph in graphs:
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_split):
+            gph.replay()
+        b.record(stream)
+        torch.cuda.synchronize(device)
+        phase_ms[name] = a.elapsed_time(b) * args.steps / n_split
     if world > 1:
         t = torch.tensor([total_ms], dtype=torch.float64, device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
