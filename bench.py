@@ -47,6 +47,23 @@ BYTES_PER_ELEM = {
 }
 STEP_BYTES_PER_ELEM = sum(BYTES_PER_ELEM.values())
 
+# DRAM traffic (read + write) of one backward phase (7 launches) of this
+# benchmark, from an ncu launch list (gpu__time_duration, dram__bytes_read,
+# dram__bytes_write; --cache-control none), and the sha256 prefix of the
+# kernel sources it was taken on.  Reported only while they are unchanged.
+BWD_TRAFFIC = {"sources": "7f8d1d796e157d46", "bytes_per_step": 762.1e6}
+
+
+def kernel_sources_sha() -> str:
+    import glob
+    import hashlib
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2608_01847_gb300", "csrc", "*"))):
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -432,7 +449,11 @@ def main():
         "phase_ms": {n: round(v, 4) for n, v in ph.items()},
         "roofline": {"bound": "hbm", "kernel": f"fq_{dom}", "achieved": round(achieved, 2),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
-                     "frac": round(achieved / peak, 4), "traffic": None},
+                     "frac": round(achieved / peak, 4),
+                     "traffic": (BWD_TRAFFIC["bytes_per_step"]
+                                 if dom == "bwd" and kernel_sources_sha() == BWD_TRAFFIC["sources"]
+                                 else None),
+                     "traffic_unit": "bytes per phase (7 launches)"},
         "clocks": r["clocks"],
         "e2e": {"value": round(world * step_bytes / (r["e2e_ms"] * 1e-3) / 1e9, 2), "unit": "GB/s",
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
