@@ -25,8 +25,9 @@
  *   synchronises the host: work is enqueued on `stream` (NULL = the legacy
  *   default stream) and completes asynchronously.
  * - x, y, g and gx are row-major [rows, ld] arrays of desc->dtype; only the
- *   first `cols` elements of each row are read or written.  They must be
- *   16-byte aligned, and ld must be a multiple of 8 elements.
+ *   first `cols` elements of each row are read or written.  Every row must
+ *   start on a 32-byte boundary: the arrays 32-byte aligned (16 bytes suffice
+ *   for the alpha pass) and ld * sizeof(element) a multiple of 32.
  * - Coefficient arrays are dense fp32: crs / gcrs are [rows, cols/block] and
  *   dgs / gdgs are [rows, cols/sub_block]; with coef_shared_rows = 1 both are
  *   a single row ([cols/block], [cols/sub_block]) shared by all rows.  They
@@ -34,7 +35,7 @@
  * - Scale bytes are dense uint8 [rows, cols/block] (E8M0 biased exponent for
  *   MXFP4, E4M3FN for NVFP4).  Codes are dense uint8 [rows, cols/2]: element
  *   2t of a row in the low nibble of byte t, element 2t+1 in the high nibble;
- *   a code is sign(1) | E2M1 magnitude index(3).  Codes must be 4-byte aligned.
+ *   a code is sign(1) | E2M1 magnitude index(3).  Codes must be 16-byte aligned.
  * - Every call returns FOCUS_OK (0) or a negative focus_status_t.  Argument
  *   errors are detected on the host before anything is launched; a launch
  *   failure is reported as FOCUS_ERR_CUDA (cudaGetLastError is consumed).

@@ -42,7 +42,8 @@ int check_desc(const focus_desc_t* d, bool method)
     if (d->rows < 0 || d->cols < 0 || d->ld < d->cols || d->ld < 0) return FOCUS_ERR_INVALID_ARG;
     if (d->dtype != FOCUS_F32 && d->dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
     if (d->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
-    if (d->ld % 8 != 0) return FOCUS_ERR_MISALIGNED;
+    // rows start on 32-byte boundaries (256-bit accesses)
+    if ((d->ld * (d->dtype == FOCUS_BF16 ? 2 : 4)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
     if (d->rows > 0 && d->cols > 0 && d->rows > kMaxChunks / (d->cols / 8)) return FOCUS_ERR_UNSUPPORTED;
     if (!method) return FOCUS_OK;
     if (d->fmt != FOCUS_MXFP4 && d->fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;
@@ -67,6 +68,11 @@ KParams make_params(const focus_desc_t* d)
     p.rows = static_cast<uint32_t>(d->rows);
     p.n_chunks = static_cast<uint32_t>(d->rows * (d->cols / 8));
     p.div_cpr = make_fastdiv(p.cpr > 0 ? p.cpr : 1u);
+    const int B = d->fmt == FOCUS_NVFP4 ? 16 : 32;
+    p.bpr = static_cast<uint32_t>(d->cols / B);
+    p.n_blocks = static_cast<uint32_t>(d->rows * (d->cols / B));
+    p.div_bpr = make_fastdiv(p.bpr > 0 ? p.bpr : 1u);
+    p.tx = shared_tx(p.bpr);
     p.strided = d->ld != d->cols;
     p.shared = d->coef_shared_rows;
     p.ste = d->ste;
@@ -94,8 +100,8 @@ int check_coef_ptrs(const float* a, const float* b, const float* c, const float*
 size_t bwd_ws_bytes(const focus_desc_t* d)
 {
     if (!d->coef_shared_rows || d->rows == 0 || d->cols == 0) return 0;
-    const uint32_t cpr = static_cast<uint32_t>(d->cols / 8);
-    const uint32_t ny = shared_row_groups(static_cast<uint32_t>(d->rows), cpr, d->dtype);
+    const uint32_t bpr = static_cast<uint32_t>(d->cols / d->block);
+    const uint32_t ny = shared_row_groups(static_cast<uint32_t>(d->rows), bpr);
     return static_cast<size_t>(ny) * static_cast<size_t>(d->cols / d->sub_block) * 2 * sizeof(float);
 }
 
@@ -157,7 +163,7 @@ FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float*
     if (rc) return rc;
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !y || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 16) || misaligned(y, 16) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if (misaligned(x, 32) || misaligned(y, 32) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
     p.x = x;
@@ -179,7 +185,7 @@ FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* c
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !codes || !scale_bytes || (desc->fmt == FOCUS_NVFP4 && !alpha))
         return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 16) || misaligned(codes, 4) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if (misaligned(x, 32) || misaligned(codes, 16) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
     p.x = x;
@@ -201,7 +207,7 @@ FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float*
     if (rc) return rc;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool want_T = gcrs != nullptr || gdgs != nullptr;
-    if (misaligned(x, 16) || misaligned(g, 16) || misaligned(gx, 16) || misaligned(alpha, 4))
+    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4))
         return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
     if (desc->rows == 0 || desc->cols == 0) {
@@ -233,7 +239,7 @@ FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float*
         if (misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
         p.ws = static_cast<float*>(ws);
         p.nsub = static_cast<uint32_t>(desc->cols / sub);
-        const uint32_t ny = shared_row_groups(p.rows, p.cpr, desc->dtype);
+        const uint32_t ny = shared_row_groups(p.rows, p.bpr);
         return map_cuda(launch_bwd_shared(desc->fmt, desc->dtype, sub, p, ny, st));
     }
     return map_cuda(launch_bwd(desc->fmt, desc->dtype, sub, p, st));

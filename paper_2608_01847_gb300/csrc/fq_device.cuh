@@ -294,6 +294,89 @@ __device__ __forceinline__ df shfl_xor_df(df a, int o)
 }
 
 // ---------------------------------------------------------------------------
+// Packed binary32 pairs (sm_100-family f32x2 instructions): each lane is an
+// ordinary IEEE round-to-nearest operation, two lanes per instruction.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 mul2(float2 a, float2 b)
+{
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rr;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rr, ra, rb;\n\tmov.b64 {%0, %1}, rr;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+__device__ __forceinline__ float2 add2(float2 a, float2 b)
+{
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rr;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rr, ra, rb;\n\tmov.b64 {%0, %1}, rr;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+__device__ __forceinline__ float2 sub2(float2 a, float2 b)
+{
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rr;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "sub.rn.f32x2 rr, ra, rb;\n\tmov.b64 {%0, %1}, rr;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c)
+{
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rc, rr;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rr, ra, rb, rc;\n\tmov.b64 {%0, %1}, rr;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return r;
+}
+
+// Two interleaved Sum2 accumulators (even and odd terms of a sum) in one
+// packed pair each: s holds the running sums, c the accumulated errors.
+struct Sum2x2 {
+    float2 s, c;
+};
+
+__device__ __forceinline__ void sum2x2_add(Sum2x2& a, float2 p)
+{
+    const float2 s = add2(a.s, p);
+    const float2 bb = sub2(s, a.s);
+    const float2 e = add2(sub2(a.s, sub2(s, bb)), sub2(p, bb));
+    a.s = s;
+    a.c = add2(a.c, e);
+}
+
+// ---------------------------------------------------------------------------
+// 256-bit global accesses (sm_100 family): one 32-byte sector per lane.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void ld_v8(uint32_t (&w)[8], const void* p)
+{
+    asm("ld.global.nc.L1::no_allocate.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+        : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]),
+          "=r"(w[7])
+        : "l"(p));
+}
+
+__device__ __forceinline__ void st_v8(void* p, const uint32_t (&w)[8])
+{
+    asm volatile("st.global.cs.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};"
+                 :
+                 : "l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]),
+                   "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+
+// ---------------------------------------------------------------------------
 // Global memory: one "chunk" is 8 consecutive elements of a row (16 B bf16,
 // 32 B fp32), read with 128-bit non-coherent loads.
 // ---------------------------------------------------------------------------
@@ -351,38 +434,6 @@ __device__ __forceinline__ void store_chunk(void* base, uint64_t off, const floa
                              __float_as_uint(v[2]), __float_as_uint(v[3])));
         __stcs(p + 1, make_uint4(__float_as_uint(v[4]), __float_as_uint(v[5]),
                                  __float_as_uint(v[6]), __float_as_uint(v[7])));
-    }
-}
-
-// N consecutive fp32 coefficients (N = 1, 2 or 4), one vector load.
-template <int N>
-__device__ __forceinline__ void load_coefs(const float* p, float (&d)[N])
-{
-    if (N == 1) {
-        d[0] = __ldg(p);
-    } else if (N == 2) {
-        const float2 v = __ldg(reinterpret_cast<const float2*>(p));
-        d[0] = v.x;
-        d[N > 1 ? 1 : 0] = v.y;
-    } else {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(p));
-        d[0] = v.x;
-        d[N > 1 ? 1 : 0] = v.y;
-        d[N > 2 ? 2 : 0] = v.z;
-        d[N > 3 ? 3 : 0] = v.w;
-    }
-}
-
-template <int N>
-__device__ __forceinline__ void store_coefs(float* p, const float (&d)[N])
-{
-    if (N == 1) {
-        p[0] = d[0];
-    } else if (N == 2) {
-        *reinterpret_cast<float2*>(p) = make_float2(d[0], d[N > 1 ? 1 : 0]);
-    } else {
-        *reinterpret_cast<float4*>(p) =
-            make_float4(d[0], d[N > 1 ? 1 : 0], d[N > 2 ? 2 : 0], d[N > 3 ? 3 : 0]);
     }
 }
 

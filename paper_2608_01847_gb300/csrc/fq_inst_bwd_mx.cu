@@ -6,12 +6,11 @@ namespace focus {
 template <int FMT, int DT, int SUB>
 cudaError_t run_bwd_shared(const KParams& p, uint32_t ny, cudaStream_t st)
 {
-    const dim3 grid(shared_col_ctas(p.cpr), ny);
+    const dim3 grid(shared_col_ctas(p.bpr), ny);
     fq_bwd_shared_kernel<FMT, DT, SUB><<<grid, kThreads, 0, st>>>(p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || (p.gcrs == nullptr && p.gdgs == nullptr)) return e;
-    const uint32_t nblk = p.cpr / (Geo<FMT, SUB>::LPB);
-    fq_bwd_shared_finalize<FMT, SUB><<<nblk, kThreads, 0, st>>>(p, ny);
+    fq_bwd_shared_finalize<FMT, SUB><<<p.bpr, kThreads, 0, st>>>(p, ny);
     return cudaGetLastError();
 }
 

@@ -1,13 +1,13 @@
 // fq_kernels.cuh -- CUDA kernels of the FOCUS FP4 fake-quantizer (sm_103a).
 //
-// Work decomposition.  A row of `cols` elements is split into chunks of 8
-// consecutive elements (one 128-bit load in bf16).  One thread owns one chunk
-// at a time; the B/8 lanes that hold one hardware block (4 for MXFP4's 32, 2
-// for NVFP4's 16) are adjacent lanes of a warp, so the block absmax and the
-// per-block coefficient-gradient sums are warp shuffles -- no shared memory,
-// no atomics.  The streaming kernels walk a linear chunk index with a
-// grid-stride loop sized to the resident CTAs, U chunks per thread per step
-// with all loads issued before any arithmetic.
+// Work decomposition.  One thread owns one hardware block at a time (B = 32
+// elements for MXFP4, 16 for NVFP4, contiguous along a row): its absmax, its
+// scale, its coefficients and its coefficient gradients are computed once,
+// in registers, with no shuffles.  A block of bf16 is one (NVFP4) or two
+// (MXFP4) 256-bit loads, i.e. exactly one 32-byte sector per lane per load.
+// The streaming kernels walk a linear block index with a grid-stride loop
+// sized to the resident CTAs, issuing every load of a step before any
+// arithmetic; pairs of elements go through the packed f32x2 instructions.
 //
 // Per element the arithmetic is the paper's, in this order (Sec. 3.1-3.4):
 //   m      = block absmax                       (Eq. 2-3)
@@ -42,27 +42,139 @@ struct KParams {
     uint8_t* scales;
     float* ws;            // scratch: per-CTA partials
     uint64_t ld;          // row pitch of x / y / g / gx in elements
-    uint32_t n_chunks;    // rows * cols / 8
-    uint32_t cpr;         // chunks per row = cols / 8
+    uint32_t n_chunks;    // rows * cols / 8 (alpha pass)
+    uint32_t cpr;         // 8-element chunks per row
     FastDiv div_cpr;
+    uint32_t n_blocks;    // rows * cols / B
+    uint32_t bpr;         // hardware blocks per row = cols / B
+    FastDiv div_bpr;
     uint32_t rows;
     uint32_t nsub;        // sub-blocks per row = cols / sub_block
+    uint32_t tx;          // shared-row backward: block columns per CTA
     int strided;          // ld != cols
     int shared;           // one coefficient set for all rows
     int ste;              // 0 identity, 1 clipped
     int mx_rule;          // 0 ceiling, 1 OCP floor
 };
 
-template <int FMT, int SUB>
+template <int FMT, int DT, int SUB>
 struct Geo {
-    static constexpr int B = FMT == 0 ? 32 : 16;  // hardware block (Sec. 3.1)
-    static constexpr int LPB = B / 8;             // lanes per block
-    static constexpr int NS = SUB < 8 ? 8 / SUB : 1;   // sub-blocks per chunk
-    static constexpr int LPS = SUB > 8 ? SUB / 8 : 1;  // lanes per sub-block
-    static constexpr int EPS = 8 / NS;                 // chunk elements per sub-block
+    static constexpr int B = FMT == 0 ? 32 : 16;   // hardware block (Sec. 3.1)
+    static constexpr int K = B / SUB;              // sub-blocks per block (Sec. 3.4)
+    static constexpr int W = DT == 1 ? B / 2 : B;  // 32-bit words of a block of x
     static_assert(SUB >= 2 && SUB <= B && B % SUB == 0, "sub-block must divide the block");
 };
 
+// ---------------------------------------------------------------------------
+// block I/O
+// ---------------------------------------------------------------------------
+template <int W>
+__device__ __forceinline__ void load_block(uint32_t (&w)[W], const void* base, uint64_t byte_off)
+{
+    const char* p = static_cast<const char*>(base) + byte_off;
+#pragma unroll
+    for (int i = 0; i < W / 8; ++i) {
+        uint32_t t[8];
+        ld_v8(t, p + 32 * i);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[8 * i + k] = t[k];
+    }
+}
+
+template <int W>
+__device__ __forceinline__ void store_block(void* base, uint64_t byte_off, const uint32_t (&w)[W])
+{
+    char* p = static_cast<char*>(base) + byte_off;
+#pragma unroll
+    for (int i = 0; i < W / 8; ++i) {
+        uint32_t t[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t[k] = w[8 * i + k];
+        st_v8(p + 32 * i, t);
+    }
+}
+
+// Elements 2i and 2i+1 of a block as binary32 (exact).
+template <int DT>
+__device__ __forceinline__ float2 elem_pair(const uint32_t* w, int i)
+{
+    if (DT == 1) return make_float2(bf16_lo(w[i]), bf16_hi(w[i]));
+    return make_float2(__uint_as_float(w[2 * i]), __uint_as_float(w[2 * i + 1]));
+}
+
+// Store a pair of results in the block's output words (bf16 round to
+// nearest even, or binary32 as is).
+template <int DT>
+__device__ __forceinline__ void put_pair(uint32_t* w, int i, float2 v)
+{
+    if (DT == 1) {
+        w[i] = pack_bf16x2(v.x, v.y);
+    } else {
+        w[2 * i] = __float_as_uint(v.x);
+        w[2 * i + 1] = __float_as_uint(v.y);
+    }
+}
+
+// max |x| over a block, read off the stored bits (non-negative floats order
+// like their encodings): packed u16x2 maxima for bf16, u32 for binary32.
+template <int DT, int W>
+__device__ __forceinline__ float block_absmax(const uint32_t (&w)[W])
+{
+    if (DT == 1) {
+        uint32_t m = w[0] & 0x7fff7fffu;
+#pragma unroll
+        for (int i = 1; i < W; ++i) {
+            const uint32_t a = w[i] & 0x7fff7fffu;
+            asm("max.u16x2 %0, %0, %1;" : "+r"(m) : "r"(a));
+        }
+        return __uint_as_float(max(m << 16, m & 0xffff0000u));
+    }
+    uint32_t m = w[0] & 0x7fffffffu;
+#pragma unroll
+    for (int i = 1; i < W; ++i) m = max(m, w[i] & 0x7fffffffu);
+    return __uint_as_float(m);
+}
+
+// N consecutive fp32 coefficients (N = 1, 2, 4, 8, 16), vector loads.
+template <int N>
+__device__ __forceinline__ void load_coefs(const float* p, float (&d)[N])
+{
+    if constexpr (N == 1) {
+        d[0] = __ldg(p);
+    } else if constexpr (N == 2) {
+        const float2 v = __ldg(reinterpret_cast<const float2*>(p));
+        d[0] = v.x;
+        d[1] = v.y;
+    } else {
+#pragma unroll
+        for (int i = 0; i < N / 4; ++i) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(p) + i);
+            d[4 * i] = v.x;
+            d[4 * i + 1] = v.y;
+            d[4 * i + 2] = v.z;
+            d[4 * i + 3] = v.w;
+        }
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void store_coefs(float* p, const float (&d)[N])
+{
+    if constexpr (N == 1) {
+        p[0] = d[0];
+    } else if constexpr (N == 2) {
+        *reinterpret_cast<float2*>(p) = make_float2(d[0], d[1]);
+    } else {
+#pragma unroll
+        for (int i = 0; i < N / 4; ++i)
+            reinterpret_cast<float4*>(p)[i] =
+                make_float4(d[4 * i], d[4 * i + 1], d[4 * i + 2], d[4 * i + 3]);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// block scale (Eq. 2-3) and relaxed scales (Eq. 6, 8)
+// ---------------------------------------------------------------------------
 // Per-tensor constants of the block-scale step: NVFP4's alpha, fl(alpha * 6)
 // and the bracket of its reciprocal.
 struct TensorScale {
@@ -85,8 +197,6 @@ template <int FMT>
 __device__ __forceinline__ float block_scale(float m, const TensorScale& ts, int mx_rule,
                                              uint32_t& byte)
 {
-#pragma unroll
-    for (int o = 1; o < (FMT == 0 ? 4 : 2); o <<= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, o));
     if (FMT == 0) {
         const int e = mx_exponent_fast(m, mx_rule);
         byte = static_cast<uint32_t>(e + 127);
@@ -95,270 +205,340 @@ __device__ __forceinline__ float block_scale(float m, const TensorScale& ts, int
     return nv_scale(m, ts.alpha, ts.den, ts.bd, byte);
 }
 
-__device__ __forceinline__ float chunk_absmax(const float (&v)[8])
-{
-    float m = 0.0f;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(v[e]));
-    return m;
-}
-
-// Relaxed quantization scale per sub-block of the chunk; "dead" when S^dq or
-// S^q is zero or infinite (outputs +0, no gradient).
-template <int NS>
-__device__ __forceinline__ void relaxed_scales(float sdq, float c, const float (&d)[NS],
-                                               float (&sq)[NS], bool (&dead)[NS])
+// S^q per sub-block; "dead" when S^dq or S^q is zero or infinite (outputs
+// +0, no gradient).
+template <int K>
+__device__ __forceinline__ void relaxed_scales(float sdq, float c, const float (&d)[K],
+                                               float (&sq)[K], bool (&dead)[K])
 {
 #pragma unroll
-    for (int t = 0; t < NS; ++t) {
-        sq[t] = __fmul_rn(sdq, __fmul_rn(c, d[t]));
-        dead[t] = (sdq == 0.0f) || (sq[t] == 0.0f) || isinf(sq[t]);
+    for (int k = 0; k < K; ++k) {
+        sq[k] = __fmul_rn(sdq, __fmul_rn(c, d[k]));
+        dead[k] = (sdq == 0.0f) | (sq[k] == 0.0f) | isinf(sq[k]);
     }
 }
 
-// Nibble mask of the live sub-blocks of a chunk (4 bits per element).
-template <int NS>
-__device__ __forceinline__ uint32_t live_nibbles(const bool (&dead)[NS])
+// Nibble mask (4 bits per element) of the live elements of code word w.
+template <int SUB, int K>
+__device__ __forceinline__ uint32_t live_word(const bool (&dead)[K], int w)
 {
-    constexpr int EPS = 8 / NS;
-    constexpr uint32_t sub_mask = EPS == 8 ? 0xffffffffu : ((1u << (4 * EPS)) - 1u);
-    uint32_t m = 0u;
+    if constexpr (SUB >= 8) {
+        return dead[(8 * w) / SUB] ? 0u : 0xffffffffu;
+    } else {
+        constexpr uint32_t sub_mask = (1u << (4 * SUB)) - 1u;
+        uint32_t m = 0u;
 #pragma unroll
-    for (int t = 0; t < NS; ++t) m |= dead[t] ? 0u : (sub_mask << (4 * EPS * t));
-    return m;
+        for (int t = 0; t < 8 / SUB; ++t)
+            m |= dead[(8 * w) / SUB + t] ? 0u : (sub_mask << (4 * SUB * t));
+        return m;
+    }
 }
 
-// E2M1 codes (Eq. 1) of u = fl(x / S^q) for the eight elements of a chunk,
-// exact: both brackets of every quotient (see make_bracket) are converted,
-// and when the two code words differ on a live element the quotients are
-// recomputed by IEEE division.  Dead sub-blocks get code 0.
-template <int NS>
-__device__ __forceinline__ uint32_t chunk_codes(const float (&v)[8], const float (&sq)[NS],
-                                                const bool (&dead)[NS])
+// E2M1 codes (Eq. 1) of u = fl(x / S^q) for a whole block, exact: both
+// brackets of every quotient (see make_bracket) are converted; where the two
+// code words differ on a live element, the block's quotients are recomputed
+// by IEEE division.  Dead sub-blocks get code 0.  codes[w] holds elements
+// 8w .. 8w+7, element 8w+2t in the low nibble of byte t.
+template <int DT, int B, int K>
+__device__ __forceinline__ void block_codes(const uint32_t* xw, const float (&sq)[K],
+                                            const bool (&dead)[K], uint32_t (&codes)[B / 8])
 {
-    constexpr int EPS = 8 / NS;
-    Bracket br[NS];
+    constexpr int SUB = B / K;
+    Bracket br[K];
     bool ok = true;
 #pragma unroll
-    for (int t = 0; t < NS; ++t) {
-        br[t] = make_bracket(sq[t]);
-        ok = ok & (dead[t] | br[t].ok);
+    for (int k = 0; k < K; ++k) {
+        br[k] = make_bracket(sq[k]);
+        ok = ok & (dead[k] | br[k].ok);
     }
-    float lo[8], hi[8];
+    uint32_t diff = 0u;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        lo[e] = __fmul_rn(v[e], br[e / EPS].lo);
-        hi[e] = __fmul_rn(v[e], br[e / EPS].hi);
-    }
-    const uint32_t live = live_nibbles<NS>(dead);
-    uint32_t c = e2m1_pack8(lo);
-    if (!ok | (((c ^ e2m1_pack8(hi)) & live) != 0u)) {
-        float u[8];
+    for (int w = 0; w < B / 8; ++w) {
+        float lo[8], hi[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) u[e] = __fdiv_rn(v[e], sq[e / EPS]);
-        c = e2m1_pack8(u);
+        for (int e = 0; e < 8; e += 2) {
+            const int k = (8 * w + e) / SUB;
+            const float2 x2 = elem_pair<DT>(xw, (8 * w + e) / 2);
+            const float2 l2 = mul2(x2, make_float2(br[k].lo, br[k].lo));
+            const float2 h2 = mul2(x2, make_float2(br[k].hi, br[k].hi));
+            lo[e] = l2.x;
+            lo[e + 1] = l2.y;
+            hi[e] = h2.x;
+            hi[e + 1] = h2.y;
+        }
+        codes[w] = e2m1_pack8(lo);
+        diff |= (codes[w] ^ e2m1_pack8(hi)) & live_word<SUB, K>(dead, w);
     }
-    return c & live;
+    if (!ok | (diff != 0u)) {
+#pragma unroll
+        for (int w = 0; w < B / 8; ++w) {
+            float u[8];
+#pragma unroll
+            for (int e = 0; e < 8; e += 2) {
+                const int k = (8 * w + e) / SUB;
+                const float2 x2 = elem_pair<DT>(xw, (8 * w + e) / 2);
+                u[e] = __fdiv_rn(x2.x, sq[k]);
+                u[e + 1] = __fdiv_rn(x2.y, sq[k]);
+            }
+            codes[w] = e2m1_pack8(u);
+        }
+    }
+#pragma unroll
+    for (int w = 0; w < B / 8; ++w) codes[w] &= live_word<SUB, K>(dead, w);
 }
 
-// Clipping mask of the STE (|fl(x / S^q)| <= 6, live sub-blocks only),
-// decided on the brackets and exactly when they straddle 6.
-template <int NS>
-__device__ __forceinline__ void chunk_clip_mask(const float (&v)[8], const float (&sq)[NS],
-                                                const bool (&dead)[NS], bool (&live)[8])
+// Clipping mask of the STE (|fl(x / S^q)| <= 6 on live sub-blocks), decided
+// on the brackets and exactly when they straddle 6.  Bit e = element e.
+template <int DT, int B, int K>
+__device__ __forceinline__ uint32_t block_clip_mask(const uint32_t* xw, const float (&sq)[K],
+                                                    const bool (&dead)[K])
 {
-    constexpr int EPS = 8 / NS;
-    Bracket br[NS];
+    constexpr int SUB = B / K;
+    Bracket br[K];
 #pragma unroll
-    for (int t = 0; t < NS; ++t) br[t] = make_bracket(sq[t]);
+    for (int k = 0; k < K; ++k) br[k] = make_bracket(sq[k]);
+    uint32_t live = 0u;
     bool ambiguous = false;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const int t = e / EPS;
-        const float lo = fabsf(__fmul_rn(v[e], br[t].lo));
-        const float hi = fabsf(__fmul_rn(v[e], br[t].hi));
-        live[e] = !dead[t] & (hi <= 6.0f);
-        ambiguous = ambiguous | (!dead[t] & (!br[t].ok | ((lo <= 6.0f) != (hi <= 6.0f))));
+    for (int e = 0; e < B; e += 2) {
+        const int k = e / SUB;
+        const float2 x2 = elem_pair<DT>(xw, e / 2);
+        const float2 l2 = mul2(x2, make_float2(br[k].lo, br[k].lo));
+        const float2 h2 = mul2(x2, make_float2(br[k].hi, br[k].hi));
+        const bool a0 = fabsf(h2.x) <= 6.0f, a1 = fabsf(h2.y) <= 6.0f;
+        const bool b0 = fabsf(l2.x) <= 6.0f, b1 = fabsf(l2.y) <= 6.0f;
+        live |= ((!dead[k] & a0) ? 1u : 0u) << e;
+        live |= ((!dead[k] & a1) ? 1u : 0u) << (e + 1);
+        ambiguous = ambiguous | (!dead[k] & (!br[k].ok | (a0 != b0) | (a1 != b1)));
     }
     if (ambiguous) {
+        live = 0u;
 #pragma unroll
-        for (int e = 0; e < 8; ++e)
-            live[e] = !dead[e / EPS] & (fabsf(__fdiv_rn(v[e], sq[e / EPS])) <= 6.0f);
-    }
-}
-
-// STE backward of one chunk: input gradient g * rho (rho = S^dq / S^q of the
-// sub-block, Sec. 3.2; rho = 0 on dead sub-blocks, and the +0 addend turns
-// -0 into +0) and the per-sub-block Sum2 of mask*g*x.
-template <int DT, int NS>
-__device__ __forceinline__ void bwd_chunk(const float (&v)[8], const float (&gv)[8],
-                                          const float (&sq)[NS], const float (&rho)[NS],
-                                          const bool (&dead)[NS], int ste, bool want_gx,
-                                          bool want_T, float (&gxo)[8], df (&T)[NS])
-{
-    constexpr int EPS = 8 / NS;
-    if (ste == 1) {
-        bool live[8];
-        chunk_clip_mask<NS>(v, sq, dead, live);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int t = e / EPS;
-            if (want_gx) gxo[e] = live[e] ? __fmul_rn(gv[e], rho[t]) : 0.0f;
-            if (want_T) {
-                const float a = live[e] ? gv[e] : 0.0f;
-                const float p = __fmul_rn(a, v[e]);  // exact for bf16 inputs
-                if (e % EPS == 0) T[t] = {p, 0.0f};
-                else sum2_add(T[t], p);
-                if (DT == 0) T[t].l = __fadd_rn(T[t].l, __fmaf_rn(a, v[e], -p));
-            }
-        }
-        return;
-    }
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const int t = e / EPS;
-        if (want_gx) gxo[e] = __fmaf_rn(gv[e], rho[t], 0.0f);
-        if (want_T) {
-            const float p = __fmul_rn(gv[e], v[e]);  // exact for bf16 inputs
-            if (e % EPS == 0) T[t] = {p, 0.0f};
-            else sum2_add(T[t], p);
-            if (DT == 0) T[t].l = __fadd_rn(T[t].l, __fmaf_rn(gv[e], v[e], -p));
+        for (int e = 0; e < B; e += 2) {
+            const int k = e / SUB;
+            const float2 x2 = elem_pair<DT>(xw, e / 2);
+            live |= ((!dead[k] & (fabsf(__fdiv_rn(x2.x, sq[k])) <= 6.0f)) ? 1u : 0u) << e;
+            live |= ((!dead[k] & (fabsf(__fdiv_rn(x2.y, sq[k])) <= 6.0f)) ? 1u : 0u) << (e + 1);
         }
     }
-    if (want_T) {
-#pragma unroll
-        for (int t = 0; t < NS; ++t)
-            if (dead[t]) T[t] = {0.0f, 0.0f};
-    }
+    return live;
 }
 
 // Scale ratio rho = fl(S^dq / S^q) per sub-block (0 for dead sub-blocks).
-template <int NS>
-__device__ __forceinline__ void scale_ratios(float sdq, const float (&sq)[NS], const bool (&dead)[NS],
-                                             float (&rho)[NS])
+template <int K>
+__device__ __forceinline__ void scale_ratios(float sdq, const float (&sq)[K], const bool (&dead)[K],
+                                             float (&rho)[K])
 {
 #pragma unroll
-    for (int t = 0; t < NS; ++t) rho[t] = dead[t] ? 0.0f : __fdiv_rn(sdq, sq[t]);
+    for (int k = 0; k < K; ++k) rho[k] = dead[k] ? 0.0f : __fdiv_rn(sdq, sq[k]);
+}
+
+// Merge the two interleaved Sum2 chains of a sub-block into one pair.
+__device__ __forceinline__ df sum2x2_merge(const Sum2x2& a)
+{
+    const df s = two_sum(a.s.x, a.s.y);
+    return fast_two_sum(s.h, __fadd_rn(s.l, __fadd_rn(a.c.x, a.c.y)));
 }
 
 // ---------------------------------------------------------------------------
-// Forward / pack / per-row backward over a linear chunk index.
+// STE backward of one block, sub-block by sub-block: the input gradient
+// (stored one 256-bit group at a time as soon as it is complete), the
+// compensated sum T_k of mask*g*x (two interleaved Sum2 chains in a packed
+// pair), and the coefficient gradients
+//   gd_k = -(T_k / d_k) / (c d_k),   gc = -(sum_k T_k / d_k) / c^2,
+// with T_k / d_k in double-fp32 and the sum over k compensated.
 // ---------------------------------------------------------------------------
-template <int DT, int MODE>
+template <int DT, int B, int K>
+__device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw,
+                                          const float (&sq)[K], const bool (&dead)[K],
+                                          const float (&rho)[K], float c, const float (&d)[K],
+                                          int ste, bool want_gx, bool want_T, void* gx_base,
+                                          uint64_t off, float (&gd)[K], float& gc, df (&T)[K])
+{
+    constexpr int SUB = B / K;
+    constexpr int EPG = DT == 1 ? 16 : 8;  // elements per 256-bit group
+    const uint32_t live = (ste == 1) ? block_clip_mask<DT, B, K>(xw, sq, dead) : 0xffffffffu;
+    const float rc = rcp_approx(c);
+    df Q = {0.0f, 0.0f};
+    uint32_t grp[8];
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        Sum2x2 acc;
+#pragma unroll
+        for (int e = k * SUB; e < (k + 1) * SUB; e += 2) {
+            const float2 x2 = elem_pair<DT>(xw, e / 2);
+            float2 g2 = elem_pair<DT>(gw, e / 2);
+            if (ste == 1) {
+                g2.x = ((live >> e) & 1u) ? g2.x : 0.0f;
+                g2.y = ((live >> (e + 1)) & 1u) ? g2.y : 0.0f;
+            }
+            if (want_gx) {
+                // rho = 0 on dead sub-blocks; the +0 addend turns -0 into +0
+                put_pair<DT>(grp, (e % EPG) / 2,
+                             fma2(g2, make_float2(rho[k], rho[k]), make_float2(0.0f, 0.0f)));
+                if (e % EPG == EPG - 2) {
+                    st_v8(static_cast<char*>(gx_base) + off + (e / EPG) * 32, grp);
+                }
+            }
+            if (want_T) {
+                const float2 p = mul2(g2, x2);  // exact for bf16 inputs
+                if (e == k * SUB) {
+                    acc.s = p;
+                    acc.c = make_float2(0.0f, 0.0f);
+                } else {
+                    sum2x2_add(acc, p);
+                }
+                if (DT == 0) acc.c = add2(acc.c, fma2(g2, x2, make_float2(-p.x, -p.y)));
+            }
+        }
+        if (want_T) {
+            T[k] = dead[k] ? df{0.0f, 0.0f} : sum2x2_merge(acc);
+            const float rd = rcp_approx(d[k]);
+            const df qk = df_div_f(T[k], d[k], rd);
+            gd[k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
+            Q = (k == 0) ? qk : df_add(Q, qk);
+        }
+    }
+    gc = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
+}
+
+// Coefficient gradients from finished sub-block sums (the shared-row
+// finalisation): the same formulas as block_bwd.
+template <int K>
+__device__ __forceinline__ void block_coef_grads(const df (&T)[K], float c, const float (&d)[K],
+                                                 float (&gd)[K], float& gc)
+{
+    const float rc = rcp_approx(c);
+    df Q = {0.0f, 0.0f};
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        const float rd = rcp_approx(d[k]);
+        const df qk = df_div_f(T[k], d[k], rd);
+        gd[k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
+        Q = (k == 0) ? qk : df_add(Q, qk);
+    }
+    gc = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
+}
+
+// ---------------------------------------------------------------------------
+// Forward / pack / per-row backward over a linear block index.
+// ---------------------------------------------------------------------------
+template <int FMT, int DT, int MODE>
 struct Unroll {
-    static constexpr int U = DT == 1 ? (MODE == kBwd ? 2 : 4) : (MODE == kBwd ? 1 : 2);
+    // blocks per thread per step: 64 bytes of x in flight for the streaming
+    // passes, one block (x and g) for the backward
+    static constexpr int U = (MODE == kBwd) ? 1 : ((FMT == 1 && DT == 1) ? 2 : 1);
+};
+
+// Resident CTAs per SM the register allocation must allow: enough 256-thread
+// CTAs to keep >= 48 KB of loads in flight per SM.
+// (one fewer for 2-element sub-blocks, whose per-sub-block state is largest).
+template <int FMT, int SUB, int MODE>
+struct MinCtas {
+    static constexpr int value = ((MODE == kBwd) ? (FMT == 1 ? 3 : 2) : 4) - (SUB == 2 ? 1 : 0);
 };
 
 template <int FMT, int DT, int SUB, int MODE>
-__global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
+__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
+    fq_block_kernel(const KParams p)
 {
-    using G = Geo<FMT, SUB>;
-    constexpr int U = Unroll<DT, MODE>::U;
-    constexpr int NS = G::NS;
+    using G = Geo<FMT, DT, SUB>;
+    constexpr int B = G::B, K = G::K, W = G::W;
+    constexpr int U = Unroll<FMT, DT, MODE>::U;
+    constexpr int ESZ = DT == 1 ? 2 : 4;
     const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = (MODE == kBwd) && p.gx != nullptr;
     const bool want_T = (MODE == kBwd) && (p.gcrs != nullptr || p.gdgs != nullptr);
     const uint32_t span = U * kThreads;
 
-    for (uint32_t base = blockIdx.x * span; base < p.n_chunks; base += gridDim.x * span) {
-        ChunkRaw<DT> xr[U];
-        ChunkRaw<DT> gr[MODE == kBwd ? U : 1];
+    for (uint32_t base = blockIdx.x * span; base < p.n_blocks; base += gridDim.x * span) {
+        uint32_t xr[U][W];
+        uint32_t gr[MODE == kBwd ? U : 1][MODE == kBwd ? W : 1];
         uint64_t off[U];
         float cv[U];
-        float dv[U][NS];
+        float dv[U][K];
         // ---- issue every load of this step first ----
 #pragma unroll
         for (int j = 0; j < U; ++j) {
-            const uint32_t s = base + j * kThreads + threadIdx.x;
+            const uint32_t blk = base + j * kThreads + threadIdx.x;
             cv[j] = 1.0f;
 #pragma unroll
-            for (int t = 0; t < NS; ++t) dv[j][t] = 1.0f;
+            for (int k = 0; k < K; ++k) dv[j][k] = 1.0f;
             off[j] = 0;
-            if (s < p.n_chunks) {
-                uint32_t cc = 0;
+            if (blk < p.n_blocks) {
+                uint32_t cb = 0;
                 if (p.strided || p.shared) {
-                    const uint32_t row = fast_div(s, p.div_cpr);
-                    cc = s - row * p.cpr;
-                    off[j] = static_cast<uint64_t>(row) * p.ld + static_cast<uint64_t>(cc) * 8u;
+                    const uint32_t row = fast_div(blk, p.div_bpr);
+                    cb = blk - row * p.bpr;
+                    off[j] = (static_cast<uint64_t>(row) * p.ld + static_cast<uint64_t>(cb) * B) * ESZ;
                 } else {
-                    off[j] = static_cast<uint64_t>(s) * 8u;
+                    off[j] = static_cast<uint64_t>(blk) * (B * ESZ);
                 }
-                load_chunk<DT>(xr[j], p.x, off[j]);
-                if (MODE == kBwd) load_chunk<DT>(gr[j], p.g, off[j]);
-                const uint32_t q = p.shared ? cc : s;
-                if (p.crs) cv[j] = __ldg(p.crs + q / G::LPB);
-                if (p.dgs) {
-                    if (SUB <= 8) load_coefs<NS>(p.dgs + static_cast<size_t>(q) * NS, dv[j]);
-                    else dv[j][0] = __ldg(p.dgs + q / G::LPS);
-                }
+                load_block<W>(xr[j], p.x, off[j]);
+                if constexpr (MODE == kBwd) load_block<W>(gr[j], p.g, off[j]);
+                const uint32_t q = p.shared ? cb : blk;
+                if (p.crs) cv[j] = __ldg(p.crs + q);
+                if (p.dgs) load_coefs<K>(p.dgs + static_cast<size_t>(q) * K, dv[j]);
             } else {
-                zero_chunk<DT>(xr[j]);
-                if (MODE == kBwd) zero_chunk<DT>(gr[MODE == kBwd ? j : 0]);
+#pragma unroll
+                for (int i = 0; i < W; ++i) xr[j][i] = 0u;
+                if constexpr (MODE == kBwd) {
+#pragma unroll
+                    for (int i = 0; i < W; ++i) gr[j][i] = 0u;
+                }
             }
         }
         // ---- arithmetic and stores ----
 #pragma unroll
         for (int j = 0; j < U; ++j) {
-            const uint32_t s = base + j * kThreads + threadIdx.x;
-            const bool valid = s < p.n_chunks;
-            float v[8];
-            unpack_chunk<DT>(xr[j], v);
+            const uint32_t blk = base + j * kThreads + threadIdx.x;
+            if (blk >= p.n_blocks) continue;
             uint32_t sbyte;
-            const float sdq = block_scale<FMT>(chunk_absmax(v), ts, p.mx_rule, sbyte);
-            float sq[NS];
-            bool dead[NS];
-            relaxed_scales<NS>(sdq, cv[j], dv[j], sq, dead);
+            const float sdq = block_scale<FMT>(block_absmax<DT, W>(xr[j]), ts, p.mx_rule, sbyte);
+            float sq[K];
+            bool dead[K];
+            relaxed_scales<K>(sdq, cv[j], dv[j], sq, dead);
 
-            if (MODE != kBwd) {
-                const uint32_t codes = chunk_codes<NS>(v, sq, dead);
-                if (valid) {
-                    if (MODE == kFwd) {
+            if constexpr (MODE != kBwd) {
+                uint32_t codes[B / 8];
+                block_codes<DT, B, K>(xr[j], sq, dead, codes);
+                if constexpr (MODE == kFwd) {
+                    constexpr int EPG = DT == 1 ? 16 : 8;  // elements per 256-bit group
+                    uint32_t grp[8];
+#pragma unroll
+                    for (int w = 0; w < B / 8; ++w) {
                         float q[8];
-                        e2m1_unpack8(codes, q);
+                        e2m1_unpack8(codes[w], q);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) q[e] = __fmul_rn(q[e], sdq);
-                        store_chunk<DT>(p.y, off[j], q);
-                    } else {
-                        __stcs(reinterpret_cast<unsigned int*>(p.codes) + s, codes);
-                    }
-                    if (p.scales && (s % G::LPB) == 0)
-                        p.scales[s / G::LPB] = static_cast<uint8_t>(sbyte);
-                }
-            } else {
-                float gv[8];
-                unpack_chunk<DT>(gr[MODE == kBwd ? j : 0], gv);
-                float gxo[8];
-                float rho[NS];
-                df T[NS];
-                if (want_gx) scale_ratios<NS>(sdq, sq, dead, rho);
-                bwd_chunk<DT, NS>(v, gv, sq, rho, dead, p.ste, want_gx, want_T, gxo, T);
-                if (want_gx && valid) store_chunk<DT>(p.gx, off[j], gxo);
-                if (want_T) {
-                    // sub-blocks wider than a chunk: combine their lanes
-#pragma unroll
-                    for (int o = 1; o < G::LPS; o <<= 1) T[0] = df_add(T[0], shfl_xor_df(T[0], o));
-                    const float c = cv[j];
-                    const float rc = rcp_approx(c);
-                    df Q = {0.0f, 0.0f};
-                    float gd[NS];
-#pragma unroll
-                    for (int t = 0; t < NS; ++t) {
-                        const float d = dv[j][t];
-                        const float rd = rcp_approx(d);
-                        const df qk = df_div_f(T[t], d, rd);  // T_ik / c_i^k
-                        gd[t] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
-                        if (G::LPS == 1 || (s % G::LPS) == 0) Q = (t == 0) ? qk : df_add(Q, qk);
-                    }
-#pragma unroll
-                    for (int o = G::LPS; o < G::LPB; o <<= 1) Q = df_add(Q, shfl_xor_df(Q, o));
-                    if (valid) {
-                        if (p.gdgs) {
-                            if (SUB <= 8) store_coefs<NS>(p.gdgs + static_cast<size_t>(s) * NS, gd);
-                            else if ((s % G::LPS) == 0) p.gdgs[s / G::LPS] = gd[0];
+                        for (int e = 0; e < 8; e += 2) {
+                            const int el = 8 * w + e;
+                            put_pair<DT>(grp, (el % EPG) / 2,
+                                         mul2(make_float2(q[e], q[e + 1]), make_float2(sdq, sdq)));
+                            if (el % EPG == EPG - 2)
+                                st_v8(static_cast<char*>(p.y) + off[j] + (el / EPG) * 32, grp);
                         }
-                        if (p.gcrs && (s % G::LPB) == 0)
-                            p.gcrs[s / G::LPB] = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
                     }
+                } else {
+                    uint32_t* dst =
+                        reinterpret_cast<uint32_t*>(p.codes) + static_cast<size_t>(blk) * (B / 8);
+                    if constexpr (B == 32) {
+                        __stcs(reinterpret_cast<uint4*>(dst),
+                               make_uint4(codes[0], codes[1], codes[2], codes[3]));
+                    } else {
+                        __stcs(reinterpret_cast<uint2*>(dst), make_uint2(codes[0], codes[1]));
+                    }
+                }
+                if (p.scales) p.scales[blk] = static_cast<uint8_t>(sbyte);
+            } else {
+                float rho[K];
+                if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
+                float gd[K], gc;
+                df T[K];
+                block_bwd<DT, B, K>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], p.ste, want_gx,
+                                    want_T, p.gx, off[j], gd, gc, T);
+                if (want_T) {
+                    if (p.gdgs) store_coefs<K>(p.gdgs + static_cast<size_t>(blk) * K, gd);
+                    if (p.gcrs) p.gcrs[blk] = gc;
                 }
             }
         }
@@ -366,99 +546,85 @@ __global__ void __launch_bounds__(kThreads) fq_linear_kernel(const KParams p)
 }
 
 // ---------------------------------------------------------------------------
-// Backward with coefficients shared by all rows.  Thread x owns column chunk
-// cc = blockIdx.x * kThreads + threadIdx.x for the rows of its row group
-// (rows blockIdx.y*U + k*gridDim.y*U ...), so its coefficients stay in
-// registers and its T sums accumulate in registers across rows; each row
-// group then writes one partial (a double-fp32 pair) per sub-block column to
-// scratch, and fq_bwd_shared_finalize sums them in a fixed order.
+// Backward with coefficients shared by all rows.  A CTA is p.tx columns of
+// blocks x (kThreads / p.tx) row slots; thread (tx, ty) owns column block
+// cb = blockIdx.x * p.tx + tx and walks the rows of its slot, keeping that
+// column's coefficients and its K running sums in registers.  The CTA then
+// combines its row slots in a fixed order and writes one double-fp32 partial
+// per (row group, sub-block column) to scratch; fq_bwd_shared_finalize sums
+// the row groups in a fixed order.
 // ---------------------------------------------------------------------------
 template <int FMT, int DT, int SUB>
 __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p)
 {
-    using G = Geo<FMT, SUB>;
-    constexpr int NS = G::NS;
-    constexpr int U = DT == 1 ? 2 : 1;
+    using G = Geo<FMT, DT, SUB>;
+    constexpr int B = G::B, K = G::K, W = G::W;
+    constexpr int ESZ = DT == 1 ? 2 : 4;
+    __shared__ float2 red[kThreads * K];
     const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = p.gx != nullptr;
-    const bool want_T = p.gcrs != nullptr || p.gdgs != nullptr;
-    const uint32_t cc = blockIdx.x * kThreads + threadIdx.x;
-    const bool col_ok = cc < p.cpr;
+    const uint32_t tx = threadIdx.x % p.tx, ty = threadIdx.x / p.tx, nty = kThreads / p.tx;
+    const uint32_t cb = blockIdx.x * p.tx + tx;
+    const bool col_ok = cb < p.bpr;
 
     float c = 1.0f;
-    float d[NS];
+    float d[K];
 #pragma unroll
-    for (int t = 0; t < NS; ++t) d[t] = 1.0f;
+    for (int k = 0; k < K; ++k) d[k] = 1.0f;
     if (col_ok) {
-        if (p.crs) c = __ldg(p.crs + cc / G::LPB);
-        if (p.dgs) {
-            if (SUB <= 8) load_coefs<NS>(p.dgs + static_cast<size_t>(cc) * NS, d);
-            else d[0] = __ldg(p.dgs + cc / G::LPS);
-        }
+        if (p.crs) c = __ldg(p.crs + cb);
+        if (p.dgs) load_coefs<K>(p.dgs + static_cast<size_t>(cb) * K, d);
     }
-    df acc[NS];
+    df acc[K];
 #pragma unroll
-    for (int t = 0; t < NS; ++t) acc[t] = {0.0f, 0.0f};
+    for (int k = 0; k < K; ++k) acc[k] = {0.0f, 0.0f};
 
-    for (uint32_t r0 = blockIdx.y * U; r0 < p.rows; r0 += gridDim.y * U) {
-        ChunkRaw<DT> xr[U], gr[U];
-        uint64_t off[U];
-#pragma unroll
-        for (int j = 0; j < U; ++j) {
-            const uint32_t r = r0 + j;
-            off[j] = static_cast<uint64_t>(r) * p.ld + static_cast<uint64_t>(cc) * 8u;
-            if (col_ok && r < p.rows) {
-                load_chunk<DT>(xr[j], p.x, off[j]);
-                load_chunk<DT>(gr[j], p.g, off[j]);
-            } else {
-                zero_chunk<DT>(xr[j]);
-                zero_chunk<DT>(gr[j]);
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < U; ++j) {
-            const bool valid = col_ok && (r0 + j) < p.rows;
-            float v[8], gv[8];
-            unpack_chunk<DT>(xr[j], v);
-            unpack_chunk<DT>(gr[j], gv);
+    if (col_ok) {
+        for (uint32_t r = blockIdx.y * nty + ty; r < p.rows; r += gridDim.y * nty) {
+            uint32_t xr[W], gr[W];
+            const uint64_t off =
+                (static_cast<uint64_t>(r) * p.ld + static_cast<uint64_t>(cb) * B) * ESZ;
+            load_block<W>(xr, p.x, off);
+            load_block<W>(gr, p.g, off);
             uint32_t sbyte;
-            const float sdq = block_scale<FMT>(chunk_absmax(v), ts, p.mx_rule, sbyte);
-            float sq[NS];
-            bool dead[NS];
-            relaxed_scales<NS>(sdq, c, d, sq, dead);
-            float gxo[8];
-            float rho[NS];
-            df T[NS];
-            if (want_gx) scale_ratios<NS>(sdq, sq, dead, rho);
-            bwd_chunk<DT, NS>(v, gv, sq, rho, dead, p.ste, want_gx, want_T, gxo, T);
-            if (want_gx && valid) store_chunk<DT>(p.gx, off[j], gxo);
-            if (want_T) {
+            const float sdq = block_scale<FMT>(block_absmax<DT, W>(xr), ts, p.mx_rule, sbyte);
+            float sq[K];
+            bool dead[K];
+            relaxed_scales<K>(sdq, c, d, sq, dead);
+            float rho[K];
+            if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
+            float gd[K], gc;
+            df T[K];
+            block_bwd<DT, B, K>(xr, gr, sq, dead, rho, c, d, p.ste, want_gx, true, p.gx, off,
+                                gd, gc, T);
 #pragma unroll
-                for (int t = 0; t < NS; ++t) acc[t] = df_add(acc[t], T[t]);
-            }
+            for (int k = 0; k < K; ++k) acc[k] = df_add(acc[k], T[k]);
         }
     }
-    if (!want_T) return;
 #pragma unroll
-    for (int o = 1; o < G::LPS; o <<= 1) acc[0] = df_add(acc[0], shfl_xor_df(acc[0], o));
-    if (!col_ok) return;
+    for (int k = 0; k < K; ++k) red[threadIdx.x * K + k] = make_float2(acc[k].h, acc[k].l);
+    __syncthreads();
+    if (ty != 0 || !col_ok) return;
     float2* part = reinterpret_cast<float2*>(p.ws) + static_cast<size_t>(blockIdx.y) * p.nsub;
-    if (SUB <= 8) {
 #pragma unroll
-        for (int t = 0; t < NS; ++t) part[static_cast<size_t>(cc) * NS + t] = make_float2(acc[t].h, acc[t].l);
-    } else if ((cc % G::LPS) == 0) {
-        part[cc / G::LPS] = make_float2(acc[0].h, acc[0].l);
+    for (int k = 0; k < K; ++k) {
+        df a = acc[k];
+        for (uint32_t t = 1; t < nty; ++t) {
+            const float2 v = red[(t * p.tx + tx) * K + k];
+            a = df_add(a, df{v.x, v.y});
+        }
+        part[static_cast<size_t>(cb) * K + k] = make_float2(a.h, a.l);
     }
 }
 
 // One CTA per hardware-block column j: sums the row-group partials of its K
 // sub-blocks (fixed strided split, then a fixed shared-memory tree), then
-// dL/dc^k_j = -S_k / (c_j (c^k_j)^2) and dL/dc_j = -(sum_k S_k / c^k_j) / c_j^2.
+// the coefficient gradients of the column.
 template <int FMT, int SUB>
 __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams p, uint32_t ny)
 {
-    using G = Geo<FMT, SUB>;
-    constexpr int K = G::B / SUB;
+    constexpr int B = FMT == 0 ? 32 : 16;
+    constexpr int K = B / SUB;
     __shared__ float sh_h[kThreads], sh_l[kThreads];
     __shared__ float res_h[K], res_l[K];
     const uint32_t j = blockIdx.x;
@@ -490,16 +656,17 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams
     }
     if (threadIdx.x != 0) return;
     const float c = p.crs ? __ldg(p.crs + j) : 1.0f;
-    const float rc = rcp_approx(c);
-    df Q = {0.0f, 0.0f};
+    float d[K];
+    df T[K];
     for (int k = 0; k < K; ++k) {
-        const float d = p.dgs ? __ldg(p.dgs + j * K + k) : 1.0f;
-        const float rd = rcp_approx(d);
-        const df qk = df_div_f(df{res_h[k], res_l[k]}, d, rd);
-        if (p.gdgs) p.gdgs[j * K + k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
-        Q = df_add(Q, qk);
+        d[k] = p.dgs ? __ldg(p.dgs + j * K + k) : 1.0f;
+        T[k] = df{res_h[k], res_l[k]};
     }
-    if (p.gcrs) p.gcrs[j] = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
+    float gd[K], gc;
+    block_coef_grads<K>(T, c, d, gd, gc);
+    if (p.gdgs)
+        for (int k = 0; k < K; ++k) p.gdgs[j * K + k] = gd[k];
+    if (p.gcrs) p.gcrs[j] = gc;
 }
 
 // ---------------------------------------------------------------------------
@@ -535,7 +702,8 @@ __global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p
         for (int j = 0; j < U; ++j) {
             float v[8];
             unpack_chunk<DT>(xr[j], v);
-            m = fmaxf(m, chunk_absmax(v));
+#pragma unroll
+            for (int e = 0; e < 8; ++e) m = fmaxf(m, fabsf(v[e]));
         }
     }
 #pragma unroll

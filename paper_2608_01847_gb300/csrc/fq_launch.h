@@ -36,14 +36,23 @@ inline uint32_t alpha_grid(uint32_t n_chunks)
     return static_cast<uint32_t>(std::max<uint64_t>(1, std::min(need, cap)));
 }
 
-inline uint32_t shared_col_ctas(uint32_t cpr) { return (cpr + kThreads - 1) / kThreads; }
-
-inline uint32_t shared_row_groups(uint32_t rows, uint32_t cpr, int dtype)
+// Shared-row backward: block columns per CTA (a power of two from 32 to the
+// CTA size, covering the row when it is short) and the number of row groups.
+inline uint32_t shared_tx(uint32_t bpr)
 {
-    const uint32_t u = dtype == 1 ? 2u : 1u;
-    const uint64_t need = (static_cast<uint64_t>(rows) + u - 1) / u;
+    uint32_t tx = 32;
+    while (tx < bpr && tx < static_cast<uint32_t>(kThreads)) tx <<= 1;
+    return tx;
+}
+
+inline uint32_t shared_col_ctas(uint32_t bpr) { return (bpr + shared_tx(bpr) - 1) / shared_tx(bpr); }
+
+inline uint32_t shared_row_groups(uint32_t rows, uint32_t bpr)
+{
+    const uint32_t nty = kThreads / shared_tx(bpr);
+    const uint64_t need = (static_cast<uint64_t>(rows) + nty - 1) / nty;
     const uint64_t cap = std::max<uint64_t>(
-        1, static_cast<uint64_t>(device_sms()) * kCtasPerSm / shared_col_ctas(cpr));
+        1, static_cast<uint64_t>(device_sms()) * kCtasPerSm / shared_col_ctas(bpr));
     return static_cast<uint32_t>(std::max<uint64_t>(1, std::min<uint64_t>({need, cap, 65535})));
 }
 
@@ -63,11 +72,11 @@ inline uint32_t stream_grid(Kern kern, int& occ_cache, uint32_t n_chunks, uint32
 }
 
 template <int FMT, int DT, int SUB, int MODE>
-cudaError_t run_linear(const KParams& p, cudaStream_t st)
+cudaError_t run_block(const KParams& p, cudaStream_t st)
 {
     static int occ = 0;
-    auto kern = fq_linear_kernel<FMT, DT, SUB, MODE>;
-    const uint32_t grid = stream_grid(kern, occ, p.n_chunks, Unroll<DT, MODE>::U * kThreads);
+    auto kern = fq_block_kernel<FMT, DT, SUB, MODE>;
+    const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Unroll<FMT, DT, MODE>::U * kThreads);
     kern<<<grid, kThreads, 0, st>>>(p);
     return cudaGetLastError();
 }
@@ -77,12 +86,12 @@ template <int FMT, int DT, int MODE>
 cudaError_t linear_by_sub(int sub, const KParams& p, cudaStream_t st)
 {
     switch (sub) {
-    case 2: return run_linear<FMT, DT, 2, MODE>(p, st);
-    case 4: return run_linear<FMT, DT, 4, MODE>(p, st);
-    case 8: return run_linear<FMT, DT, 8, MODE>(p, st);
-    case 16: return run_linear<FMT, DT, 16, MODE>(p, st);
+    case 2: return run_block<FMT, DT, 2, MODE>(p, st);
+    case 4: return run_block<FMT, DT, 4, MODE>(p, st);
+    case 8: return run_block<FMT, DT, 8, MODE>(p, st);
+    case 16: return run_block<FMT, DT, 16, MODE>(p, st);
     case 32:
-        if constexpr (FMT == 0) return run_linear<FMT, DT, 32, MODE>(p, st);
+        if constexpr (FMT == 0) return run_block<FMT, DT, 32, MODE>(p, st);
         break;
     default: break;
     }

@@ -62,7 +62,8 @@ def _desc(rows=4, cols=64, ld=None, dtype=1, fmt=0, block=None, sub=8, shared=0,
 P = ctypes.c_void_p
 ALIGNED = P(0x100000)       # placeholder device addresses: never dereferenced
 ALIGNED2 = P(0x200000)
-ODD = P(0x100008)           # 8-byte aligned only
+ODD = P(0x100010)           # 16-byte aligned only (rows need 32)
+ODD8 = P(0x100008)          # 8-byte aligned only (coefficient arrays need 16)
 
 
 def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None):
@@ -72,6 +73,7 @@ def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None
 @pytest.mark.parametrize("kw,status", [
     (dict(block=64), -2), (dict(fmt=1, block=32), -2), (dict(sub=3), -2), (dict(sub=32, fmt=1), -2),
     (dict(sub=64), -2), (dict(cols=48), -1), (dict(ld=60), -1), (dict(ld=68), -3),
+    (dict(ld=72), -3), (dict(ld=72, dtype=0, rows=0), 0),
     (dict(dtype=2), -1), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
     (dict(shared=2), -1), (dict(rows=-1), -1), (dict(rows=1 << 40, cols=1 << 20), -2),
 ])
@@ -86,7 +88,7 @@ def test_null_and_alignment_rejections(L):
     assert fwd(L, _desc(fmt=1), alpha=None) == -1                 # NVFP4 needs alpha
     assert fwd(L, _desc(), x=ODD) == -3
     assert fwd(L, _desc(), y=ODD) == -3
-    assert fwd(L, _desc(), crs=ODD) == -3
+    assert fwd(L, _desc(), crs=ODD8) == -3
     assert fwd(L, _desc(rows=0)) == 0                             # empty: nothing to do
     d = _desc()
     assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, None, ALIGNED2, None) == -1
