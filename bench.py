@@ -1,17 +1,22 @@
 """Benchmark of the FOCUS FP4 fake-quantizer hot path on GB300.
 
-One step = one pass of the whole hot path over the Qwen3-4B-shaped decoder
-layer (7 bf16 projections, 100.9 M elements), NVFP4 (block 16, E4M3 + fp32
-alpha), per-block CRS and per-sub-block (8) DGS coefficients:
+Default case: one step = one pass of the whole hot path over the Qwen3-4B
+decoder layer (7 bf16 projections, 100.9 M elements), NVFP4 (block 16, E4M3
++ fp32 alpha), per-block CRS and per-sub-block (8) DGS coefficients:
   alpha (per tensor)  ->  fake-quant forward  ->  STE backward (input
   gradient + both coefficient gradients)  ->  export pack,
-each phase over all 7 tensors before the next (as a calibration step runs
-all forwards, then all backwards), inputs resident in HBM.  Each phase is
-captured once as a CUDA graph (its 7 tensors on parallel branches) and a
-step replays the four graphs in order.  `value` is the
-algorithmic bytes of the step (per-element figures below) over the step time.
+each phase over all tensors before the next (as a calibration step runs all
+forwards, then all backwards), inputs resident in HBM.  Each phase is
+captured once as a CUDA graph (its tensors on parallel branches) and a step
+replays the phase graphs in order.  `value` is the algorithmic bytes of the
+step (per-element figures in bytes_per_elem) over the step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+                  [--workload NAME --fmt mxfp4|nvfp4 --shared]
+
+Other workloads (the Llama-3-8B block, the 70B layer set, the W4A4
+activations, a sweep tensor) are measured the same way with --workload; the
+driver's line is the default case.
 
 Under torchrun (N > 1) every rank runs the same workload on its own GPU
 (replicas; no data-path collective), the step time is the max over ranks and
@@ -20,6 +25,7 @@ Under torchrun (N > 1) every rank runs the same workload on its own GPU
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -32,25 +38,42 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "fake-quant fwd+bwd GB/s and elems/s vs GB300 HBM peak; pack GB/s"
-WORKLOAD = "qwen3_4b_layer"
-FMT_NAME = "nvfp4"
-SUB = 8
 L2_BYTES = 129 * 1024 * 1024
 
-# Algorithmic bytes per element, bf16 I/O, fp32 coefficients, NVFP4 (B = 16),
-# sub-block 8: what each phase must move at minimum.
-BYTES_PER_ELEM = {
-    "alpha": 2.0,                                 # read x
-    "fwd": 2 + 2 + 4 / 16 + 4 / 8,                # x, y, c_i, c_i^k        = 4.75
-    "bwd": 2 + 2 + 2 + 2 * (4 / 16 + 4 / 8),      # x, g, gx, (c, c^k) in+out = 7.5
-    "pack": 2 + 4 / 16 + 4 / 8 + 0.5 + 1 / 16,    # x, c, c^k, codes, scales  = 3.3125
-}
-STEP_BYTES_PER_ELEM = sum(BYTES_PER_ELEM.values())
 
-# DRAM traffic (read + write) of one backward phase (7 launches) of this
-# benchmark, from an ncu launch list (gpu__time_duration, dram__bytes_read,
-# dram__bytes_write; --cache-control none), and the sha256 prefix of the
-# kernel sources it was taken on.  Reported only while they are unchanged.
+@dataclasses.dataclass(frozen=True)
+class Case:
+    workload: str = "qwen3_4b_layer"
+    fmt: str = "nvfp4"
+    sub: int = 8
+    shared: bool = False       # one coefficient set for all rows (activations)
+
+    @property
+    def block(self) -> int:
+        return 16 if self.fmt == "nvfp4" else 32
+
+    def phases(self):
+        return (["alpha"] if self.fmt == "nvfp4" else []) + ["fwd", "bwd", "pack"]
+
+
+def bytes_per_elem(case: Case, esz: int) -> dict:
+    """Algorithmic bytes per element of each phase (what it must move at
+    minimum): x, y, g, gx at `esz` bytes; fp32 coefficients in (and their
+    gradients out) per element unless shared by all rows; codes 0.5 B, one
+    scale byte per block."""
+    coef = 0.0 if case.shared else 4.0 / case.block + 4.0 / case.sub
+    out = {"fwd": 2 * esz + coef, "bwd": 3 * esz + 2 * coef,
+           "pack": esz + coef + 0.5 + 1.0 / case.block}
+    if case.fmt == "nvfp4":
+        out["alpha"] = float(esz)
+    return out
+
+
+# DRAM traffic (read + write) of one backward phase of the default case,
+# from an ncu launch list of this benchmark (gpu__time_duration,
+# dram__bytes_read, dram__bytes_write; --cache-control none), and the sha256
+# prefix of the kernel sources it was taken on.  Reported only for the
+# default case and while the sources are unchanged.
 BWD_TRAFFIC = {"sources": "7f8d1d796e157d46", "bytes_per_step": 762.1e6}
 
 
@@ -84,6 +107,7 @@ class ClockSampler:
     def __init__(self, index):
         self.index = index
         self.proc = None
+        self.out = ""
 
     def __enter__(self):
         try:
@@ -96,7 +120,6 @@ class ClockSampler:
         return self
 
     def __exit__(self, *a):
-        self.out = ""
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -125,76 +148,68 @@ class ClockSampler:
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
-class Layer:
-    """Device tensors of one projection plus its preallocated outputs."""
+class Tensor:
+    """Device tensors of one projection (or activation) plus its outputs."""
 
-    def __init__(self, w, idx, device):
+    def __init__(self, case: Case, w, idx, device):
         import torch
         from paper_2608_01847_gb300 import focus as F
         from paper_2608_01847_gb300 import workloads as W
+        self.fmt = F.FOCUS_NVFP4 if case.fmt == "nvfp4" else F.FOCUS_MXFP4
+        self.case = case
         self.x, self.g = W.device_tensor(w, idx, device)
-        self.crs, self.dgs = W.device_coefs(w, idx, 16, SUB, device)
+        self.crs, self.dgs = W.device_coefs(w, idx, case.block, case.sub, device, shared=case.shared)
         rows, cols = self.x.shape
         self.n = rows * cols
-        self.alpha = torch.empty(1, dtype=torch.float32, device=device)
+        self.alpha = torch.zeros(1, dtype=torch.float32, device=device)
         self.y = torch.empty_like(self.x)
         self.gx = torch.empty_like(self.x)
         self.gcrs = torch.empty_like(self.crs)
         self.gdgs = torch.empty_like(self.dgs)
         self.codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device=device)
-        self.scales = torch.empty((rows, cols // 16), dtype=torch.uint8, device=device)
-        d = F.make_desc(self.x, F.FOCUS_NVFP4, SUB)
-        self.ws = torch.empty(max(16, F.focus_workspace_bytes(d, F.FOCUS_WS_ALPHA)),
-                              dtype=torch.uint8, device=device)
+        self.scales = torch.empty((rows, cols // case.block), dtype=torch.uint8, device=device)
+        d = F.make_desc(self.x, self.fmt, case.sub, case.shared)
+        self.ws_alpha = torch.empty(max(16, F.focus_workspace_bytes(d, F.FOCUS_WS_ALPHA)),
+                                    dtype=torch.uint8, device=device)
+        self.ws_bwd = torch.empty(max(16, F.focus_workspace_bytes(d, F.FOCUS_WS_BWD)),
+                                  dtype=torch.uint8, device=device)
+
+    def run(self, phase):
+        from paper_2608_01847_gb300 import focus as F
+        c = self.case
+        if phase == "alpha":
+            F.focus_nvfp4_alpha(self.x, self.alpha, self.ws_alpha)
+        elif phase == "fwd":
+            F.focus_fq_fwd(self.x, self.fmt, self.crs, self.dgs, self.alpha, sub_block=c.sub,
+                           shared=c.shared, y=self.y)
+        elif phase == "bwd":
+            F.focus_fq_bwd(self.x, self.g, self.fmt, self.crs, self.dgs, self.alpha,
+                           sub_block=c.sub, shared=c.shared, gx=self.gx, gcrs=self.gcrs,
+                           gdgs=self.gdgs, ws=self.ws_bwd)
+        else:
+            F.focus_pack(self.x, self.fmt, self.crs, self.dgs, self.alpha, sub_block=c.sub,
+                         shared=c.shared, codes=self.codes, scale_bytes=self.scales)
+
+    def launches(self, phase):
+        return 2 if phase == "alpha" else (2 if (phase == "bwd" and self.case.shared) else 1)
 
 
-def phase_alpha(layers):
-    from paper_2608_01847_gb300 import focus as F
-    for L in layers:
-        F.focus_nvfp4_alpha(L.x, L.alpha, L.ws)
+class BranchGraph:
+    """A CUDA graph whose branches (one stream each) run `body(i)` for every
+    tensor i; the branches are independent and join at the end."""
 
-
-def phase_fwd(layers):
-    from paper_2608_01847_gb300 import focus as F
-    for L in layers:
-        F.focus_fq_fwd(L.x, F.FOCUS_NVFP4, L.crs, L.dgs, L.alpha, sub_block=SUB, y=L.y)
-
-
-def phase_bwd(layers):
-    from paper_2608_01847_gb300 import focus as F
-    for L in layers:
-        F.focus_fq_bwd(L.x, L.g, F.FOCUS_NVFP4, L.crs, L.dgs, L.alpha, sub_block=SUB, gx=L.gx,
-                       gcrs=L.gcrs, gdgs=L.gdgs)
-
-
-def phase_pack(layers):
-    from paper_2608_01847_gb300 import focus as F
-    for L in layers:
-        F.focus_pack(L.x, F.FOCUS_NVFP4, L.crs, L.dgs, L.alpha, sub_block=SUB, codes=L.codes,
-                     scale_bytes=L.scales)
-
-
-PHASES = [("alpha", phase_alpha), ("fwd", phase_fwd), ("bwd", phase_bwd), ("pack", phase_pack)]
-LAUNCHES_PER_TENSOR = {"alpha": 2, "fwd": 1, "bwd": 1, "pack": 1}
-
-
-class PhaseGraph:
-    """One phase (alpha, fwd, bwd or pack over all 7 tensors) captured as a
-    CUDA graph whose 7 tensors run on parallel branches (one stream each), so
-    small tensors fill the GPU alongside large ones."""
-
-    def __init__(self, fn, layers, device):
+    def __init__(self, n, body, device):
         import torch
         self.graph = torch.cuda.CUDAGraph()
-        side = [torch.cuda.Stream(device) for _ in layers]
+        side = [torch.cuda.Stream(device) for _ in range(n)]
         cap = torch.cuda.Stream(device)
         cap.wait_stream(torch.cuda.current_stream(device))
         with torch.cuda.graph(self.graph, stream=cap):
             main = torch.cuda.current_stream(device)
-            for L, st in zip(layers, side):
+            for i, st in enumerate(side):
                 st.wait_stream(main)
                 with torch.cuda.stream(st):
-                    fn([L])
+                    body(i)
             for st in side:
                 main.wait_stream(st)
         torch.cuda.current_stream(device).wait_stream(cap)
@@ -203,24 +218,28 @@ class PhaseGraph:
         self.graph.replay()
 
 
-def gpu_arm(args, rank, world, device):
+def gpu_arm(case, args, rank, world, device):
     import torch
     import torch.distributed as dist
     from paper_2608_01847_gb300 import focus as F
     from paper_2608_01847_gb300 import workloads as W
 
     F.lib()
-    w = W.WORKLOADS[WORKLOAD]
-    layers = [Layer(w, i, device) for i in range(len(w.tensors))]
-    n_elem = sum(L.n for L in layers)
+    w = W.WORKLOADS[case.workload] if case.workload in W.WORKLOADS else W.sweep_workload(
+        int(case.workload.split("_")[-1]))
+    ts = [Tensor(case, w, i, device) for i in range(len(w.tensors))]
+    n_elem = sum(t.n for t in ts)
+    esz = ts[0].x.element_size()
     stream = torch.cuda.current_stream(device)
+    phases = case.phases()
     torch.cuda.synchronize(device)
 
-    # eager warm-up (resolves launch configurations), then capture one step
-    for name, fn in PHASES:
-        fn(layers)
+    # eager warm-up (resolves launch configurations), then capture each phase
+    for ph in phases:
+        for t in ts:
+            t.run(ph)
     torch.cuda.synchronize(device)
-    graphs = [(name, PhaseGraph(fn, layers, device)) for name, fn in PHASES]
+    graphs = [(ph, BranchGraph(len(ts), lambda i, ph=ph: ts[i].run(ph), device)) for ph in phases]
 
     def step():
         for _, gph in graphs:
@@ -235,18 +254,18 @@ def gpu_arm(args, rank, world, device):
             dist.barrier()
         torch.cuda.synchronize(device)
 
-    # ---- device-resident timing: K graph replays; per-phase events ----
-    phase_ms = {n: 0.0 for n, _ in PHASES}
+    # ---- device-resident timing: K steps ----
     with ClockSampler(device.index if device.index is not None else 0) as clk:
         barrier()
         start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         start.record(stream)
-        for k in range(args.steps):
+        for _ in range(args.steps):
             step()
         end.record(stream)
         barrier()
     total_ms = start.elapsed_time(end)
     # phase split: each phase graph replayed on its own, timed the same way
+    phase_ms = {}
     n_split = max(1, min(args.steps, 100))
     for name, gph in graphs:
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -261,36 +280,37 @@ def gpu_arm(args, rank, world, device):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         total_ms = float(t.item())
 
+    res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, clocks=clk.summary(),
+               ntensors=len(ts), launches_per_step=sum(t.launches(ph) for t in ts for ph in phases))
+    if args.no_e2e:
+        return res
+
     # ---- end to end through the public API with pinned host buffers ----
-    e2e_steps = max(1, min(args.steps, 5))
-    host_in = [(L.x.cpu().pin_memory(), L.g.cpu().pin_memory(), L.crs.cpu().pin_memory(),
-                L.dgs.cpu().pin_memory()) for L in layers]
-    host_out = [(torch.empty_like(L.y, device="cpu").pin_memory(),
-                 torch.empty_like(L.gx, device="cpu").pin_memory(),
-                 torch.empty_like(L.gcrs, device="cpu").pin_memory(),
-                 torch.empty_like(L.gdgs, device="cpu").pin_memory(),
-                 torch.empty_like(L.codes, device="cpu").pin_memory(),
-                 torch.empty_like(L.scales, device="cpu").pin_memory()) for L in layers]
-    h2d = sum(sum(t.numel() * t.element_size() for t in h) for h in host_in)
-    d2h = sum(sum(t.numel() * t.element_size() for t in h) for h in host_out)
+    # Each tensor is one branch: H2D of its inputs, its phases, D2H of its
+    # outputs; the branches overlap (transfers of one with compute of others).
+    host_in = [[a.cpu().pin_memory() for a in (t.x, t.g, t.crs, t.dgs)] for t in ts]
+    host_out = [[torch.empty_like(a, device="cpu").pin_memory()
+                 for a in (t.y, t.gx, t.gcrs, t.gdgs, t.codes, t.scales)] for t in ts]
+    h2d = sum(a.numel() * a.element_size() for h in host_in for a in h)
+    d2h = sum(a.numel() * a.element_size() for h in host_out for a in h)
 
-    def e2e_step():
-        for L, (hx, hg, hc, hd) in zip(layers, host_in):
-            L.x.copy_(hx, non_blocking=True)
-            L.g.copy_(hg, non_blocking=True)
-            L.crs.copy_(hc, non_blocking=True)
-            L.dgs.copy_(hd, non_blocking=True)
-        step()
-        for L, outs in zip(layers, host_out):
-            for h, d in zip(outs, (L.y, L.gx, L.gcrs, L.gdgs, L.codes, L.scales)):
-                h.copy_(d, non_blocking=True)
+    def e2e_branch(i):
+        t = ts[i]
+        for d, h in zip((t.x, t.g, t.crs, t.dgs), host_in[i]):
+            d.copy_(h, non_blocking=True)
+        for ph in phases:
+            t.run(ph)
+        for h, d in zip(host_out[i], (t.y, t.gx, t.gcrs, t.gdgs, t.codes, t.scales)):
+            h.copy_(d, non_blocking=True)
 
-    e2e_step()
+    e2e_graph = BranchGraph(len(ts), e2e_branch, device)
+    e2e_steps = max(3, min(args.steps, 20))
+    e2e_graph.replay()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(e2e_steps):
-        e2e_step()
+        e2e_graph.replay()
     e1.record(stream)
     barrier()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
@@ -298,83 +318,90 @@ def gpu_arm(args, rank, world, device):
         t = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_ms = float(t.item())
-
-    return dict(n_elem=n_elem, total_ms=total_ms, phase_ms=phase_ms, clocks=clk.summary(),
-                e2e_ms=e2e_ms, h2d=h2d, d2h=d2h, ntensors=len(layers))
+    res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
+    return res
 
 
 # ----------------------------------------------------------------------------
 # oracle (CPU) runs: cpu_baseline leg and the reference arm
 # ----------------------------------------------------------------------------
-def oracle_step(samples):
-    """One pass of alpha, fwd, bwd, pack of the oracle over host samples."""
+def oracle_step(case, samples):
+    """One pass of the oracle's alpha, fwd, bwd, pack over host samples."""
     import oracle as O
+    fmt = O.NVFP4 if case.fmt == "nvfp4" else O.MXFP4
     for x, g, crs, dgs in samples:
-        a = O.alpha(x)
-        O.fwd(x, O.NVFP4, crs=crs, dgs=dgs, alpha=a, sub=SUB, want_scales=False)
-        O.bwd(x, g, O.NVFP4, crs=crs, dgs=dgs, alpha=a, sub=SUB)
-        O.fwd(x, O.NVFP4, crs=crs, dgs=dgs, alpha=a, sub=SUB, want_y=False, want_codes=True)
+        a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+        kw = dict(crs=crs, dgs=dgs, alpha=a, sub=case.sub, shared=case.shared)
+        O.fwd(x, fmt, want_scales=False, **kw)
+        O.bwd(x, g, fmt, **kw)
+        O.fwd(x, fmt, want_y=False, want_codes=True, **kw)
 
 
-def oracle_samples(rows_per_tensor):
+def oracle_samples(case, rows_per_tensor):
     from paper_2608_01847_gb300 import workloads as W
-    w = W.WORKLOADS[WORKLOAD]
+    w = W.WORKLOADS[case.workload]
     out = []
     for i in range(len(w.tensors)):
         x, g = W.host_tensor(w, i, rows=rows_per_tensor)
-        crs, dgs = W.host_coefs(w, i, 16, SUB, rows=rows_per_tensor)
+        crs, dgs = W.host_coefs(w, i, case.block, case.sub, shared=case.shared,
+                                rows=rows_per_tensor)
         out.append((x, g, crs, dgs))
     return out
 
 
-def calibrate_oracle(target_s):
+def calibrate_oracle(case, target_s):
     """Rows per tensor so that one oracle step takes about target_s seconds."""
-    probe = oracle_samples(8)
+    probe = oracle_samples(case, 8)
     t0 = time.perf_counter()
-    oracle_step(probe)
+    oracle_step(case, probe)
     dt = max(time.perf_counter() - t0, 1e-6)
-    rows = int(8 * target_s / dt)
-    return max(1, min(rows, 1 << 20))
+    return max(1, min(int(8 * target_s / dt), 1 << 20))
 
 
-def cpu_baseline(target_s=15.0):
+def sample_elems_and_bytes(case, samples):
+    n = sum(s[0].size for s in samples)
+    esz = samples[0][0].itemsize
+    return n, n * sum(bytes_per_elem(case, esz).values())
+
+
+def cpu_baseline(case, target_s=15.0):
     import oracle as O
     O.build()
-    rows = calibrate_oracle(target_s)
-    samples = oracle_samples(rows)
-    n = sum(s[0].size for s in samples)
+    rows = calibrate_oracle(case, target_s)
+    samples = oracle_samples(case, rows)
+    n, nbytes = sample_elems_and_bytes(case, samples)
     t0 = time.perf_counter()
-    oracle_step(samples)
+    oracle_step(case, samples)
     dt = time.perf_counter() - t0
-    return {"value": round(n * STEP_BYTES_PER_ELEM / dt / 1e9, 6), "unit": "GB/s", "cores": 1,
-            "kind": "oracle",
-            "sample": f"first {rows} rows of each of the 7 {WORKLOAD} projections "
-                      f"({n} elements; alpha+fwd+bwd+pack, single thread), {dt:.1f} s",
+    return {"value": round(nbytes / dt / 1e9, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"first {rows} rows of each tensor of {case.workload} ({n} elements; "
+                      f"{'+'.join(case.phases())}, single thread), {dt:.1f} s",
             "elems_per_s": round(n / dt, 1)}
 
 
-def reference_arm(args):
+def reference_arm(case, args):
     import oracle as O
     O.build()
     budget = 150.0 / max(1, args.steps + args.warmup)
-    rows = calibrate_oracle(min(budget, 20.0))
-    samples = oracle_samples(rows)
-    n = sum(s[0].size for s in samples)
+    rows = calibrate_oracle(case, min(budget, 20.0))
+    samples = oracle_samples(case, rows)
+    n, nbytes = sample_elems_and_bytes(case, samples)
     for _ in range(args.warmup):
-        oracle_step(samples)
+        oracle_step(case, samples)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle_step(samples)
+        oracle_step(case, samples)
     dt = (time.perf_counter() - t0) / max(1, args.steps)
-    value = n * STEP_BYTES_PER_ELEM / dt / 1e9
+    value = nbytes / dt / 1e9
     return {"metric": METRIC, "value": round(value, 6), "unit": "GB/s", "impl": "reference",
             "n_gpus": 0, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD, "fmt": FMT_NAME, "io_dtype": "bf16", "sub_block": SUB,
-                       "sample_rows_per_tensor": rows, "elements_per_step": n},
+            "config": {"workload": case.workload, "fmt": case.fmt, "sub_block": case.sub,
+                       "shared_coefficients": case.shared, "sample_rows_per_tensor": rows,
+                       "elements_per_step": n},
             "cpu_baseline": {"value": round(value, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                             "sample": f"first {rows} rows of each projection per step, "
+                             "sample": f"first {rows} rows of each tensor per step, "
                                        f"single-threaded CPU oracle"},
             "e2e": {"value": round(value, 6), "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -387,8 +414,15 @@ def main():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="focus", choices=["focus", "reference"])
+    ap.add_argument("--workload", default="qwen3_4b_layer")
+    ap.add_argument("--fmt", default="nvfp4", choices=["nvfp4", "mxfp4"])
+    ap.add_argument("--sub", type=int, default=8)
+    ap.add_argument("--shared", action="store_true", help="coefficients shared by all rows")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
+    case = Case(args.workload, args.fmt, args.sub, args.shared)
+    default_case = case == Case()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -396,7 +430,7 @@ def main():
 
     if args.impl == "reference":
         if rank == 0:
-            print(json.dumps(reference_arm(args)))
+            print(json.dumps(reference_arm(case, args)))
         return
 
     args.warmup = max(args.warmup, 3)
@@ -414,7 +448,7 @@ def main():
         dist.barrier()
         build()
 
-    r = gpu_arm(args, rank, world, device)
+    r = gpu_arm(case, args, rank, world, device)
     if rank != 0:
         if world > 1:
             import torch.distributed as dist
@@ -424,43 +458,47 @@ def main():
     peak, peak_kind = load_peaks()
     K = args.steps
     ms_step = r["total_ms"] / K
-    step_bytes = r["n_elem"] * STEP_BYTES_PER_ELEM
+    bpe = bytes_per_elem(case, r["esz"])
+    step_bytes = r["n_elem"] * sum(bpe.values())
     value = world * step_bytes / (ms_step * 1e-3) / 1e9
     ph = {n: r["phase_ms"][n] / K for n in r["phase_ms"]}
-    gbs = {n: r["n_elem"] * BYTES_PER_ELEM[n] / (ph[n] * 1e-3) / 1e9 for n in ph}
+    gbs = {n: r["n_elem"] * bpe[n] / (ph[n] * 1e-3) / 1e9 for n in ph}
     dom = max(ph, key=ph.get)
-    achieved = gbs[dom]
-    fb_bytes = r["n_elem"] * (BYTES_PER_ELEM["fwd"] + BYTES_PER_ELEM["bwd"])
+    fb_bytes = r["n_elem"] * (bpe["fwd"] + bpe["bwd"])
+    traffic = None
+    if default_case and dom == "bwd" and kernel_sources_sha() == BWD_TRAFFIC["sources"]:
+        traffic = BWD_TRAFFIC["bytes_per_step"]
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "tensors": r["ntensors"], "elements": r["n_elem"],
-                   "fmt": FMT_NAME, "io_dtype": "bf16", "sub_block": SUB,
-                   "coefficients": "per-block CRS + per-sub-block DGS, U(0.9,1.1)",
-                   "step": "alpha, fwd, bwd (gx + gcrs + gdgs), pack over all 7 tensors",
-                   "bytes_per_elem": round(STEP_BYTES_PER_ELEM, 4),
-                   "l2": f"inputs larger than L2: x+g = {r['n_elem'] * 4 / 2**20:.0f} MiB per step",
+        "config": {"workload": case.workload, "tensors": r["ntensors"], "elements": r["n_elem"],
+                   "fmt": case.fmt, "io_dtype": "bf16" if r["esz"] == 2 else "f32",
+                   "sub_block": case.sub,
+                   "coefficients": ("shared by all rows" if case.shared else
+                                    "per-block CRS + per-sub-block DGS"),
+                   "step": "+".join(case.phases()) + " over all tensors (bwd: gx + gcrs + gdgs)",
+                   "bytes_per_elem": round(sum(bpe.values()), 4),
+                   "l2": f"inputs larger than L2: x+g = {r['n_elem'] * 2 * r['esz'] / 2**20:.0f} MiB"
+                         " per step",
                    "parallelism": f"replicas x{world}"},
         "elems_per_s": round(world * r["n_elem"] / (ms_step * 1e-3), 1),
         "fwd_bwd_gbs": round(fb_bytes / ((ph["fwd"] + ph["bwd"]) * 1e-3) / 1e9, 2),
         "pack_gbs": round(gbs["pack"], 2),
         "phase_gbs": {n: round(v, 2) for n, v in gbs.items()},
         "phase_ms": {n: round(v, 4) for n, v in ph.items()},
-        "roofline": {"bound": "hbm", "kernel": f"fq_{dom}", "achieved": round(achieved, 2),
+        "roofline": {"bound": "hbm", "kernel": f"fq_{dom}", "achieved": round(gbs[dom], 2),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
-                     "frac": round(achieved / peak, 4),
-                     "traffic": (BWD_TRAFFIC["bytes_per_step"]
-                                 if dom == "bwd" and kernel_sources_sha() == BWD_TRAFFIC["sources"]
-                                 else None),
-                     "traffic_unit": "bytes per phase (7 launches)"},
+                     "frac": round(gbs[dom] / peak, 4), "traffic": traffic,
+                     "traffic_unit": "bytes per phase (one launch per tensor)"},
         "clocks": r["clocks"],
-        "e2e": {"value": round(world * step_bytes / (r["e2e_ms"] * 1e-3) / 1e9, 2), "unit": "GB/s",
-                "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
-        "gpu_launches": K * r["ntensors"] * sum(LAUNCHES_PER_TENSOR.values()),
+        "gpu_launches": K * r["launches_per_step"],
     }
+    if "e2e_ms" in r:
+        out["e2e"] = {"value": round(world * step_bytes / (r["e2e_ms"] * 1e-3) / 1e9, 2),
+                      "unit": "GB/s", "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]}
     if not args.no_cpu_baseline and world == 1:
-        out["cpu_baseline"] = cpu_baseline()
+        out["cpu_baseline"] = cpu_baseline(case)
     print(json.dumps(out))
     if world > 1:
         import torch.distributed as dist
