@@ -58,7 +58,7 @@ def lib() -> ctypes.CDLL:
         L.focus_oracle_fwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32,
                                        p, p, p, f, p, p, p]
         L.focus_oracle_bwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32, i32,
-                                       p, p, p, f, p, p, p, p, p, p]
+                                       p, p, p, f, p, p, p, p, p, p, p, p]
         L.focus_oracle_dequant.argtypes = [i32, i32, i64, i64, i32, p, p, f, p]
         L.focus_oracle_e2m1_code.argtypes = [f]
         L.focus_oracle_e2m1_value.argtypes = [i32]
@@ -191,12 +191,13 @@ def fwd(x, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
 
 def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
         ste=STE_IDENTITY, mx_rule=MX_CEIL, want_gx=True, want_gcrs=True, want_gdgs=True,
-        want_abs=False):
+        want_abs=False, want_f64=False):
     """STE backward (Sec. 3.2; Eq. 6-8): input gradient and coefficient gradients.
 
     Returns dict with 'gx' (dtype of x), 'gcrs' float32 [rows or 1, cols/block],
-    'gdgs' float32 [rows or 1, cols/sub], and with want_abs the binary64
-    term-magnitude sums 'gcrs_abs', 'gdgs_abs' of the same shapes."""
+    'gdgs' float32 [rows or 1, cols/sub], with want_abs the binary64
+    term-magnitude sums 'gcrs_abs', 'gdgs_abs', and with want_f64 the
+    gradients before their final rounding, 'gcrs64', 'gdgs64' (binary64)."""
     x = np.ascontiguousarray(x)
     g = np.ascontiguousarray(g)
     assert g.dtype == x.dtype and g.shape == x.shape
@@ -209,10 +210,12 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
     gd = np.zeros((crow, cols // sub), np.float32) if want_gdgs else None
     gca = np.zeros((crow, cols // block), np.float64) if (want_abs and want_gcrs) else None
     gda = np.zeros((crow, cols // sub), np.float64) if (want_abs and want_gdgs) else None
+    gc64 = np.zeros((crow, cols // block), np.float64) if want_f64 else None
+    gd64 = np.zeros((crow, cols // sub), np.float64) if want_f64 else None
     _check(lib().focus_oracle_bwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
                                   int(bool(shared)), ste, mx_rule, _ptr(x), _ptr(crs),
                                   _ptr(dgs), float(alpha), _ptr(g), _ptr(gx), _ptr(gc),
-                                  _ptr(gd), _ptr(gca), _ptr(gda)))
+                                  _ptr(gd), _ptr(gca), _ptr(gda), _ptr(gc64), _ptr(gd64)))
     out = {}
     if want_gx:
         out["gx"] = gx
@@ -224,6 +227,8 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
         out["gdgs"] = gd
         if want_abs:
             out["gdgs_abs"] = gda
+    if want_f64:
+        out["gcrs64"], out["gdgs64"] = gc64, gd64
     return out
 
 

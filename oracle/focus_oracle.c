@@ -353,12 +353,14 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
  *   dL/dc_i   = sum_k -T_ik * c_i^k / c_eff^2
  * In shared mode (one coefficient set for all rows) both also sum over rows.
  * Optional outputs gcrs_abs / gdgs_abs receive the same sums taken over
- * |mask*g*x| (the scale of the terms, used to bound rounding error).  */
+ * |mask*g*x| (the scale of the terms, used to bound rounding error), and
+ * gcrs64 / gdgs64 the gradients themselves before the final rounding to
+ * binary32 (so that partial results can be added exactly).  */
 int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                      int block, int sub, int shared, int ste, int mx_rule,
                      const void* x, const float* crs, const float* dgs, float alpha,
                      const void* g, void* gx, float* gcrs, float* gdgs,
-                     double* gcrs_abs, double* gdgs_abs)
+                     double* gcrs_abs, double* gdgs_abs, double* gcrs64, double* gdgs64)
 {
     if (check_shape(rows, cols, ld, block, sub, dtype)) return -1;
     if (fmt != OR_MXFP4 && fmt != OR_NVFP4) return -1;
@@ -435,6 +437,7 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                     int64_t di = r * nsub + j * K + k;
                     if (gdgs) gdgs[di] = (float)(G * (double)c);
                     if (gdgs_abs) gdgs_abs[di] = Ga * (double)c;
+                    if (gdgs64) gdgs64[di] = G * (double)c;
                     ksum_add(&gc, G * (double)d);
                     ksum_add(&gca, Ga * (double)d);
                 }
@@ -442,6 +445,7 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
             if (!shared) {
                 if (gcrs) gcrs[r * nblk + j] = (float)ksum_value(&gc);
                 if (gcrs_abs) gcrs_abs[r * nblk + j] = ksum_value(&gca);
+                if (gcrs64) gcrs64[r * nblk + j] = ksum_value(&gc);
             }
         }
     }
@@ -449,10 +453,12 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
         for (int64_t j = 0; j < nblk; j++) {
             if (gcrs) gcrs[j] = (float)ksum_value(&acc_c[j]);
             if (gcrs_abs) gcrs_abs[j] = ksum_value(&acc_ca[j]);
+            if (gcrs64) gcrs64[j] = ksum_value(&acc_c[j]);
         }
         for (int64_t i = 0; i < nsub; i++) {
             if (gdgs) gdgs[i] = (float)ksum_value(&acc_d[i]);
             if (gdgs_abs) gdgs_abs[i] = ksum_value(&acc_da[i]);
+            if (gdgs64) gdgs64[i] = ksum_value(&acc_d[i]);
         }
         free(sh);
     }
