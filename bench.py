@@ -6,9 +6,9 @@ decoder layer (7 bf16 projections, 100.9 M elements), NVFP4 (block 16, E4M3
   alpha (per tensor)  ->  fake-quant forward  ->  STE backward (input
   gradient + both coefficient gradients)  ->  export pack,
 each phase over all tensors before the next (as a calibration step runs all
-forwards, then all backwards), inputs resident in HBM.  Each phase is
-captured once as a CUDA graph (its tensors on parallel branches) and a step
-replays the phase graphs in order.  `value` is the algorithmic bytes of the
+forwards, then all backwards), inputs resident in HBM.  The step is captured
+once as a CUDA graph: the phases in order, each phase's tensors on parallel
+branches that join before the next phase.  `value` is the algorithmic bytes of the
 step (per-element figures in bytes_per_elem) over the step time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
@@ -74,7 +74,7 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
 # dram__bytes_read, dram__bytes_write; --cache-control none), and the sha256
 # prefix of the kernel sources it was taken on.  Reported only for the
 # default case and while the sources are unchanged.
-BWD_TRAFFIC = {"sources": "7f8d1d796e157d46", "bytes_per_step": 762.1e6}
+BWD_TRAFFIC = {"sources": "362a9af01b1cdea8", "bytes_per_step": 745.7e6}
 
 
 def kernel_sources_sha() -> str:
@@ -195,10 +195,11 @@ class Tensor:
 
 
 class BranchGraph:
-    """A CUDA graph whose branches (one stream each) run `body(i)` for every
-    tensor i; the branches are independent and join at the end."""
+    """A CUDA graph of one or more stages run in order; in each stage the
+    branches (one stream each) run `body(i, stage)` for every tensor i
+    independently and join before the next stage."""
 
-    def __init__(self, n, body, device):
+    def __init__(self, n, body, device, stages=(None,)):
         import torch
         self.graph = torch.cuda.CUDAGraph()
         side = [torch.cuda.Stream(device) for _ in range(n)]
@@ -206,12 +207,13 @@ class BranchGraph:
         cap.wait_stream(torch.cuda.current_stream(device))
         with torch.cuda.graph(self.graph, stream=cap):
             main = torch.cuda.current_stream(device)
-            for i, st in enumerate(side):
-                st.wait_stream(main)
-                with torch.cuda.stream(st):
-                    body(i)
-            for st in side:
-                main.wait_stream(st)
+            for stage in stages:
+                for i, st in enumerate(side):
+                    st.wait_stream(main)
+                    with torch.cuda.stream(st):
+                        body(i) if stage is None else body(i, stage)
+                for st in side:
+                    main.wait_stream(st)
         torch.cuda.current_stream(device).wait_stream(cap)
 
     def replay(self):
@@ -239,11 +241,12 @@ def gpu_arm(case, args, rank, world, device):
         for t in ts:
             t.run(ph)
     torch.cuda.synchronize(device)
+    # one graph per phase (for the phase split) and one for the whole step
     graphs = [(ph, BranchGraph(len(ts), lambda i, ph=ph: ts[i].run(ph), device)) for ph in phases]
+    step_graph = BranchGraph(len(ts), lambda i, ph: ts[i].run(ph), device, stages=phases)
 
     def step():
-        for _, gph in graphs:
-            gph.replay()
+        step_graph.replay()
 
     for _ in range(args.warmup):
         step()
