@@ -146,6 +146,27 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------
+# multi-rank timing (replicas: no data-path collective)
+# ----------------------------------------------------------------------------
+def max_over_ranks(ms: float, world: int, device=None) -> float:
+    """The slowest rank's time: an all-reduce MAX of one scalar (the only
+    collective of the benchmark; it is not part of the timed work)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_gbs(bytes_per_rank_step: float, world: int, max_ms_per_step: float) -> float:
+    """Whole-job throughput under weak scaling: every rank processes the same
+    bytes per step, the job's step time is the slowest rank's."""
+    return world * bytes_per_rank_step / (max_ms_per_step * 1e-3) / 1e9
+
+
+# ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
 class Tensor:
@@ -278,10 +299,7 @@ def gpu_arm(case, args, rank, world, device):
         b.record(stream)
         torch.cuda.synchronize(device)
         phase_ms[name] = a.elapsed_time(b) * args.steps / n_split
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, device)
 
     res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, clocks=clk.summary(),
                ntensors=len(ts), launches_per_step=sum(t.launches(ph) for t in ts for ph in phases))
@@ -317,10 +335,7 @@ def gpu_arm(case, args, rank, world, device):
     e1.record(stream)
     barrier()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, device)
     res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
     return res
 
@@ -463,7 +478,7 @@ def main():
     ms_step = r["total_ms"] / K
     bpe = bytes_per_elem(case, r["esz"])
     step_bytes = r["n_elem"] * sum(bpe.values())
-    value = world * step_bytes / (ms_step * 1e-3) / 1e9
+    value = aggregate_gbs(step_bytes, world, ms_step)
     ph = {n: r["phase_ms"][n] / K for n in r["phase_ms"]}
     gbs = {n: r["n_elem"] * bpe[n] / (ph[n] * 1e-3) / 1e9 for n in ph}
     dom = max(ph, key=ph.get)
@@ -498,7 +513,7 @@ def main():
         "gpu_launches": K * r["launches_per_step"],
     }
     if "e2e_ms" in r:
-        out["e2e"] = {"value": round(world * step_bytes / (r["e2e_ms"] * 1e-3) / 1e9, 2),
+        out["e2e"] = {"value": round(aggregate_gbs(step_bytes, world, r["e2e_ms"]), 2),
                       "unit": "GB/s", "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]}
     if not args.no_cpu_baseline and world == 1:
         out["cpu_baseline"] = cpu_baseline(case)
