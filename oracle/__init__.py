@@ -56,9 +56,9 @@ def lib() -> ctypes.CDLL:
         i64, i32, p, f = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p, ctypes.c_float
         L.focus_oracle_alpha.argtypes = [i32, i64, i64, i64, p, p]
         L.focus_oracle_fwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32,
-                                       p, p, p, f, p, p, p]
+                                       p, p, p, f, p, p, p, p]
         L.focus_oracle_bwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32, i32,
-                                       p, p, p, f, p, p, p, p, p, p, p, p]
+                                       p, p, p, f, p, p, p, p, p, p, p, p, p, p, p]
         L.focus_oracle_dequant.argtypes = [i32, i32, i64, i64, i32, p, p, f, p]
         L.focus_oracle_e2m1_code.argtypes = [f]
         L.focus_oracle_e2m1_value.argtypes = [i32]
@@ -163,23 +163,24 @@ def alpha(x: np.ndarray) -> float:
 
 
 def fwd(x, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
-        mx_rule=MX_CEIL, want_y=True, want_scales=True, want_codes=False):
+        mx_rule=MX_CEIL, want_y=True, want_scales=True, want_codes=False, sfp=None):
     """Fake-quant forward / export (Eq. 1-8, Fig. 3(d)).
 
     x: [rows, cols] float32 or uint16 (bf16 bits), contiguous.
     Returns dict with 'y' (same dtype as x), 'scales' uint8 [rows, cols/block],
-    'codes' uint8 [rows, cols/2] (as requested)."""
+    'codes' uint8 [rows, cols/2] (as requested).  sfp: optional learnable
+    full-precision scales [rows, cols/block] (Eq. 4) replacing the absmax scale."""
     x = np.ascontiguousarray(x)
     rows, cols = x.shape
     block = block or default_block(fmt)
-    crs, dgs = _c32(crs), _c32(dgs)
+    crs, dgs, sfp = _c32(crs), _c32(dgs), _c32(sfp)
     out = {}
     y = np.empty_like(x) if want_y else None
     sc = np.zeros((rows, cols // block), np.uint8) if want_scales else None
     cd = np.zeros((rows, cols // 2), np.uint8) if want_codes else None
     _check(lib().focus_oracle_fwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
                                   int(bool(shared)), mx_rule, _ptr(x), _ptr(crs), _ptr(dgs),
-                                  float(alpha), _ptr(y), _ptr(sc), _ptr(cd)))
+                                  float(alpha), _ptr(sfp), _ptr(y), _ptr(sc), _ptr(cd)))
     if want_y:
         out["y"] = y
     if want_scales:
@@ -191,20 +192,24 @@ def fwd(x, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
 
 def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=False,
         ste=STE_IDENTITY, mx_rule=MX_CEIL, want_gx=True, want_gcrs=True, want_gdgs=True,
-        want_abs=False, want_f64=False):
+        want_abs=False, want_f64=False, sfp=None, want_gsfp=False):
     """STE backward (Sec. 3.2; Eq. 6-8): input gradient and coefficient gradients.
 
     Returns dict with 'gx' (dtype of x), 'gcrs' float32 [rows or 1, cols/block],
     'gdgs' float32 [rows or 1, cols/sub], with want_abs the binary64
     term-magnitude sums 'gcrs_abs', 'gdgs_abs', and with want_f64 the
-    gradients before their final rounding, 'gcrs64', 'gdgs64' (binary64)."""
+    gradients before their final rounding, 'gcrs64', 'gdgs64' (binary64).
+    sfp: optional learnable scales (Eq. 4); want_gsfp adds 'gsfp' float32
+    [rows, cols/block] (and 'gsfp_abs' with want_abs)."""
     x = np.ascontiguousarray(x)
     g = np.ascontiguousarray(g)
     assert g.dtype == x.dtype and g.shape == x.shape
     rows, cols = x.shape
     block = block or default_block(fmt)
-    crs, dgs = _c32(crs), _c32(dgs)
+    crs, dgs, sfp = _c32(crs), _c32(dgs), _c32(sfp)
     crow = 1 if shared else rows
+    gs = np.zeros((rows, cols // block), np.float32) if want_gsfp else None
+    gsa = np.zeros((rows, cols // block), np.float64) if (want_gsfp and want_abs) else None
     gx = np.empty_like(x) if want_gx else None
     gc = np.zeros((crow, cols // block), np.float32) if want_gcrs else None
     gd = np.zeros((crow, cols // sub), np.float32) if want_gdgs else None
@@ -214,8 +219,9 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
     gd64 = np.zeros((crow, cols // sub), np.float64) if want_f64 else None
     _check(lib().focus_oracle_bwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
                                   int(bool(shared)), ste, mx_rule, _ptr(x), _ptr(crs),
-                                  _ptr(dgs), float(alpha), _ptr(g), _ptr(gx), _ptr(gc),
-                                  _ptr(gd), _ptr(gca), _ptr(gda), _ptr(gc64), _ptr(gd64)))
+                                  _ptr(dgs), float(alpha), _ptr(sfp), _ptr(g), _ptr(gx), _ptr(gc),
+                                  _ptr(gd), _ptr(gs), _ptr(gca), _ptr(gda), _ptr(gsa), _ptr(gc64),
+                                  _ptr(gd64)))
     out = {}
     if want_gx:
         out["gx"] = gx
@@ -229,6 +235,10 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
             out["gdgs_abs"] = gda
     if want_f64:
         out["gcrs64"], out["gdgs64"] = gc64, gd64
+    if want_gsfp:
+        out["gsfp"] = gs
+        if want_abs:
+            out["gsfp_abs"] = gsa
     return out
 
 

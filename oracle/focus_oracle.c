@@ -191,6 +191,34 @@ static float block_scale(int fmt, int mx_rule, float m, float alpha, uint8_t* by
     return focus_oracle_e4m3_decode(b) * alpha;
 }
 
+/* Hardware scale from a learnable full-precision scale S^fp (Eq. 4):
+ * S^dq = Q_fmt(S^fp), the scale kept in full precision and quantized to the
+ * hardware format on the fly.  MXFP4: S^fp is the block scale, rounded up to
+ * a power of two (the ceiling reading of Eq. 3, so that S^fp = fl(m/6) gives
+ * the absmax scale).  NVFP4: alpha stays frozen and S^fp is the learnable
+ * Delta^fp, S^dq = alpha * Q_E4M3(Delta^fp) (so that S^fp = fl(m/fl(alpha*6))
+ * gives the absmax scale). */
+static float block_scale_fp(int fmt, float sfp, float alpha, uint8_t* byte)
+{
+    if (fmt == OR_MXFP4) {
+        int e;
+        if (sfp == 0.0f) {
+            e = -127;
+        } else {
+            int E;
+            float f = frexpf(sfp, &E);
+            e = (f == 0.5f) ? E - 1 : E;
+        }
+        if (e < -127) e = -127;
+        if (e > 127) e = 127;
+        *byte = (uint8_t)(e + 127);
+        return ldexpf(1.0f, e);
+    }
+    uint8_t b = focus_oracle_e4m3_encode(sfp);
+    *byte = b;
+    return focus_oracle_e4m3_decode(b) * alpha;
+}
+
 /* ------------------------------------------------------------------ */
 /* helpers                                                             */
 /* ------------------------------------------------------------------ */
@@ -240,8 +268,13 @@ static float block_absmax(int dtype, const void* x, int64_t base, int block)
 
 static int check_inputs(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                         int block, int sub, int shared, const void* x,
-                        const float* crs, const float* dgs, float alpha)
+                        const float* crs, const float* dgs, float alpha, const float* sfp)
 {
+    if (sfp) {
+        if (shared) return -1;             /* learnable scales are per weight block */
+        for (int64_t i = 0; i < rows * (cols / block); i++)
+            if (!(isfinite(sfp[i]) && sfp[i] >= 0.0f)) return -2;
+    }
     for (int64_t r = 0; r < rows; r++)
         for (int64_t j = 0; j < cols; j++)
             if (!isfinite(load_elem(dtype, x, r * ld + j))) return -2;
@@ -293,12 +326,12 @@ int focus_oracle_alpha(int dtype, int64_t rows, int64_t cols, int64_t ld,
 int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                      int block, int sub, int shared, int mx_rule,
                      const void* x, const float* crs, const float* dgs, float alpha,
-                     void* y, uint8_t* scales, uint8_t* codes)
+                     const float* sfp, void* y, uint8_t* scales, uint8_t* codes)
 {
     if (check_shape(rows, cols, ld, block, sub, dtype)) return -1;
     if (fmt != OR_MXFP4 && fmt != OR_NVFP4) return -1;
     if (rows > 0 && cols > 0 && !x) return -1;
-    int rc = check_inputs(fmt, dtype, rows, cols, ld, block, sub, shared, x, crs, dgs, alpha);
+    int rc = check_inputs(fmt, dtype, rows, cols, ld, block, sub, shared, x, crs, dgs, alpha, sfp);
     if (rc) return rc;
     const int64_t nblk = cols / block, nsub = cols / sub;
     const int K = block / sub;
@@ -306,9 +339,10 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
     for (int64_t r = 0; r < rows; r++) {
         for (int64_t j = 0; j < nblk; j++) {
             const int64_t base = r * ld + j * block;
-            float m = block_absmax(dtype, x, base, block);
             uint8_t sbyte;
-            float s_dq = block_scale(fmt, mx_rule, m, alpha, &sbyte);
+            float s_dq = sfp ? block_scale_fp(fmt, sfp[r * nblk + j], alpha, &sbyte)
+                             : block_scale(fmt, mx_rule, block_absmax(dtype, x, base, block),
+                                           alpha, &sbyte);
             if (scales) scales[r * nblk + j] = sbyte;
             float c = crs ? crs[(shared ? 0 : r * nblk) + j] : 1.0f;
             for (int k = 0; k < K; k++) {
@@ -352,6 +386,10 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
  *   dL/dc_i^k = -T_ik * c_i / c_eff^2
  *   dL/dc_i   = sum_k -T_ik * c_i^k / c_eff^2
  * In shared mode (one coefficient set for all rows) both also sum over rows.
+ * With the hardware scale from a learnable S^fp (Eq. 4), the STE also gives
+ *   dL/dS^dq_i = sum over block i of g * (q - mask * x / S^q)
+ * (q = E2M1 value; y = q(x / S^q) * S^dq) and dL/dS^fp_i = dL/dS^dq_i for
+ * MXFP4, alpha * dL/dS^dq_i for NVFP4 (STE through Q_fmt).
  * Optional outputs gcrs_abs / gdgs_abs receive the same sums taken over
  * |mask*g*x| (the scale of the terms, used to bound rounding error), and
  * gcrs64 / gdgs64 the gradients themselves before the final rounding to
@@ -359,14 +397,16 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
 int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                      int block, int sub, int shared, int ste, int mx_rule,
                      const void* x, const float* crs, const float* dgs, float alpha,
-                     const void* g, void* gx, float* gcrs, float* gdgs,
-                     double* gcrs_abs, double* gdgs_abs, double* gcrs64, double* gdgs64)
+                     const float* sfp, const void* g, void* gx, float* gcrs, float* gdgs,
+                     float* gsfp, double* gcrs_abs, double* gdgs_abs, double* gsfp_abs,
+                     double* gcrs64, double* gdgs64)
 {
     if (check_shape(rows, cols, ld, block, sub, dtype)) return -1;
     if (fmt != OR_MXFP4 && fmt != OR_NVFP4) return -1;
     if (ste != OR_STE_IDENTITY && ste != OR_STE_CLIPPED) return -1;
     if (rows > 0 && cols > 0 && (!x || !g)) return -1;
-    int rc = check_inputs(fmt, dtype, rows, cols, ld, block, sub, shared, x, crs, dgs, alpha);
+    if ((gsfp || gsfp_abs) && shared) return -1;
+    int rc = check_inputs(fmt, dtype, rows, cols, ld, block, sub, shared, x, crs, dgs, alpha, sfp);
     if (rc) return rc;
     for (int64_t r = 0; r < rows; r++)
         for (int64_t j = 0; j < cols; j++)
@@ -391,11 +431,12 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
     for (int64_t r = 0; r < rows; r++) {
         for (int64_t j = 0; j < nblk; j++) {
             const int64_t base = r * ld + j * block;
-            float m = block_absmax(dtype, x, base, block);
             uint8_t sbyte;
-            float s_dq = block_scale(fmt, mx_rule, m, alpha, &sbyte);
+            float s_dq = sfp ? block_scale_fp(fmt, sfp[r * nblk + j], alpha, &sbyte)
+                             : block_scale(fmt, mx_rule, block_absmax(dtype, x, base, block),
+                                           alpha, &sbyte);
             float c = crs ? crs[(shared ? 0 : r * nblk) + j] : 1.0f;
-            ksum_t gc = zero, gca = zero;
+            ksum_t gc = zero, gca = zero, gs = zero, gsa = zero;
             for (int k = 0; k < K; k++) {
                 float d = dgs ? dgs[(shared ? 0 : r * nsub) + j * K + k] : 1.0f;
                 float c_eff = c * d;
@@ -411,17 +452,24 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                     float gv = load_elem(dtype, g, r * ld + col);
                     float gxv = 0.0f;
                     if (!dead) {
+                        float u = xv / s_q;
                         int mask = 1;
-                        if (ste == OR_STE_CLIPPED) {
-                            float u = xv / s_q;
-                            mask = fabsf(u) <= 6.0f;
-                        }
+                        if (ste == OR_STE_CLIPPED) mask = fabsf(u) <= 6.0f;
                         if (mask) {
                             gxv = gv * rho;
                             double p = (double)gv * (double)xv;   /* exact */
                             ksum_add(&T, p);
                             ksum_add(&Ta, fabs(p));
                         }
+                        /* dy/dS^dq = q + S^dq * mask * du/dS^dq = q - mask * x / S^q,
+                         * q from the forward's code, S^q = S^dq * c_i * c_i^k taken
+                         * exactly like c_eff below */
+                        double q = focus_oracle_e2m1_value(focus_oracle_e2m1_code(u));
+                        double sq_exact = (double)s_dq * ((double)c * (double)d);
+                        double gq = (double)gv * q;
+                        double gu = mask ? (double)gv * (double)xv / sq_exact : 0.0;
+                        ksum_add(&gs, gq - gu);
+                        ksum_add(&gsa, fabs(gq) + fabs(gu));
                     }
                     if (gx) store_elem(dtype, gx, r * ld + col, gxv);
                 }
@@ -446,6 +494,10 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                 if (gcrs) gcrs[r * nblk + j] = (float)ksum_value(&gc);
                 if (gcrs_abs) gcrs_abs[r * nblk + j] = ksum_value(&gca);
                 if (gcrs64) gcrs64[r * nblk + j] = ksum_value(&gc);
+                /* STE through Q_fmt: dS^dq/dS^fp = 1 (MXFP4), alpha (NVFP4) */
+                double ds = (fmt == OR_NVFP4) ? (double)alpha : 1.0;
+                if (gsfp) gsfp[r * nblk + j] = (float)(ksum_value(&gs) * ds);
+                if (gsfp_abs) gsfp_abs[r * nblk + j] = ksum_value(&gsa) * ds;
             }
         }
     }

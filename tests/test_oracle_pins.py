@@ -526,3 +526,116 @@ def test_oracle_rejects_bad_inputs():
         O.fwd(x, O.MXFP4)
     with pytest.raises(O.OracleError):
         O.fwd(np.ones((2, 30), np.float32), O.MXFP4)            # cols % block
+
+
+# ---------------------------------------------------------------------------
+# learnable full-precision scale S^fp (Eq. 4): S^dq = Q_fmt(S^fp)
+# ---------------------------------------------------------------------------
+def absmax_sfp(x, fmt, alpha=0.0):
+    """The paper's initialisation of S^fp "via absmax": fl(m / 6) for MXFP4,
+    fl(m / fl(alpha * 6)) (the unrounded Delta) for NVFP4, in float32."""
+    block = 32 if fmt == O.MXFP4 else 16
+    xf = W.bf16_bits_to_f32(x) if x.dtype == np.uint16 else x
+    rows, cols = xf.shape
+    m = np.abs(xf.reshape(rows, cols // block, block)).max(axis=2).astype(np.float32)
+    if fmt == O.MXFP4:
+        return (m / np.float32(6)).astype(np.float32)
+    den = np.float32(alpha) * np.float32(6)
+    return (m / den).astype(np.float32)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_absmax_initialised_sfp_is_the_absmax_scale(fmt):
+    """S^fp initialised via absmax (Sec. 3.2) gives S^dq = Q_fmt(S^fp) equal
+    to the absmax scale of Eq. 2-3: every output is identical."""
+    w = W.WORKLOADS["llama3_8b_block"]
+    x = W.to_bf16_bits(W.draw_values(w, 24, 256, 61))
+    x[0, :32] = 0
+    g = W.to_bf16_bits(W.draw_grad(24, 256, 62))
+    block = 32 if fmt == O.MXFP4 else 16
+    crs = W.draw_coefs(w, 24 * 256 // block, 63).reshape(24, -1)
+    dgs = W.draw_coefs(w, 24 * 256 // 8, 64).reshape(24, -1)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    sfp = absmax_sfp(x, fmt, a)
+    f0 = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a, want_codes=True)
+    f1 = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a, want_codes=True, sfp=sfp)
+    for k in ("y", "codes", "scales"):
+        assert np.array_equal(f0[k], f1[k]), k
+    b0 = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a)
+    b1 = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a, sfp=sfp, want_gsfp=True)
+    for k in ("gx", "gcrs", "gdgs"):
+        assert np.array_equal(b0[k], b1[k]), k
+
+
+def test_hand_mxfp4_sfp_gradient():
+    """dL/dS^dq = sum g (q - x / S^q): block [0.7, -0.26, 0.13, 1.5, 0...],
+    S^dq = 0.25, c = 1.25 (S^q = 0.3125), g = 1 on the first four:
+    (2 - 2.24) + (-1 + 0.832) + (0.5 - 0.416) + (4 - 4.8) = -1.124."""
+    x = np.zeros((1, 32), np.float32)
+    x[0, :4] = [0.7, -0.26, 0.13, 1.5]
+    g = np.zeros_like(x)
+    g[0, :4] = 1
+    b = O.bwd(x, g, O.MXFP4, crs=np.array([[1.25]], np.float32), sfp=np.array([[0.25]], np.float32),
+              want_gsfp=True)
+    u = x[0, :4].astype(np.float64) / 0.3125
+    expect = float(np.sum(np.array([2.0, -1.0, 0.5, 4.0]) - u))
+    assert b["gsfp"][0, 0] == pytest.approx(expect, rel=1e-7)
+    assert expect == pytest.approx(-1.124, abs=1e-6)
+
+
+def test_sfp_rounding_rules():
+    """Q_E8M0 rounds S^fp up to a power of two; Q_E4M3 is round-to-nearest-even
+    (checked against torch's float8_e4m3fn)."""
+    x = np.full((4, 32), 0.01, np.float32)
+    sfp = np.array([[2.0 ** -5], [2.0 ** -5 * 1.0000001], [2.0 ** -5 * 1.9], [3e-3]], np.float32)
+    sc = O.fwd(x, O.MXFP4, sfp=sfp)["scales"][:, 0].astype(int) - 127
+    assert list(sc) == [-5, -4, -4, int(np.ceil(np.log2(np.float64(np.float32(3e-3)))))]
+    rng = np.random.default_rng(71)
+    d = rng.uniform(0, 460, 512).astype(np.float32)
+    xn = np.full((512, 16), 0.01, np.float32)
+    out = O.fwd(xn, O.NVFP4, alpha=1.0 / 2688, sfp=d.reshape(-1, 1))
+    assert np.array_equal(out["scales"][:, 0], torch_e4m3(d))
+
+
+def torch_fake_quant_sfp(x, sfp, crs, dgs, fmt, alpha, block, sub):
+    """Autograd restatement with the scale learned through Q_fmt by STE:
+    S^dq = S^fp + (Q_fmt(S^fp) - S^fp).detach() (times alpha for NVFP4)."""
+    c = crs.repeat_interleave(block, dim=1)
+    d = dgs.repeat_interleave(sub, dim=1)
+    sf = sfp.detach().numpy().astype(np.float32)
+    if fmt == O.MXFP4:
+        q = np.exp2(np.ceil(np.log2(sf.astype(np.float64))))
+        s = sfp + (torch.from_numpy(q) - sfp).detach()
+    else:
+        # the forward's scale is fl(alpha * Delta) in binary32; the STE carries
+        # d S^dq / d Delta^fp = alpha
+        dq = torch.from_numpy(torch_e4m3(sf)).view(torch.float8_e4m3fn).float()
+        sdq = (dq * torch.tensor(alpha, dtype=torch.float32)).double()
+        s = sdq + alpha * (sfp - sfp.detach())
+    s = s.repeat_interleave(block, dim=1)
+    u = x / (s * (c * d))
+    qv = torch.from_numpy(e2m1_ref(u.detach().numpy()))
+    return (u + (qv - u).detach()) * s
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_sfp_gradient_autograd(fmt):
+    rng = np.random.default_rng(81)
+    block = 32 if fmt == O.MXFP4 else 16
+    rows, cols = 5, 4 * block
+    x = (rng.standard_normal((rows, cols)) * 0.02).astype(np.float32)
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    crs = rng.uniform(0.8, 1.2, (rows, cols // block)).astype(np.float32)
+    dgs = rng.uniform(0.8, 1.2, (rows, cols // 8)).astype(np.float32)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    sfp = (absmax_sfp(x, fmt, a) * rng.uniform(0.7, 1.3, (rows, cols // block))).astype(np.float32)
+    ours = O.bwd(x, g, fmt, crs=crs, dgs=dgs, alpha=a, sfp=sfp, want_gsfp=True)
+    s6 = torch.from_numpy(sfp.astype(np.float64)).requires_grad_(True)
+    y = torch_fake_quant_sfp(torch.from_numpy(x.astype(np.float64)), s6,
+                             torch.from_numpy(crs.astype(np.float64)),
+                             torch.from_numpy(dgs.astype(np.float64)), fmt, float(a), block, 8)
+    y.backward(torch.from_numpy(g.astype(np.float64)))
+    np.testing.assert_allclose(ours["gsfp"], s6.grad.numpy(), rtol=1e-5, atol=1e-12)
+    # the forward of the restatement is the oracle's (values, through fp64)
+    fw = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a, sfp=sfp)
+    np.testing.assert_allclose(y.detach().numpy(), fw["y"].astype(np.float64), rtol=1e-6, atol=0)
