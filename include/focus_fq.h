@@ -141,13 +141,20 @@ int focus_nvfp4_alpha_noalloc(const focus_desc_t* desc, const void* x, float* al
  * dgs    DGS coefficients c_i^k, or NULL for 1 (Eq. 8).
  * alpha  NVFP4: device pointer to the fp32 per-tensor scale (required);
  *        MXFP4: ignored (may be NULL).
+ * sfp    optional learnable full-precision scales S^fp, dense fp32
+ *        [rows, cols/block], finite and >= 0 (Eq. 4): S^dq = Q_fmt(S^fp)
+ *        replaces the absmax scale -- MXFP4: the ceiling power of two of
+ *        S^fp (mx_rule is not used); NVFP4: S^fp is the learnable Delta,
+ *        S^dq = alpha * Q_E4M3(S^fp) with alpha frozen.  NULL: the absmax
+ *        scale of Eq. 2-3.  Not with coef_shared_rows = 1 (INVALID_ARG).
  * y      [rows, ld] output in dtype (may alias nothing else).
  * scale_bytes  optional [rows, cols/block] output of the stored scale bytes. */
 int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
-                 const float* dgs, const float* alpha, void* y, uint8_t* scale_bytes,
-                 focus_stream_t stream);
+                 const float* dgs, const float* alpha, const float* sfp, void* y,
+                 uint8_t* scale_bytes, focus_stream_t stream);
 
 /* Straight-through-estimator backward (Sec. 3.2) of focus_fq_fwd.
+ * x, crs, dgs, alpha, sfp  as for focus_fq_fwd.
  * g      [rows, ld] upstream gradient dL/dy (dtype).
  * gx     optional [rows, ld] output dL/dx = mask * fl(fl(g * S^dq) / S^q);
  *        NULL skips it (frozen weights, Sec. 3.2).
@@ -157,22 +164,28 @@ int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
  *        both are also summed over rows.  They are written (not accumulated).
  *        Requesting gcrs with crs == NULL gives the gradient at c_i = 1
  *        (likewise gdgs with dgs == NULL).
+ * gsfp   optional [rows, cols/block] output dL/dS^fp (Eq. 4 with the STE
+ *        through Q_fmt): dL/dS^dq_i = sum over block i of
+ *        g * (q - mask * x / S^q) (q the E2M1 value, S^q = S^dq c_i c_i^k
+ *        taken exactly), times alpha for NVFP4.  With sfp == NULL it is the
+ *        gradient at the absmax initialisation.  Per-row coefficients only.
  * ws     device scratch of focus_workspace_bytes(desc, FOCUS_WS_BWD) bytes
  *        (zero when coef_shared_rows == 0, in which case ws may be NULL).
  * Coefficient gradients are computed with compensated (double-fp32)
  * arithmetic and match an exact evaluation to about 1e-5 relative. */
 int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,
-                 const float* dgs, const float* alpha, const void* g, void* gx,
-                 float* gcrs, float* gdgs, void* ws, size_t ws_bytes,
+                 const float* dgs, const float* alpha, const float* sfp, const void* g,
+                 void* gx, float* gcrs, float* gdgs, float* gsfp, void* ws, size_t ws_bytes,
                  focus_stream_t stream);
 
 /* Export (Fig. 3(d)): the FP4 codes of Q_E2M1(x / S^q) and the scale bytes
  * of S^dq -- what the deployed MXFP4 / NVFP4 model stores; S^q and the
  * coefficients are not part of it.  NVFP4 also needs the caller's alpha.
+ * x, crs, dgs, alpha, sfp  as for focus_fq_fwd.
  * codes        [rows, cols/2] uint8 output (required).
  * scale_bytes  [rows, cols/block] uint8 output (required). */
 int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
-               const float* dgs, const float* alpha, uint8_t* codes,
+               const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
                uint8_t* scale_bytes, focus_stream_t stream);
 
 /* Device scratch (bytes) that focus_nvfp4_alpha (which = FOCUS_WS_ALPHA) or
@@ -183,7 +196,7 @@ size_t focus_workspace_bytes(const focus_desc_t* desc, int which);
 /* Static, NUL-terminated description of a status code. */
 const char* focus_status_string(int status);
 
-/* ABI version of this library (major * 100 + minor). */
+/* ABI version of this library (major * 100 + minor): 200. */
 int focus_version(void);
 
 #ifdef __cplusplus

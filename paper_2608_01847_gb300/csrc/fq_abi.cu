@@ -110,7 +110,7 @@ size_t bwd_ws_bytes(const focus_desc_t* d)
 
 using namespace focus;
 
-FOCUS_API int focus_version(void) { return 100; }
+FOCUS_API int focus_version(void) { return 200; }
 
 FOCUS_API const char* focus_status_string(int status)
 {
@@ -156,14 +156,16 @@ FOCUS_API int focus_nvfp4_alpha(const focus_desc_t* desc, const void* x, float* 
 }
 
 FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
-                           const float* dgs, const float* alpha, void* y, uint8_t* scale_bytes,
-                           focus_stream_t stream)
+                           const float* dgs, const float* alpha, const float* sfp, void* y,
+                           uint8_t* scale_bytes, focus_stream_t stream)
 {
     int rc = check_desc(desc, true);
     if (rc) return rc;
+    if (sfp && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !y || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 32) || misaligned(y, 32) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if (misaligned(x, 32) || misaligned(y, 32) || misaligned(alpha, 4) || misaligned(sfp, 4))
+        return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
     p.x = x;
@@ -171,27 +173,31 @@ FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float*
     p.crs = crs;
     p.dgs = dgs;
     p.alpha = alpha;
+    p.sfp = sfp;
     p.scales = scale_bytes;
     return map_cuda(launch_fwd(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p,
                                reinterpret_cast<cudaStream_t>(stream)));
 }
 
 FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
-                         const float* dgs, const float* alpha, uint8_t* codes,
+                         const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
                          uint8_t* scale_bytes, focus_stream_t stream)
 {
     int rc = check_desc(desc, true);
     if (rc) return rc;
+    if (sfp && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !codes || !scale_bytes || (desc->fmt == FOCUS_NVFP4 && !alpha))
         return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 32) || misaligned(codes, 16) || misaligned(alpha, 4)) return FOCUS_ERR_MISALIGNED;
+    if (misaligned(x, 32) || misaligned(codes, 16) || misaligned(alpha, 4) || misaligned(sfp, 4))
+        return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
     p.x = x;
     p.crs = crs;
     p.dgs = dgs;
     p.alpha = alpha;
+    p.sfp = sfp;
     p.codes = codes;
     p.scales = scale_bytes;
     return map_cuda(launch_pack(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p,
@@ -199,15 +205,17 @@ FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* c
 }
 
 FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,
-                           const float* dgs, const float* alpha, const void* g, void* gx,
-                           float* gcrs, float* gdgs, void* ws, size_t ws_bytes,
-                           focus_stream_t stream)
+                           const float* dgs, const float* alpha, const float* sfp, const void* g,
+                           void* gx, float* gcrs, float* gdgs, float* gsfp, void* ws,
+                           size_t ws_bytes, focus_stream_t stream)
 {
     int rc = check_desc(desc, true);
     if (rc) return rc;
+    if ((sfp || gsfp) && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool want_T = gcrs != nullptr || gdgs != nullptr;
-    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4))
+    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4) ||
+        misaligned(sfp, 4) || misaligned(gsfp, 4))
         return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
     if (desc->rows == 0 || desc->cols == 0) {
@@ -222,7 +230,7 @@ FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float*
         return FOCUS_OK;
     }
     if (!x || !g || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
-    if (!gx && !want_T) return FOCUS_OK;
+    if (!gx && !want_T && !gsfp) return FOCUS_OK;
     KParams p = make_params(desc);
     p.x = x;
     p.g = g;
@@ -230,8 +238,10 @@ FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float*
     p.crs = crs;
     p.dgs = dgs;
     p.alpha = alpha;
+    p.sfp = sfp;
     p.gcrs = gcrs;
     p.gdgs = gdgs;
+    p.gsfp = gsfp;
     const int sub = effective_sub(desc, dgs, gdgs);
     if (desc->coef_shared_rows && want_T) {
         const size_t need = bwd_ws_bytes(desc);

@@ -147,6 +147,17 @@ __device__ __forceinline__ int mx_exponent(float m, int rule)
     return min(max(e, -127), 127);
 }
 
+// ceil(log2 t) for t >= 0 clamped to [-127, 127], exact from the bits of t
+// (t = 0 gives -127): the Q_E8M0 ceiling of Eq. 3 applied to a scale.
+__device__ __forceinline__ int mx_ceil_exponent(float t)
+{
+    const uint32_t b = __float_as_uint(t);
+    const int E = static_cast<int>(b >> 23);
+    const uint32_t M = b & 0x7fffffu;
+    const int e = (E == 0) ? (M > 0x400000u ? -126 : -127) : (E - 127 + (M != 0u ? 1 : 0));
+    return min(max(e, -127), 127);
+}
+
 // 2^e for e in [-127, 127] (2^-127 is the subnormal 0x00400000).
 __device__ __forceinline__ float exp2_int(int e)
 {

@@ -32,6 +32,7 @@ cudaError_t bwd_shared_by_sub(int sub, const KParams& p, uint32_t ny, cudaStream
 
 cudaError_t launch_bwd_nv(int dt, int sub, const KParams& p, cudaStream_t st)
 {
+    if (p.gsfp) return dt ? linear_by_sub<1, 1, kBwdS>(sub, p, st) : linear_by_sub<1, 0, kBwdS>(sub, p, st);
     return dt ? linear_by_sub<1, 1, kBwd>(sub, p, st) : linear_by_sub<1, 0, kBwd>(sub, p, st);
 }
 

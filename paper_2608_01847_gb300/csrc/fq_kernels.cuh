@@ -26,7 +26,7 @@
 namespace focus {
 
 constexpr int kThreads = 256;
-enum Mode { kFwd = 0, kPack = 1, kBwd = 2 };
+enum Mode { kFwd = 0, kPack = 1, kBwd = 2, kBwdS = 3 };  // kBwdS: backward + dL/dS^fp
 
 struct KParams {
     const void* x;
@@ -36,8 +36,10 @@ struct KParams {
     const float* crs;
     const float* dgs;
     const float* alpha;
+    const float* sfp;     // learnable full-precision scales (Eq. 4), or null
     float* gcrs;
     float* gdgs;
+    float* gsfp;
     uint8_t* codes;
     uint8_t* scales;
     float* ws;            // scratch: per-CTA partials
@@ -205,6 +207,21 @@ __device__ __forceinline__ float block_scale(float m, const TensorScale& ts, int
     return nv_scale(m, ts.alpha, ts.den, ts.bd, byte);
 }
 
+// Hardware scale from a learnable full-precision scale (Eq. 4):
+// S^dq = Q_fmt(S^fp).  MXFP4: the ceiling power of two of S^fp (exact, from
+// its bits); NVFP4: alpha * Q_E4M3(S^fp), S^fp being the learnable Delta.
+template <int FMT>
+__device__ __forceinline__ float block_scale_fp(float sfp, const TensorScale& ts, uint32_t& byte)
+{
+    if (FMT == 0) {
+        const int e = mx_ceil_exponent(sfp);
+        byte = static_cast<uint32_t>(e + 127);
+        return exp2_int(e);
+    }
+    byte = e4m3_encode(sfp);
+    return __fmul_rn(e4m3_decode(byte), ts.alpha);
+}
+
 // S^q per sub-block; "dead" when S^dq or S^q is zero or infinite (outputs
 // +0, no gradient).
 template <int K>
@@ -348,12 +365,13 @@ __device__ __forceinline__ df sum2x2_merge(const Sum2x2& a)
 //   gd_k = -(T_k / d_k) / (c d_k),   gc = -(sum_k T_k / d_k) / c^2,
 // with T_k / d_k in double-fp32 and the sum over k compensated.
 // ---------------------------------------------------------------------------
-template <int DT, int B, int K>
+template <int DT, int B, int K, bool SFPG>
 __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw,
                                           const float (&sq)[K], const bool (&dead)[K],
                                           const float (&rho)[K], float c, const float (&d)[K],
-                                          int ste, bool want_gx, bool want_T, void* gx_base,
-                                          uint64_t off, float (&gd)[K], float& gc, df (&T)[K])
+                                          float sdq, int ste, bool want_gx, bool want_T,
+                                          void* gx_base, uint64_t off, float (&gd)[K], float& gc,
+                                          df (&T)[K], df& gS)
 {
     constexpr int SUB = B / K;
     constexpr int EPG = DT == 1 ? 16 : 8;  // elements per 256-bit group
@@ -361,13 +379,33 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
     const float rc = rcp_approx(c);
     df Q = {0.0f, 0.0f};
     uint32_t grp[8];
+    // dL/dS^dq needs the forward's E2M1 values q
+    uint32_t codes[SFPG ? B / 8 : 1];
+    if constexpr (SFPG) block_codes<DT, B, K>(xw, sq, dead, codes);
+    const float rs = SFPG ? rcp_approx(sdq) : 0.0f;
+    gS = {0.0f, 0.0f};
 #pragma unroll
     for (int k = 0; k < K; ++k) {
-        Sum2x2 acc;
+        Sum2x2 acc, accq;
 #pragma unroll
         for (int e = k * SUB; e < (k + 1) * SUB; e += 2) {
             const float2 x2 = elem_pair<DT>(xw, e / 2);
             float2 g2 = elem_pair<DT>(gw, e / 2);
+            if constexpr (SFPG) {
+                // g * q over the sub-block (q: 2 significant bits, so exact
+                // for bf16 g); the q term of dy/dS^dq is not masked
+                const uint32_t cb = (codes[e / 8] >> (4 * (e % 8))) & 0xffu;
+                const uint32_t h2 = e2m1x2_to_f16x2(cb);
+                const float2 q2 = __half22float2(*reinterpret_cast<const __half2*>(&h2));
+                const float2 p = mul2(g2, q2);
+                if (e == k * SUB) {
+                    accq.s = p;
+                    accq.c = make_float2(0.0f, 0.0f);
+                } else {
+                    sum2x2_add(accq, p);
+                }
+                if (DT == 0) accq.c = add2(accq.c, fma2(g2, q2, make_float2(-p.x, -p.y)));
+            }
             if (ste == 1) {
                 g2.x = ((live >> e) & 1u) ? g2.x : 0.0f;
                 g2.y = ((live >> (e + 1)) & 1u) ? g2.y : 0.0f;
@@ -397,6 +435,13 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
             const df qk = df_div_f(T[k], d[k], rd);
             gd[k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
             Q = (k == 0) ? qk : df_add(Q, qk);
+            if constexpr (SFPG) {
+                // dL/dS^dq over the sub-block: sum g q - T_k / (S^dq c c^k)
+                if (!dead[k]) {
+                    const df u = df_div_f(df_div_f(qk, c, rc), sdq, rs);
+                    gS = df_add(gS, df_add(sum2x2_merge(accq), df{-u.h, -u.l}));
+                }
+            }
         }
     }
     gc = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
@@ -427,7 +472,7 @@ template <int FMT, int DT, int MODE>
 struct Unroll {
     // blocks per thread per step: 64 bytes of x in flight for the streaming
     // passes, one block (x and g) for the backward
-    static constexpr int U = (MODE == kBwd) ? 1 : ((FMT == 1 && DT == 1) ? 2 : 1);
+    static constexpr int U = (MODE >= kBwd) ? 1 : ((FMT == 1 && DT == 1) ? 2 : 1);
 };
 
 // Resident CTAs per SM the register allocation must allow: enough 256-thread
@@ -435,7 +480,8 @@ struct Unroll {
 // (one fewer for 2-element sub-blocks, whose per-sub-block state is largest).
 template <int FMT, int SUB, int MODE>
 struct MinCtas {
-    static constexpr int value = ((MODE == kBwd) ? (FMT == 1 ? 3 : 2) : 4) - (SUB == 2 ? 1 : 0);
+    static constexpr int value =
+        ((MODE == kBwd) ? (FMT == 1 ? 3 : 2) : (MODE == kBwdS ? 2 : 4)) - (SUB == 2 ? 1 : 0);
 };
 
 template <int FMT, int DT, int SUB, int MODE>
@@ -446,22 +492,25 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
     constexpr int B = G::B, K = G::K, W = G::W;
     constexpr int U = Unroll<FMT, DT, MODE>::U;
     constexpr int ESZ = DT == 1 ? 2 : 4;
+    constexpr bool BWD = MODE == kBwd || MODE == kBwdS;
     const TensorScale ts = tensor_scale<FMT>(p.alpha);
-    const bool want_gx = (MODE == kBwd) && p.gx != nullptr;
-    const bool want_T = (MODE == kBwd) && (p.gcrs != nullptr || p.gdgs != nullptr);
+    const bool want_gx = BWD && p.gx != nullptr;
+    const bool want_T = (MODE == kBwdS) || (BWD && (p.gcrs != nullptr || p.gdgs != nullptr));
     const uint32_t span = U * kThreads;
 
     for (uint32_t base = blockIdx.x * span; base < p.n_blocks; base += gridDim.x * span) {
         uint32_t xr[U][W];
-        uint32_t gr[MODE == kBwd ? U : 1][MODE == kBwd ? W : 1];
+        uint32_t gr[BWD ? U : 1][BWD ? W : 1];
         uint64_t off[U];
         float cv[U];
         float dv[U][K];
+        float sv[U];
         // ---- issue every load of this step first ----
 #pragma unroll
         for (int j = 0; j < U; ++j) {
             const uint32_t blk = base + j * kThreads + threadIdx.x;
             cv[j] = 1.0f;
+            sv[j] = 0.0f;
 #pragma unroll
             for (int k = 0; k < K; ++k) dv[j][k] = 1.0f;
             off[j] = 0;
@@ -475,14 +524,15 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                     off[j] = static_cast<uint64_t>(blk) * (B * ESZ);
                 }
                 load_block<W>(xr[j], p.x, off[j]);
-                if constexpr (MODE == kBwd) load_block<W>(gr[j], p.g, off[j]);
+                if constexpr (BWD) load_block<W>(gr[j], p.g, off[j]);
+                if (p.sfp) sv[j] = __ldg(p.sfp + blk);
                 const uint32_t q = p.shared ? cb : blk;
                 if (p.crs) cv[j] = __ldg(p.crs + q);
                 if (p.dgs) load_coefs<K>(p.dgs + static_cast<size_t>(q) * K, dv[j]);
             } else {
 #pragma unroll
                 for (int i = 0; i < W; ++i) xr[j][i] = 0u;
-                if constexpr (MODE == kBwd) {
+                if constexpr (BWD) {
 #pragma unroll
                     for (int i = 0; i < W; ++i) gr[j][i] = 0u;
                 }
@@ -494,12 +544,13 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
             const uint32_t blk = base + j * kThreads + threadIdx.x;
             if (blk >= p.n_blocks) continue;
             uint32_t sbyte;
-            const float sdq = block_scale<FMT>(block_absmax<DT, W>(xr[j]), ts, p.mx_rule, sbyte);
+            const float sdq = p.sfp ? block_scale_fp<FMT>(sv[j], ts, sbyte)
+                                    : block_scale<FMT>(block_absmax<DT, W>(xr[j]), ts, p.mx_rule, sbyte);
             float sq[K];
             bool dead[K];
             relaxed_scales<K>(sdq, cv[j], dv[j], sq, dead);
 
-            if constexpr (MODE != kBwd) {
+            if constexpr (!BWD) {
                 uint32_t codes[B / 8];
                 block_codes<DT, B, K>(xr[j], sq, dead, codes);
                 if constexpr (MODE == kFwd) {
@@ -533,12 +584,18 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                 float rho[K];
                 if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
                 float gd[K], gc;
-                df T[K];
-                block_bwd<DT, B, K>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], p.ste, want_gx,
-                                    want_T, p.gx, off[j], gd, gc, T);
+                df T[K], gS;
+                block_bwd<DT, B, K, MODE == kBwdS>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], sdq,
+                                                   p.ste, want_gx, want_T, p.gx, off[j], gd, gc,
+                                                   T, gS);
                 if (want_T) {
                     if (p.gdgs) store_coefs<K>(p.gdgs + static_cast<size_t>(blk) * K, gd);
                     if (p.gcrs) p.gcrs[blk] = gc;
+                }
+                if constexpr (MODE == kBwdS) {
+                    // STE through Q_fmt: dS^dq/dS^fp = 1 (MXFP4), alpha (NVFP4)
+                    const float v = df_to_f(gS);
+                    p.gsfp[blk] = (FMT == 1) ? __fmul_rn(v, ts.alpha) : v;
                 }
             }
         }
@@ -594,9 +651,9 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
             float rho[K];
             if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
             float gd[K], gc;
-            df T[K];
-            block_bwd<DT, B, K>(xr, gr, sq, dead, rho, c, d, p.ste, want_gx, true, p.gx, off,
-                                gd, gc, T);
+            df T[K], gS;
+            block_bwd<DT, B, K, false>(xr, gr, sq, dead, rho, c, d, sdq, p.ste, want_gx, true,
+                                       p.gx, off, gd, gc, T, gS);
 #pragma unroll
             for (int k = 0; k < K; ++k) acc[k] = df_add(acc[k], T[k]);
         }

@@ -60,9 +60,9 @@ def lib() -> ctypes.CDLL:
         P, D, SZ = ctypes.c_void_p, ctypes.POINTER(focus_desc_t), ctypes.c_size_t
         L.focus_nvfp4_alpha.argtypes = [D, P, P, P, SZ, P]
         L.focus_nvfp4_alpha_noalloc.argtypes = [D, P, P, P]
-        L.focus_fq_fwd.argtypes = [D, P, P, P, P, P, P, P]
-        L.focus_fq_bwd.argtypes = [D, P, P, P, P, P, P, P, P, P, SZ, P]
-        L.focus_pack.argtypes = [D, P, P, P, P, P, P, P]
+        L.focus_fq_fwd.argtypes = [D, P, P, P, P, P, P, P, P]
+        L.focus_fq_bwd.argtypes = [D, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
+        L.focus_pack.argtypes = [D, P, P, P, P, P, P, P, P]
         L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
         L.focus_workspace_bytes.restype = SZ
         L.focus_status_string.argtypes = [ctypes.c_int]
@@ -173,11 +173,17 @@ def focus_nvfp4_alpha_noalloc(x: torch.Tensor, alpha_out: torch.Tensor) -> torch
     return alpha_out
 
 
+def _check_sfp(x, fmt, t, name):
+    _dense(t, x.shape[0] * (x.shape[1] // block_of(fmt)), torch.float32, name)
+
+
 def focus_fq_fwd(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
-                 mx_rule=FOCUS_MX_CEIL, y=None, scale_bytes=None, want_scales=False):
-    """y = Q_E2M1(x / S^q) * S^dq (Eq. 1-8); returns y, or (y, scale_bytes)."""
+                 mx_rule=FOCUS_MX_CEIL, y=None, scale_bytes=None, want_scales=False, sfp=None):
+    """y = Q_E2M1(x / S^q) * S^dq (Eq. 1-8); returns y, or (y, scale_bytes).
+    sfp: optional learnable full-precision scales (Eq. 4)."""
     desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
     _check_coefs(x, fmt, sub_block, shared, crs, dgs)
+    _check_sfp(x, fmt, sfp, "sfp")
     if y is None:
         y = _like_x(x)
     _same_layout(x, y, "y")
@@ -185,16 +191,19 @@ def focus_fq_fwd(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=
         scale_bytes = torch.empty((x.shape[0], x.shape[1] // block_of(fmt)), dtype=torch.uint8,
                                   device=x.device)
     _dense(scale_bytes, x.shape[0] * (x.shape[1] // block_of(fmt)), torch.uint8, "scale_bytes")
-    _check(lib().focus_fq_fwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(y),
-                              _p(scale_bytes), _stream(x.device)), "focus_fq_fwd")
+    _check(lib().focus_fq_fwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(sfp),
+                              _p(y), _p(scale_bytes), _stream(x.device)), "focus_fq_fwd")
     return (y, scale_bytes) if (want_scales or scale_bytes is not None) else y
 
 
 def focus_fq_bwd(x, g, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
                  ste=FOCUS_STE_IDENTITY, mx_rule=FOCUS_MX_CEIL, want_gx=True, want_gcrs=None,
-                 want_gdgs=None, gx=None, gcrs=None, gdgs=None, ws=None):
-    """STE backward (Sec. 3.2): returns (gx, gcrs, gdgs); an unrequested output is None.
-    By default gcrs / gdgs are produced when crs / dgs are given."""
+                 want_gdgs=None, gx=None, gcrs=None, gdgs=None, ws=None, sfp=None,
+                 want_gsfp=None, gsfp=None):
+    """STE backward (Sec. 3.2): returns (gx, gcrs, gdgs) -- or (gx, gcrs, gdgs, gsfp)
+    when the S^fp gradient is requested (by default when sfp is given); an
+    unrequested output is None.  By default gcrs / gdgs are produced when
+    crs / dgs are given."""
     desc = make_desc(x, fmt, sub_block, shared, ste, mx_rule)
     rows, cols = x.shape
     crow = 1 if shared else rows
@@ -209,16 +218,24 @@ def focus_fq_bwd(x, g, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shar
         gcrs = torch.empty((crow, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
     if gdgs is None and want_gdgs:
         gdgs = torch.empty((crow, cols // sub_block), dtype=torch.float32, device=x.device)
+    want_gsfp = (sfp is not None or gsfp is not None) if want_gsfp is None else want_gsfp
+    if gsfp is None and want_gsfp:
+        gsfp = torch.empty((rows, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
+    _check_sfp(x, fmt, sfp, "sfp")
+    _check_sfp(x, fmt, gsfp, "gsfp")
     _check_coefs(x, fmt, sub_block, shared, gcrs, gdgs)
     ws, nb = _workspace(desc, FOCUS_WS_BWD, x.device, ws)
-    _check(lib().focus_fq_bwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(g),
-                              _p(gx), _p(gcrs), _p(gdgs), _p(ws), nb, _stream(x.device)),
+    _check(lib().focus_fq_bwd(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(sfp),
+                              _p(g), _p(gx), _p(gcrs), _p(gdgs), _p(gsfp), _p(ws), nb,
+                              _stream(x.device)),
            "focus_fq_bwd")
+    if want_gsfp:
+        return gx, gcrs, gdgs, gsfp
     return gx, gcrs, gdgs
 
 
 def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
-               mx_rule=FOCUS_MX_CEIL, codes=None, scale_bytes=None):
+               mx_rule=FOCUS_MX_CEIL, codes=None, scale_bytes=None, sfp=None):
     """Export (Fig. 3(d)): returns (codes [rows, cols/2] uint8, scale bytes [rows, cols/B])."""
     desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
     rows, cols = x.shape
@@ -229,8 +246,9 @@ def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=Fa
     _check_coefs(x, fmt, sub_block, shared, crs, dgs)
     _dense(codes, rows * cols // 2, torch.uint8, "codes")
     _dense(scale_bytes, rows * cols // block_of(fmt), torch.uint8, "scale_bytes")
-    _check(lib().focus_pack(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(codes),
-                            _p(scale_bytes), _stream(x.device)), "focus_pack")
+    _check_sfp(x, fmt, sfp, "sfp")
+    _check(lib().focus_pack(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(sfp),
+                            _p(codes), _p(scale_bytes), _stream(x.device)), "focus_pack")
     return codes, scale_bytes
 
 

@@ -47,7 +47,7 @@ def test_exports_exactly_the_declared_symbols(L):
 
 
 def test_version_and_status_strings(L):
-    assert F.focus_version() == 100
+    assert F.focus_version() == 200
     for code in (0, -1, -2, -3, -4, -5):
         assert L.focus_status_string(code)
     assert L.focus_status_string(42) == b"unknown status"
@@ -66,8 +66,9 @@ ODD = P(0x100010)           # 16-byte aligned only (rows need 32)
 ODD8 = P(0x100008)          # 8-byte aligned only (coefficient arrays need 16)
 
 
-def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None):
-    return L.focus_fq_fwd(ctypes.byref(d) if d is not None else None, x, crs, dgs, alpha, y, sb, None)
+def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None, sfp=None):
+    return L.focus_fq_fwd(ctypes.byref(d) if d is not None else None, x, crs, dgs, alpha, sfp, y,
+                          sb, None)
 
 
 @pytest.mark.parametrize("kw,status", [
@@ -91,13 +92,19 @@ def test_null_and_alignment_rejections(L):
     assert fwd(L, _desc(), crs=ODD8) == -3
     assert fwd(L, _desc(rows=0)) == 0                             # empty: nothing to do
     d = _desc()
-    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, None, ALIGNED2, None) == -1
-    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, P(0x100002), ALIGNED2, None) == -3
+    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, None, None, ALIGNED2,
+                        None) == -1
+    assert L.focus_pack(ctypes.byref(d), ALIGNED, None, None, None, None, P(0x100002), ALIGNED2,
+                        None) == -3
     g = ALIGNED2
-    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, g, None, None, None, 0,
-                          None) == -1                             # g missing
-    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, g, ODD, None, None, None, 0,
-                          None) == -3                             # gx misaligned
+    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, None, g, None, None,
+                          None, None, 0, None) == -1              # g missing
+    assert L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, g, ODD, None, None,
+                          None, None, 0, None) == -3              # gx misaligned
+    assert fwd(L, _desc(), sfp=P(0x100002)) == -3                 # S^fp must be 4-byte aligned
+    assert fwd(L, _desc(shared=1), sfp=ALIGNED2) == -1            # S^fp is per row
+    assert L.focus_fq_bwd(ctypes.byref(_desc(shared=1)), ALIGNED, None, None, None, None, g, None,
+                          None, None, ALIGNED2, None, 0, None) == -1
     assert L.focus_nvfp4_alpha(ctypes.byref(d), ALIGNED, None, ALIGNED2, 1 << 20, None) == -1
 
 
@@ -106,11 +113,11 @@ def test_shared_backward_needs_workspace(L):
     need = L.focus_workspace_bytes(ctypes.byref(d), F.FOCUS_WS_BWD)
     assert need > 0
     gc = ALIGNED2
-    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, ALIGNED2, None, gc, None,
-                        None, 0, None)
+    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, ALIGNED2, None, gc, None,
+                        None, None, 0, None)
     assert rc == -4
-    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, ALIGNED2, None, gc, None,
-                        ALIGNED, need - 1, None)
+    rc = L.focus_fq_bwd(ctypes.byref(d), ALIGNED, None, None, None, None, ALIGNED2, None, gc, None,
+                        None, ALIGNED, need - 1, None)
     assert rc == -4
     assert L.focus_nvfp4_alpha(ctypes.byref(d), ALIGNED, ALIGNED2, None, 0, None) == -4
 

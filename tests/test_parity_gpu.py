@@ -269,3 +269,74 @@ def test_deterministic():
     for a, b in zip(r1, r2):
         assert torch.equal(a.view(torch.int16) if a.dtype == torch.bfloat16 else a.view(torch.int32),
                            b.view(torch.int16) if b.dtype == torch.bfloat16 else b.view(torch.int32))
+
+
+# ---------------------------------------------------------------------------
+# learnable full-precision scale S^fp (Eq. 4)
+# ---------------------------------------------------------------------------
+def absmax_sfp_host(x, fmt, alpha):
+    block = 32 if fmt == O.MXFP4 else 16
+    xf = W.bf16_bits_to_f32(x) if x.dtype == np.uint16 else x
+    rows, cols = xf.shape
+    m = np.abs(xf.reshape(rows, cols // block, block)).max(axis=2).astype(np.float32)
+    den = np.float32(6) if fmt == O.MXFP4 else np.float32(alpha) * np.float32(6)
+    return (m / den).astype(np.float32)
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("sub", [8, 4])
+@pytest.mark.parametrize("ste", [O.STE_IDENTITY, O.STE_CLIPPED])
+def test_learnable_scale(fmt, dtype, sub, ste):
+    rows, cols = 96, 640
+    w, x, g = seeded(rows, cols, dtype, seed=7 + sub, coef=(0.8, 1.2))
+    f = FMT[fmt]
+    block = 32 if f == O.MXFP4 else 16
+    crs = W.draw_coefs(w, rows * cols // block, 14).reshape(rows, -1)
+    dgs = W.draw_coefs(w, rows * cols // sub, 15).reshape(rows, -1)
+    a = O.alpha(x) if f == O.NVFP4 else 0.0
+    jitter = W.draw_coefs(w, rows * cols // block, 16).reshape(rows, -1)
+    sfp = (absmax_sfp_host(x, f, a) * jitter).astype(np.float32)
+    sfp[3, :2] = 0.0                                   # zero scale: dead blocks
+    xd, gd, cd, dd, sd = dev(x), dev(g), dev(crs), dev(dgs), dev(sfp)
+    a_dev = torch.tensor([a], dtype=torch.float32, device="cuda") if f == O.NVFP4 else None
+    kw = dict(sub_block=sub, sfp=sd)
+    y, sb = F.focus_fq_fwd(xd, f, cd, dd, a_dev, want_scales=True, **kw)
+    codes, sb2 = F.focus_pack(xd, f, cd, dd, a_dev, **kw)
+    gx, gc, gdg, gs = F.focus_fq_bwd(xd, gd, f, cd, dd, a_dev, ste=ste, **kw)
+    torch.cuda.synchronize()
+    ref = O.fwd(x, f, crs=crs, dgs=dgs, alpha=a, sub=sub, sfp=sfp, want_codes=True)
+    rb = O.bwd(x, g, f, crs=crs, dgs=dgs, alpha=a, sub=sub, ste=ste, sfp=sfp, want_abs=True,
+               want_gsfp=True)
+    assert_bits_equal(host(y), ref["y"], "y")
+    assert_bits_equal(host(sb), ref["scales"], "scale bytes")
+    assert_bits_equal(host(sb2), ref["scales"], "scale bytes (pack)")
+    assert_bits_equal(host(codes), ref["codes"], "codes")
+    assert_bits_equal(host(gx), rb["gx"], "gx")
+    assert_grad_close(host(gc), rb["gcrs"], rb["gcrs_abs"], FLOOR_ROW, "dL/dc")
+    assert_grad_close(host(gdg), rb["gdgs"], rb["gdgs_abs"], FLOOR_ROW, "dL/dc^k")
+    assert_grad_close(host(gs), rb["gsfp"], rb["gsfp_abs"], FLOOR_ROW, "dL/dS^fp")
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_absmax_sfp_matches_absmax_path_on_gpu(fmt):
+    """S^fp initialised via absmax reproduces the absmax path bit for bit;
+    the S^fp gradient is also available without S^fp (at the absmax scale)."""
+    w, x, g = seeded(64, 512, "bf16", seed=31)
+    f = FMT[fmt]
+    block = 32 if f == O.MXFP4 else 16
+    crs = W.draw_coefs(w, 64 * 512 // block, 17).reshape(64, -1)
+    a = O.alpha(x) if f == O.NVFP4 else 0.0
+    sfp = absmax_sfp_host(x, f, a)
+    xd, gd, cd, sd = dev(x), dev(g), dev(crs), dev(sfp)
+    a_dev = torch.tensor([a], dtype=torch.float32, device="cuda") if f == O.NVFP4 else None
+    y0 = F.focus_fq_fwd(xd, f, cd, None, a_dev)
+    y1 = F.focus_fq_fwd(xd, f, cd, None, a_dev, sfp=sd)
+    r0 = F.focus_fq_bwd(xd, gd, f, cd, None, a_dev, want_gsfp=True)
+    r1 = F.focus_fq_bwd(xd, gd, f, cd, None, a_dev, sfp=sd)
+    torch.cuda.synchronize()
+    assert torch.equal(y0.view(torch.int16), y1.view(torch.int16))
+    assert torch.equal(r0[0].view(torch.int16), r1[0].view(torch.int16))
+    assert torch.equal(r0[1], r1[1]) and torch.equal(r0[3], r1[3])
+    rb = O.bwd(x, g, f, crs=crs, alpha=a, want_abs=True, want_gsfp=True)
+    assert_grad_close(host(r0[3]), rb["gsfp"], rb["gsfp_abs"], FLOOR_ROW, "dL/dS^fp at absmax")
