@@ -47,6 +47,7 @@ class Case:
     fmt: str = "nvfp4"
     sub: int = 8
     shared: bool = False       # one coefficient set for all rows (activations)
+    sfp: bool = False          # learnable full-precision scales S^fp (Eq. 4) and dL/dS^fp
 
     @property
     def block(self) -> int:
@@ -62,8 +63,9 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
     gradients out) per element unless shared by all rows; codes 0.5 B, one
     scale byte per block."""
     coef = 0.0 if case.shared else 4.0 / case.block + 4.0 / case.sub
-    out = {"fwd": 2 * esz + coef, "bwd": 3 * esz + 2 * coef,
-           "pack": esz + coef + 0.5 + 1.0 / case.block}
+    sfp = 4.0 / case.block if case.sfp else 0.0     # S^fp in (and dL/dS^fp out)
+    out = {"fwd": 2 * esz + coef + sfp, "bwd": 3 * esz + 2 * coef + 2 * sfp,
+           "pack": esz + coef + sfp + 0.5 + 1.0 / case.block}
     if case.fmt == "nvfp4":
         out["alpha"] = float(esz)
     return out
@@ -194,6 +196,20 @@ class Tensor:
                                     dtype=torch.uint8, device=device)
         self.ws_bwd = torch.empty(max(16, F.focus_workspace_bytes(d, F.FOCUS_WS_BWD)),
                                   dtype=torch.uint8, device=device)
+        self.sfp = self.gsfp = None
+        if case.sfp:
+            # S^fp initialised via absmax (Sec. 3.2), then moved by U(0.9, 1.1)
+            m = self.x.float().abs().view(rows, cols // case.block, case.block).amax(-1)
+            if case.fmt == "nvfp4":
+                F.focus_nvfp4_alpha(self.x, self.alpha, self.ws_alpha)
+                den = self.alpha * 6.0
+            else:
+                den = torch.full((1,), 6.0, device=device)
+            gen = torch.Generator(device=device)
+            gen.manual_seed(4242 + idx)
+            jit = torch.rand(m.shape, generator=gen, device=device) * 0.2 + 0.9
+            self.sfp = (m / den * jit).contiguous()
+            self.gsfp = torch.empty_like(self.sfp)
 
     def run(self, phase):
         from paper_2608_01847_gb300 import focus as F
@@ -202,14 +218,23 @@ class Tensor:
             F.focus_nvfp4_alpha(self.x, self.alpha, self.ws_alpha)
         elif phase == "fwd":
             F.focus_fq_fwd(self.x, self.fmt, self.crs, self.dgs, self.alpha, sub_block=c.sub,
-                           shared=c.shared, y=self.y)
+                           shared=c.shared, y=self.y, sfp=self.sfp)
         elif phase == "bwd":
             F.focus_fq_bwd(self.x, self.g, self.fmt, self.crs, self.dgs, self.alpha,
                            sub_block=c.sub, shared=c.shared, gx=self.gx, gcrs=self.gcrs,
-                           gdgs=self.gdgs, ws=self.ws_bwd)
+                           gdgs=self.gdgs, ws=self.ws_bwd, sfp=self.sfp, gsfp=self.gsfp)
         else:
             F.focus_pack(self.x, self.fmt, self.crs, self.dgs, self.alpha, sub_block=c.sub,
-                         shared=c.shared, codes=self.codes, scale_bytes=self.scales)
+                         shared=c.shared, codes=self.codes, scale_bytes=self.scales, sfp=self.sfp)
+
+    def inputs(self):
+        """Device tensors a step reads from the host (end-to-end leg)."""
+        return (self.x, self.g, self.crs, self.dgs) + ((self.sfp,) if self.sfp is not None else ())
+
+    def outputs(self):
+        """Device tensors a step returns to the host (end-to-end leg)."""
+        out = (self.y, self.gx, self.gcrs, self.gdgs, self.codes, self.scales)
+        return out + ((self.gsfp,) if self.gsfp is not None else ())
 
     def launches(self, phase):
         return 2 if phase == "alpha" else (2 if (phase == "bwd" and self.case.shared) else 1)
@@ -264,7 +289,7 @@ class PipelineGraph:
                 st.wait_stream(main)
             for t, hin, hout in zip(ts, host_in, host_out):
                 with torch.cuda.stream(s_in):
-                    for d, h in zip((t.x, t.g, t.crs, t.dgs), hin):
+                    for d, h in zip(t.inputs(), hin):
                         d.copy_(h, non_blocking=True)
                 s_cmp.wait_stream(s_in)
                 with torch.cuda.stream(s_cmp):
@@ -272,7 +297,7 @@ class PipelineGraph:
                         t.run(ph)
                 s_out.wait_stream(s_cmp)
                 with torch.cuda.stream(s_out):
-                    for h, d in zip(hout, (t.y, t.gx, t.gcrs, t.gdgs, t.codes, t.scales)):
+                    for h, d in zip(hout, t.outputs()):
                         h.copy_(d, non_blocking=True)
             for st in (s_in, s_cmp, s_out):
                 main.wait_stream(st)
@@ -352,9 +377,8 @@ def gpu_arm(case, args, rank, world, device):
     # (tensor after tensor), a compute chain (tensor k's phases once its
     # inputs are in HBM) and a D2H chain (tensor k's outputs once computed),
     # so that tensor k's D2H overlaps tensor k+1's H2D on the full-duplex link.
-    host_in = [[a.cpu().pin_memory() for a in (t.x, t.g, t.crs, t.dgs)] for t in ts]
-    host_out = [[torch.empty_like(a, device="cpu").pin_memory()
-                 for a in (t.y, t.gx, t.gcrs, t.gdgs, t.codes, t.scales)] for t in ts]
+    host_in = [[a.cpu().pin_memory() for a in t.inputs()] for t in ts]
+    host_out = [[torch.empty_like(a, device="cpu").pin_memory() for a in t.outputs()] for t in ts]
     h2d = sum(a.numel() * a.element_size() for h in host_in for a in h)
     d2h = sum(a.numel() * a.element_size() for h in host_out for a in h)
     e2e_graph = PipelineGraph(ts, host_in, host_out, phases, device)
@@ -380,15 +404,16 @@ def oracle_step(case, samples):
     """One pass of the oracle's alpha, fwd, bwd, pack over host samples."""
     import oracle as O
     fmt = O.NVFP4 if case.fmt == "nvfp4" else O.MXFP4
-    for x, g, crs, dgs in samples:
+    for x, g, crs, dgs, sfp in samples:
         a = O.alpha(x) if fmt == O.NVFP4 else 0.0
-        kw = dict(crs=crs, dgs=dgs, alpha=a, sub=case.sub, shared=case.shared)
+        kw = dict(crs=crs, dgs=dgs, alpha=a, sub=case.sub, shared=case.shared, sfp=sfp)
         O.fwd(x, fmt, want_scales=False, **kw)
-        O.bwd(x, g, fmt, **kw)
+        O.bwd(x, g, fmt, want_gsfp=sfp is not None, **kw)
         O.fwd(x, fmt, want_y=False, want_codes=True, **kw)
 
 
 def oracle_samples(case, rows_per_tensor):
+    import numpy as np
     from paper_2608_01847_gb300 import workloads as W
     w = W.WORKLOADS[case.workload]
     out = []
@@ -396,7 +421,17 @@ def oracle_samples(case, rows_per_tensor):
         x, g = W.host_tensor(w, i, rows=rows_per_tensor)
         crs, dgs = W.host_coefs(w, i, case.block, case.sub, shared=case.shared,
                                 rows=rows_per_tensor)
-        out.append((x, g, crs, dgs))
+        sfp = None
+        if case.sfp:
+            # absmax initialisation moved by U(0.9, 1.1), as on the device
+            xf = x.astype(np.uint32) << 16 if x.dtype == np.uint16 else x
+            m = np.abs(xf.view(np.float32)).reshape(x.shape[0], -1, case.block).max(-1)
+            den = np.float32(6.0)
+            if case.fmt == "nvfp4":
+                den = np.float32(m.max() / np.float32(2688.0)) * np.float32(6.0)
+            jit = np.random.default_rng(4242 + i).uniform(0.9, 1.1, m.shape).astype(np.float32)
+            sfp = np.ascontiguousarray(m / den * jit, dtype=np.float32)
+        out.append((x, g, crs, dgs, sfp))
     return out
 
 
@@ -406,7 +441,9 @@ def calibrate_oracle(case, target_s):
     t0 = time.perf_counter()
     oracle_step(case, probe)
     dt = max(time.perf_counter() - t0, 1e-6)
-    return max(1, min(int(8 * target_s / dt), 1 << 20))
+    from paper_2608_01847_gb300 import workloads as W
+    most = max(t.rows for t in W.WORKLOADS[case.workload].tensors)
+    return max(1, min(int(8 * target_s / dt), most))
 
 
 def sample_elems_and_bytes(case, samples):
@@ -449,7 +486,8 @@ def reference_arm(case, args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
             "config": {"workload": case.workload, "fmt": case.fmt, "sub_block": case.sub,
-                       "shared_coefficients": case.shared, "sample_rows_per_tensor": rows,
+                       "shared_coefficients": case.shared, "learnable_sfp": case.sfp,
+                       "sample_rows_per_tensor": rows,
                        "elements_per_step": n},
             "cpu_baseline": {"value": round(value, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
                              "sample": f"first {rows} rows of each tensor per step, "
@@ -469,10 +507,12 @@ def main():
     ap.add_argument("--fmt", default="nvfp4", choices=["nvfp4", "mxfp4"])
     ap.add_argument("--sub", type=int, default=8)
     ap.add_argument("--shared", action="store_true", help="coefficients shared by all rows")
+    ap.add_argument("--sfp", action="store_true",
+                    help="learnable full-precision scales S^fp and their gradient")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
-    case = Case(args.workload, args.fmt, args.sub, args.shared)
+    case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp)
     default_case = case == Case()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -528,6 +568,7 @@ def main():
                    "sub_block": case.sub,
                    "coefficients": ("shared by all rows" if case.shared else
                                     "per-block CRS + per-sub-block DGS"),
+                   "scales": "learnable S^fp (+ dL/dS^fp)" if case.sfp else "absmax",
                    "step": "+".join(case.phases()) + " over all tensors (bwd: gx + gcrs + gdgs)",
                    "bytes_per_elem": round(sum(bpe.values()), 4),
                    "l2": f"inputs larger than L2: x+g = {r['n_elem'] * 2 * r['esz'] / 2**20:.0f} MiB"

@@ -304,6 +304,44 @@ __device__ __forceinline__ void block_codes(const uint32_t* xw, const float (&sq
     for (int w = 0; w < B / 8; ++w) codes[w] &= live_word<SUB, K>(dead, w);
 }
 
+// E2M1 code word of elements 8w .. 8w+7 of a block (exact, as block_codes,
+// but one word at a time so that a caller streaming over the block keeps a
+// single word live).  br holds the sub-blocks' brackets.
+template <int DT, int B, int K>
+__device__ __forceinline__ uint32_t word_codes(const uint32_t* xw, int w, const float (&sq)[K],
+                                               const bool (&dead)[K], const Bracket (&br)[K])
+{
+    constexpr int SUB = B / K;
+    float lo[8], hi[8];
+    bool ok = true;
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) {
+        const int k = (8 * w + e) / SUB;
+        const float2 x2 = elem_pair<DT>(xw, (8 * w + e) / 2);
+        const float2 l2 = mul2(x2, make_float2(br[k].lo, br[k].lo));
+        const float2 h2 = mul2(x2, make_float2(br[k].hi, br[k].hi));
+        lo[e] = l2.x;
+        lo[e + 1] = l2.y;
+        hi[e] = h2.x;
+        hi[e + 1] = h2.y;
+        ok = ok & (dead[k] | br[k].ok);
+    }
+    const uint32_t live = live_word<SUB, K>(dead, w);
+    uint32_t c = e2m1_pack8(lo);
+    if (!ok | (((c ^ e2m1_pack8(hi)) & live) != 0u)) {
+        float u[8];
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) {
+            const int k = (8 * w + e) / SUB;
+            const float2 x2 = elem_pair<DT>(xw, (8 * w + e) / 2);
+            u[e] = __fdiv_rn(x2.x, sq[k]);
+            u[e + 1] = __fdiv_rn(x2.y, sq[k]);
+        }
+        c = e2m1_pack8(u);
+    }
+    return c & live;
+}
+
 // Clipping mask of the STE (|fl(x / S^q)| <= 6 on live sub-blocks), decided
 // on the brackets and exactly when they straddle 6.  Bit e = element e.
 template <int DT, int B, int K>
@@ -379,9 +417,13 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
     const float rc = rcp_approx(c);
     df Q = {0.0f, 0.0f};
     uint32_t grp[8];
-    // dL/dS^dq needs the forward's E2M1 values q
-    uint32_t codes[SFPG ? B / 8 : 1];
-    if constexpr (SFPG) block_codes<DT, B, K>(xw, sq, dead, codes);
+    // dL/dS^dq needs the forward's E2M1 values q, one code word at a time
+    Bracket br[SFPG ? K : 1];
+    if constexpr (SFPG) {
+#pragma unroll
+        for (int k = 0; k < K; ++k) br[k] = make_bracket(sq[k]);
+    }
+    uint32_t cw = 0u;
     const float rs = SFPG ? rcp_approx(sdq) : 0.0f;
     gS = {0.0f, 0.0f};
 #pragma unroll
@@ -394,7 +436,8 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
             if constexpr (SFPG) {
                 // g * q over the sub-block (q: 2 significant bits, so exact
                 // for bf16 g); the q term of dy/dS^dq is not masked
-                const uint32_t cb = (codes[e / 8] >> (4 * (e % 8))) & 0xffu;
+                if (e % 8 == 0) cw = word_codes<DT, B, K>(xw, e / 8, sq, dead, br);
+                const uint32_t cb = (cw >> (4 * (e % 8))) & 0xffu;
                 const uint32_t h2 = e2m1x2_to_f16x2(cb);
                 const float2 q2 = __half22float2(*reinterpret_cast<const __half2*>(&h2));
                 const float2 p = mul2(g2, q2);
@@ -481,7 +524,7 @@ struct Unroll {
 template <int FMT, int SUB, int MODE>
 struct MinCtas {
     static constexpr int value =
-        ((MODE == kBwd) ? (FMT == 1 ? 3 : 2) : (MODE == kBwdS ? 2 : 4)) - (SUB == 2 ? 1 : 0);
+        ((MODE >= kBwd) ? (FMT == 1 ? 3 : 2) : 4) - (SUB == 2 ? 1 : 0);
 };
 
 template <int FMT, int DT, int SUB, int MODE>
