@@ -58,7 +58,7 @@ def lib() -> ctypes.CDLL:
         L.focus_oracle_fwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32,
                                        p, p, p, f, p, p, p, p]
         L.focus_oracle_bwd.argtypes = [i32, i32, i64, i64, i64, i32, i32, i32, i32, i32,
-                                       p, p, p, f, p, p, p, p, p, p, p, p, p, p, p]
+                                       p, p, p, f, p, p, p, p, p, p, p, p, p, p, p, p]
         L.focus_oracle_dequant.argtypes = [i32, i32, i64, i64, i32, p, p, f, p]
         L.focus_oracle_e2m1_code.argtypes = [f]
         L.focus_oracle_e2m1_value.argtypes = [i32]
@@ -200,7 +200,8 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
     term-magnitude sums 'gcrs_abs', 'gdgs_abs', and with want_f64 the
     gradients before their final rounding, 'gcrs64', 'gdgs64' (binary64).
     sfp: optional learnable scales (Eq. 4); want_gsfp adds 'gsfp' float32
-    [rows, cols/block] (and 'gsfp_abs' with want_abs)."""
+    [rows, cols/block] (and 'gsfp_abs' with want_abs, 'gsfp64' with
+    want_f64)."""
     x = np.ascontiguousarray(x)
     g = np.ascontiguousarray(g)
     assert g.dtype == x.dtype and g.shape == x.shape
@@ -217,11 +218,12 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
     gda = np.zeros((crow, cols // sub), np.float64) if (want_abs and want_gdgs) else None
     gc64 = np.zeros((crow, cols // block), np.float64) if want_f64 else None
     gd64 = np.zeros((crow, cols // sub), np.float64) if want_f64 else None
+    gs64 = np.zeros((rows, cols // block), np.float64) if (want_f64 and want_gsfp) else None
     _check(lib().focus_oracle_bwd(fmt, _dtype_code(x), rows, cols, cols, block, sub,
                                   int(bool(shared)), ste, mx_rule, _ptr(x), _ptr(crs),
                                   _ptr(dgs), float(alpha), _ptr(sfp), _ptr(g), _ptr(gx), _ptr(gc),
                                   _ptr(gd), _ptr(gs), _ptr(gca), _ptr(gda), _ptr(gsa), _ptr(gc64),
-                                  _ptr(gd64)))
+                                  _ptr(gd64), _ptr(gs64)))
     out = {}
     if want_gx:
         out["gx"] = gx
@@ -239,6 +241,69 @@ def bwd(x, g, fmt, crs=None, dgs=None, alpha=0.0, block=None, sub=8, shared=Fals
         out["gsfp"] = gs
         if want_abs:
             out["gsfp_abs"] = gsa
+        if want_f64:
+            out["gsfp64"] = gs64
+    return out
+
+
+# --------------------------------------------------------------------------
+# AdamW (the optimizer of the paper's calibration, Sec. 4.1 "Implementation
+# Details": AdamW with a constant learning rate, separate rates for the
+# block scale and the relaxation coefficients; weights frozen, Sec. 4.4)
+# --------------------------------------------------------------------------
+def adamw(p, grad, m, v, lr, beta1, beta2, eps, weight_decay, step):
+    """One AdamW step in binary64: decoupled weight decay (Loshchilov &
+    Hutter), written with PyTorch's conventions (the paper's framework):
+
+        p <- p * (1 - lr * weight_decay)
+        m <- beta1 * m + (1 - beta1) * grad
+        v <- beta2 * v + (1 - beta2) * grad^2
+        p <- p - lr * (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps)
+
+    `step` is t >= 1, the number of this update.  Hyper-parameters are taken
+    as the binary32 values a caller passes to the device.  Returns the new
+    (p, m, v) as float64 arrays; the inputs are not modified."""
+    f = lambda a: float(np.float32(a))
+    lr, beta1, beta2, eps, weight_decay = f(lr), f(beta1), f(beta2), f(eps), f(weight_decay)
+    t = int(step)
+    if t < 1:
+        raise OracleError("AdamW step counts from 1")
+    p = np.asarray(p, np.float64) * (1.0 - lr * weight_decay)
+    g = np.asarray(grad, np.float64)
+    m = beta1 * np.asarray(m, np.float64) + (1.0 - beta1) * g
+    v = beta2 * np.asarray(v, np.float64) + (1.0 - beta2) * g * g
+    mhat = m / (1.0 - beta1 ** t)
+    vhat = v / (1.0 - beta2 ** t)
+    p = p - lr * mhat / (np.sqrt(vhat) + eps)
+    return p, m, v
+
+
+def bwd_adamw(x, g, fmt, params, moments, hp, step, alpha=0.0, sub=8, shared=False,
+              ste=STE_IDENTITY, mx_rule=MX_CEIL, want_gx=True):
+    """The STE backward followed by one AdamW step on every learnable array.
+
+    params: dict with any of 'crs', 'dgs', 'sfp' (float32 arrays; missing =
+    not learned: coefficient 1 / absmax scale).  moments: dict name ->
+    (m, v).  hp: dict lr_coef, lr_scale, beta1, beta2, eps, weight_decay
+    (S^fp takes lr_scale, c_i and c_i^k take lr_coef).  The gradients are the
+    oracle's binary64 sums before rounding.  Returns dict with 'gx' (if
+    wanted), per learned name: 'grad' (float64), 'grad_abs', and the new
+    'p', 'm', 'v' (float64)."""
+    sfp = params.get("sfp")
+    r = bwd(x, g, fmt, crs=params.get("crs"), dgs=params.get("dgs"), alpha=alpha, sub=sub,
+            shared=shared, ste=ste, mx_rule=mx_rule, want_gx=want_gx, want_abs=True,
+            want_f64=True, sfp=sfp, want_gsfp=sfp is not None)
+    out = {"gx": r["gx"]} if want_gx else {}
+    grads = {"crs": ("gcrs64", "gcrs_abs"), "dgs": ("gdgs64", "gdgs_abs"),
+             "sfp": ("gsfp64", "gsfp_abs")}
+    for name, (gk, ak) in grads.items():
+        if params.get(name) is None:
+            continue
+        lr = hp["lr_scale"] if name == "sfp" else hp["lr_coef"]
+        m, v = moments[name]
+        pn, mn, vn = adamw(params[name], r[gk], m, v, lr, hp["beta1"], hp["beta2"], hp["eps"],
+                           hp["weight_decay"], step)
+        out[name] = {"grad": r[gk], "grad_abs": r[ak], "p": pn, "m": mn, "v": vn}
     return out
 
 

@@ -392,20 +392,20 @@ int focus_oracle_fwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
  * MXFP4, alpha * dL/dS^dq_i for NVFP4 (STE through Q_fmt).
  * Optional outputs gcrs_abs / gdgs_abs receive the same sums taken over
  * |mask*g*x| (the scale of the terms, used to bound rounding error), and
- * gcrs64 / gdgs64 the gradients themselves before the final rounding to
- * binary32 (so that partial results can be added exactly).  */
+ * gcrs64 / gdgs64 / gsfp64 the gradients themselves before the final
+ * rounding to binary32 (so that partial results can be added exactly).  */
 int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                      int block, int sub, int shared, int ste, int mx_rule,
                      const void* x, const float* crs, const float* dgs, float alpha,
                      const float* sfp, const void* g, void* gx, float* gcrs, float* gdgs,
                      float* gsfp, double* gcrs_abs, double* gdgs_abs, double* gsfp_abs,
-                     double* gcrs64, double* gdgs64)
+                     double* gcrs64, double* gdgs64, double* gsfp64)
 {
     if (check_shape(rows, cols, ld, block, sub, dtype)) return -1;
     if (fmt != OR_MXFP4 && fmt != OR_NVFP4) return -1;
     if (ste != OR_STE_IDENTITY && ste != OR_STE_CLIPPED) return -1;
     if (rows > 0 && cols > 0 && (!x || !g)) return -1;
-    if ((gsfp || gsfp_abs) && shared) return -1;
+    if ((gsfp || gsfp_abs || gsfp64) && shared) return -1;
     int rc = check_inputs(fmt, dtype, rows, cols, ld, block, sub, shared, x, crs, dgs, alpha, sfp);
     if (rc) return rc;
     for (int64_t r = 0; r < rows; r++)
@@ -498,6 +498,7 @@ int focus_oracle_bwd(int fmt, int dtype, int64_t rows, int64_t cols, int64_t ld,
                 double ds = (fmt == OR_NVFP4) ? (double)alpha : 1.0;
                 if (gsfp) gsfp[r * nblk + j] = (float)(ksum_value(&gs) * ds);
                 if (gsfp_abs) gsfp_abs[r * nblk + j] = ksum_value(&gsa) * ds;
+                if (gsfp64) gsfp64[r * nblk + j] = ksum_value(&gs) * ds;
             }
         }
     }

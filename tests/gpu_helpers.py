@@ -71,3 +71,71 @@ def assert_grad_close(got: np.ndarray, ref: np.ndarray, ref_abs: np.ndarray, flo
 
 def oracle_dtype(a: np.ndarray) -> int:
     return O.BF16 if a.dtype == np.uint16 else O.F32
+
+
+# ---------------------------------------------------------------------------
+# AdamW: the device updates in binary32 from its own binary32 gradient, the
+# oracle in binary64 from the exact gradient.  The bound is interval
+# arithmetic over both: the gradient anywhere within its tolerance, every
+# binary32 operation of the update rounded (u = 2^-24 per operation), the
+# bias corrections 1 - beta^t (device: -expm1(t * log1p(-(1 - beta)))) within
+# 16 u.  A value outside the interval is wrong.
+# ---------------------------------------------------------------------------
+U32 = 2.0 ** -24
+
+
+def adamw_bounds(p, m, v, g, g_abs, floor, lr, beta1, beta2, eps, wd, step):
+    """Intervals (lo, hi) for the device's new p, m, v (float64 arrays)."""
+    f = lambda a: float(np.float32(a))
+    lr, b1, b2, eps, wd = f(lr), f(beta1), f(beta2), f(eps), f(wd)
+    o1, o2 = 1.0 - b1, 1.0 - b2
+    p, m, v = (np.asarray(a, np.float64) for a in (p, m, v))
+    g = np.asarray(g, np.float64)
+    dg = (REL + 2 * U32) * np.abs(g) + floor * np.asarray(g_abs, np.float64) + 2.0 ** -126
+    gl, gh = g - dg, g + dg
+    gmax = np.maximum(np.abs(gl), np.abs(gh))
+    tiny = 2.0 ** -148
+    # first moment
+    rm = 3 * U32 * (b1 * np.abs(m) + o1 * gmax) + tiny
+    ml, mh = b1 * m + o1 * gl - rm, b1 * m + o1 * gh + rm
+    # second moment
+    g2h = gmax * gmax
+    g2l = np.where((gl <= 0) & (gh >= 0), 0.0, np.minimum(gl * gl, gh * gh))
+    rv = 4 * U32 * (b2 * v + o2 * g2h) + tiny
+    vl, vh = b2 * v + o2 * g2l - rv, b2 * v + o2 * g2h + rv
+    # denominator sqrt(v) / sqrt(1 - beta2^t) + eps
+    R = 1.0 / np.sqrt(1.0 - b2 ** step)
+    dl = np.sqrt(np.maximum(vl, 0.0)) * R
+    dh = np.sqrt(np.maximum(vh, 0.0)) * R
+    dl = dl * (1 - 20 * U32) + eps * (1 - U32)
+    dh = dh * (1 + 20 * U32) + eps * (1 + U32)
+    # m / den over the corners (den > 0), plus the division's rounding
+    c = np.stack([ml / dl, ml / dh, mh / dl, mh / dh])
+    ul, uh = c.min(0), c.max(0)
+    umax = np.maximum(np.abs(ul), np.abs(uh))
+    ul, uh = ul - U32 * umax, uh + U32 * umax
+    # p (1 - lr wd) - lr / (1 - beta1^t) * (m / den)
+    S = lr / (1.0 - b1 ** step)
+    pd = p * (1.0 - lr * wd)
+    rp = 3 * U32 * np.abs(pd) + 23 * U32 * S * umax + tiny
+    pl, ph = pd - S * uh - rp, pd - S * ul + rp
+    return (pl, ph), (ml, mh), (vl, vh)
+
+
+def assert_adamw_close(got, p0, m0, v0, ref, floor, lr, hp, step, what):
+    """got: the device's new (p, m, v); p0, m0, v0: the values before the
+    step; ref: the oracle's bwd_adamw entry for this array (its exact
+    gradient 'grad', 'grad_abs', and new 'p')."""
+    (pl, ph), (ml, mh), (vl, vh) = adamw_bounds(
+        p0, m0, v0, ref["grad"], ref["grad_abs"], floor, lr, hp["beta1"], hp["beta2"], hp["eps"],
+        hp["weight_decay"], step)
+    for name, val, lo, hi in (("p", got[0], pl, ph), ("m", got[1], ml, mh), ("v", got[2], vl, vh)):
+        val = np.asarray(val, np.float64).reshape(lo.shape)
+        bad = np.flatnonzero(~((val >= lo) & (val <= hi)))
+        if bad.size:
+            i = bad[0]
+            raise AssertionError(f"{what} {name}: {bad.size} of {val.size} outside the AdamW bound; "
+                                 f"first at {i}: gpu {val.reshape(-1)[i]!r} not in "
+                                 f"[{lo.reshape(-1)[i]!r}, {hi.reshape(-1)[i]!r}]")
+    # the interval contains the oracle's exact step
+    assert np.all((ref["p"] >= pl) & (ref["p"] <= ph)), f"{what}: oracle p outside its bound"

@@ -608,8 +608,10 @@ def torch_fake_quant_sfp(x, sfp, crs, dgs, fmt, alpha, block, sub):
         s = sfp + (torch.from_numpy(q) - sfp).detach()
     else:
         # the forward's scale is fl(alpha * Delta) in binary32; the STE carries
-        # d S^dq / d Delta^fp = alpha
-        dq = torch.from_numpy(torch_e4m3(sf)).view(torch.float8_e4m3fn).float()
+        # d S^dq / d Delta^fp = alpha; Q_E4M3 saturates at 448 (torch's cast
+        # gives NaN above it)
+        dq = torch.from_numpy(torch_e4m3(np.minimum(sf, np.float32(448)))).view(
+            torch.float8_e4m3fn).float()
         sdq = (dq * torch.tensor(alpha, dtype=torch.float32)).double()
         s = sdq + alpha * (sfp - sfp.detach())
     s = s.repeat_interleave(block, dim=1)
@@ -639,3 +641,95 @@ def test_sfp_gradient_autograd(fmt):
     # the forward of the restatement is the oracle's (values, through fp64)
     fw = O.fwd(x, fmt, crs=crs, dgs=dgs, alpha=a, sfp=sfp)
     np.testing.assert_allclose(y.detach().numpy(), fw["y"].astype(np.float64), rtol=1e-6, atol=0)
+
+
+# ---------------------------------------------------------------------------
+# AdamW on the learnable arrays (Sec. 4.1: AdamW, constant learning rate)
+# ---------------------------------------------------------------------------
+HP = dict(lr_coef=5e-2, lr_scale=2e-2, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+
+
+def fp32(v):
+    return float(np.float32(v))
+
+
+def test_adamw_matches_torch():
+    """Five AdamW steps of the oracle equal torch.optim.AdamW in float64 (the
+    library routine the paper's PyTorch setup calls)."""
+    rng = np.random.default_rng(91)
+    p0 = rng.uniform(0.5, 1.5, 64)
+    m = np.zeros(64)
+    v = np.zeros(64)
+    lr, b1, b2, eps, wd = fp32(3e-2), fp32(0.9), fp32(0.999), fp32(1e-8), fp32(0.01)
+    pt = torch.tensor(p0, dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.AdamW([pt], lr=lr, betas=(b1, b2), eps=eps, weight_decay=wd)
+    p = p0.copy()
+    for t in range(1, 6):
+        g = rng.standard_normal(64) * 10.0 ** rng.uniform(-6, 1, 64)
+        pt.grad = torch.tensor(g)
+        opt.step()
+        p, m, v = O.adamw(p, g, m, v, lr, b1, b2, eps, wd, t)
+        np.testing.assert_allclose(p, pt.detach().numpy(), rtol=1e-14, atol=0)
+        np.testing.assert_allclose(m, opt.state[pt]["exp_avg"].numpy(), rtol=1e-14, atol=0)
+        np.testing.assert_allclose(v, opt.state[pt]["exp_avg_sq"].numpy(), rtol=1e-14, atol=0)
+
+
+def test_adamw_first_step_closed_form():
+    """From zero moments the first step is p (1 - lr wd) - lr g / (|g| + eps)."""
+    g = np.array([3.0, -2e-3, 0.0, 1e-9, -7.5])
+    p = np.array([1.0, 0.9, 1.1, 2.0, 0.5])
+    lr, wd, eps = fp32(5e-3), fp32(0.01), fp32(1e-8)
+    pn, mn, vn = O.adamw(p, g, np.zeros(5), np.zeros(5), lr, 0.9, 0.999, eps, wd, 1)
+    np.testing.assert_allclose(pn, p * (1 - lr * wd) - lr * g / (np.abs(g) + eps), rtol=1e-13, atol=0)
+    np.testing.assert_allclose(mn, (1 - fp32(0.9)) * g, rtol=1e-15, atol=0)
+    np.testing.assert_allclose(vn, (1 - fp32(0.999)) * g * g, rtol=1e-15, atol=0)
+    with pytest.raises(O.OracleError):
+        O.adamw(p, g, mn, vn, lr, 0.9, 0.999, eps, wd, 0)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_bwd_adamw_equals_autograd_and_torch_adamw(fmt):
+    """The fused backward + AdamW of the oracle equals autograd of the STE
+    restatement followed by torch.optim.AdamW on S^fp (lr_scale) and c_i,
+    c_i^k (lr_coef), from moments of an earlier step."""
+    rng = np.random.default_rng(93)
+    block = 32 if fmt == O.MXFP4 else 16
+    rows, cols = 4, 4 * block
+    x = (rng.standard_normal((rows, cols)) * 0.02).astype(np.float32)
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    crs = rng.uniform(0.8, 1.2, (rows, cols // block)).astype(np.float32)
+    dgs = rng.uniform(0.8, 1.2, (rows, cols // 8)).astype(np.float32)
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    sfp = (absmax_sfp(x, fmt, a) * rng.uniform(0.7, 1.3, (rows, cols // block))).astype(np.float32)
+    params = {"crs": crs, "dgs": dgs, "sfp": sfp}
+    moments = {k: (rng.standard_normal(v.shape).astype(np.float32) * np.float32(0.1),
+                   rng.uniform(0.01, 1.0, v.shape).astype(np.float32)) for k, v in params.items()}
+    step = 7
+    ours = O.bwd_adamw(x, g, fmt, params, moments, HP, step, alpha=a)
+    t = {k: torch.from_numpy(v.astype(np.float64)).requires_grad_(True) for k, v in params.items()}
+    y = torch_fake_quant_sfp(torch.from_numpy(x.astype(np.float64)), t["sfp"], t["crs"], t["dgs"],
+                             fmt, float(a), block, 8)
+    y.backward(torch.from_numpy(g.astype(np.float64)))
+    opt = torch.optim.AdamW(
+        [{"params": [t["sfp"]], "lr": fp32(HP["lr_scale"])},
+         {"params": [t["crs"], t["dgs"]], "lr": fp32(HP["lr_coef"])}],
+        betas=(fp32(HP["beta1"]), fp32(HP["beta2"])), eps=fp32(HP["eps"]),
+        weight_decay=fp32(HP["weight_decay"]))
+    for k, (m, v) in moments.items():
+        opt.state[t[k]] = {"step": torch.tensor(float(step - 1)),
+                           "exp_avg": torch.from_numpy(m.astype(np.float64)),
+                           "exp_avg_sq": torch.from_numpy(v.astype(np.float64))}
+    grads = {k: t[k].grad.numpy().copy() for k in t}
+    opt.step()
+    for k in params:
+        np.testing.assert_allclose(ours[k]["grad"], grads[k], rtol=1e-5, atol=1e-12)
+        lr = fp32(HP["lr_scale"] if k == "sfp" else HP["lr_coef"])
+        # gradients agree to ~1e-7 relative; the step moves by about lr
+        np.testing.assert_allclose(ours[k]["p"], t[k].detach().numpy(), rtol=0, atol=1e-5 * lr)
+        np.testing.assert_allclose(ours[k]["m"], opt.state[t[k]]["exp_avg"].numpy(), rtol=1e-5,
+                                   atol=1e-12)
+        np.testing.assert_allclose(ours[k]["v"], opt.state[t[k]]["exp_avg_sq"].numpy(), rtol=1e-5,
+                                   atol=0)
+    # arrays that are not learned are not in the result
+    part = O.bwd_adamw(x, g, fmt, {"dgs": dgs}, {"dgs": moments["dgs"]}, HP, step, alpha=a)
+    assert set(part) == {"gx", "dgs"}
