@@ -48,6 +48,7 @@ class Case:
     sub: int = 8
     shared: bool = False       # one coefficient set for all rows (activations)
     sfp: bool = False          # learnable full-precision scales S^fp (Eq. 4) and dL/dS^fp
+    adam: bool = False         # backward fused with the AdamW step on c, c^k (and S^fp)
 
     @property
     def block(self) -> int:
@@ -64,7 +65,9 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
     scale byte per block."""
     coef = 0.0 if case.shared else 4.0 / case.block + 4.0 / case.sub
     sfp = 4.0 / case.block if case.sfp else 0.0     # S^fp in (and dL/dS^fp out)
-    out = {"fwd": 2 * esz + coef + sfp, "bwd": 3 * esz + 2 * coef + 2 * sfp,
+    # fused AdamW: per learned value p, m, v in and p, m, v out; no gradient
+    bwd_params = 6 * (coef + sfp) if case.adam else 2 * (coef + sfp)
+    out = {"fwd": 2 * esz + coef + sfp, "bwd": 3 * esz + bwd_params,
            "pack": esz + coef + sfp + 0.5 + 1.0 / case.block}
     if case.fmt == "nvfp4":
         out["alpha"] = float(esz)
@@ -76,14 +79,28 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
 # dram__bytes_read, dram__bytes_write; --cache-control none), and the sha256
 # prefix of the kernel sources it was taken on.  Reported only for the
 # default case and while the sources are unchanged.
-BWD_TRAFFIC = {"sources": "362a9af01b1cdea8", "bytes_per_step": 745.7e6}
+BWD_TRAFFIC = {"sources": "ef542681ea9e268d", "bytes_per_step": 746.5e6}
+
+# AdamW hyper-parameters of the fused optimizer: the paper's learning rates
+# per format (Sec. 4.1: block scale / relaxation coefficients) and PyTorch's
+# AdamW defaults, which the paper does not override.  S^fp is learned in the
+# linear domain, where an MXFP4 block scale of these weights is about 2^-7;
+# Adam's first steps move a parameter by about the learning rate, so the
+# MXFP4 scale rate 2e-2 is applied relative to that magnitude.
+ADAMW_HP = {"mxfp4": dict(lr_coef=5e-2, lr_scale=2e-2 * 2.0 ** -7, beta1=0.9, beta2=0.999,
+                          eps=1e-8, weight_decay=0.01),
+            "nvfp4": dict(lr_coef=1e-3, lr_scale=5e-3, beta1=0.9, beta2=0.999, eps=1e-8,
+                          weight_decay=0.01)}
+
+
+# the sources the default backward kernel is compiled from
+BWD_SOURCES = ("fq_device.cuh", "fq_kernels.cuh", "fq_launch.h", "fq_inst_bwd_nv.cu")
 
 
 def kernel_sources_sha() -> str:
-    import glob
     import hashlib
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2608_01847_gb300", "csrc", "*"))):
+    for f in sorted(os.path.join(ROOT, "paper_2608_01847_gb300", "csrc", n) for n in BWD_SOURCES):
         h.update(os.path.basename(f).encode())
         with open(f, "rb") as fh:
             h.update(fh.read())
@@ -174,7 +191,7 @@ def aggregate_gbs(bytes_per_rank_step: float, world: int, max_ms_per_step: float
 class Tensor:
     """Device tensors of one projection (or activation) plus its outputs."""
 
-    def __init__(self, case: Case, w, idx, device):
+    def __init__(self, case: Case, w, idx, device, step=None):
         import torch
         from paper_2608_01847_gb300 import focus as F
         from paper_2608_01847_gb300 import workloads as W
@@ -210,10 +227,29 @@ class Tensor:
             jit = torch.rand(m.shape, generator=gen, device=device) * 0.2 + 0.9
             self.sfp = (m / den * jit).contiguous()
             self.gsfp = torch.empty_like(self.sfp)
+        if case.adam:
+            # optimizer state resident in HBM; the paper's learning rates
+            # (Sec. 4.1); two synthetic batches alternate, the second's
+            # output gradient the negation of the first's, so that a fixed
+            # gradient does not drive the parameters out of range over
+            # thousands of steps
+            self.step = step
+            self.g_alt = -self.g
+            learned = {"crs": self.crs, "dgs": self.dgs}
+            if self.sfp is not None:
+                learned["sfp"] = self.sfp
+            self.moments = {k: (torch.zeros_like(v), torch.zeros_like(v)) for k, v in learned.items()}
+            self.hp = ADAMW_HP[case.fmt]
 
-    def run(self, phase):
+    def run(self, phase, parity=0):
         from paper_2608_01847_gb300 import focus as F
         c = self.case
+        if phase == "bwd" and c.adam:
+            F.focus_fq_bwd_adamw(self.x, self.g_alt if parity else self.g, self.fmt, self.step,
+                                 self.hp, crs=self.crs, dgs=self.dgs, sfp=self.sfp,
+                                 moments=self.moments, alpha=self.alpha, sub_block=c.sub,
+                                 shared=c.shared, gx=self.gx, ws=self.ws_bwd)
+            return
         if phase == "alpha":
             F.focus_nvfp4_alpha(self.x, self.alpha, self.ws_alpha)
         elif phase == "fwd":
@@ -227,12 +263,17 @@ class Tensor:
             F.focus_pack(self.x, self.fmt, self.crs, self.dgs, self.alpha, sub_block=c.sub,
                          shared=c.shared, codes=self.codes, scale_bytes=self.scales, sfp=self.sfp)
 
-    def inputs(self):
-        """Device tensors a step reads from the host (end-to-end leg)."""
+    def inputs(self, parity=0):
+        """Device tensors a step reads from the host (end-to-end leg).  With
+        the fused optimizer the parameters and moments stay in HBM."""
+        if self.case.adam:
+            return (self.x, self.g_alt if parity else self.g)
         return (self.x, self.g, self.crs, self.dgs) + ((self.sfp,) if self.sfp is not None else ())
 
     def outputs(self):
         """Device tensors a step returns to the host (end-to-end leg)."""
+        if self.case.adam:
+            return (self.y, self.gx, self.codes, self.scales)
         out = (self.y, self.gx, self.gcrs, self.gdgs, self.codes, self.scales)
         return out + ((self.gsfp,) if self.gsfp is not None else ())
 
@@ -245,7 +286,7 @@ class BranchGraph:
     branches (one stream each) run `body(i, stage)` for every tensor i
     independently and join before the next stage."""
 
-    def __init__(self, n, body, device, stages=(None,)):
+    def __init__(self, n, body, device, stages=(None,), before=None):
         import torch
         self.graph = torch.cuda.CUDAGraph()
         side = [torch.cuda.Stream(device) for _ in range(n)]
@@ -254,6 +295,8 @@ class BranchGraph:
         with torch.cuda.graph(self.graph, stream=cap):
             main = torch.cuda.current_stream(device)
             for stage in stages:
+                if before is not None:
+                    before(stage)
                 for i, st in enumerate(side):
                     st.wait_stream(main)
                     with torch.cuda.stream(st):
@@ -270,7 +313,7 @@ class PipelineGraph:
     """End-to-end step as a graph of three chained streams: H2D copies of
     each tensor's inputs, then its phases, then D2H copies of its outputs."""
 
-    def __init__(self, ts, host_in, host_out, phases, device):
+    def __init__(self, ts, host_in, host_out, phases, device, parity=0, before=None):
         import torch
         # the smallest tensor first (short pipeline fill: its H2D runs alone)
         # and the second smallest last (short drain: its D2H runs alone)
@@ -285,16 +328,18 @@ class PipelineGraph:
         cap.wait_stream(torch.cuda.current_stream(device))
         with torch.cuda.graph(self.graph, stream=cap):
             main = torch.cuda.current_stream(device)
+            if before is not None:
+                before()
             for st in (s_in, s_cmp, s_out):
                 st.wait_stream(main)
             for t, hin, hout in zip(ts, host_in, host_out):
                 with torch.cuda.stream(s_in):
-                    for d, h in zip(t.inputs(), hin):
+                    for d, h in zip(t.inputs(parity), hin):
                         d.copy_(h, non_blocking=True)
                 s_cmp.wait_stream(s_in)
                 with torch.cuda.stream(s_cmp):
                     for ph in phases:
-                        t.run(ph)
+                        t.run(ph, parity)
                 s_out.wait_stream(s_cmp)
                 with torch.cuda.stream(s_out):
                     for h, d in zip(hout, t.outputs()):
@@ -316,24 +361,39 @@ def gpu_arm(case, args, rank, world, device):
     F.lib()
     w = W.WORKLOADS[case.workload] if case.workload in W.WORKLOADS else W.sweep_workload(
         int(case.workload.split("_")[-1]))
-    ts = [Tensor(case, w, i, device) for i in range(len(w.tensors))]
+    # the fused optimizer's step counter t, advanced on the device before
+    # every backward phase (inside the captured graphs)
+    step_t = torch.zeros(1, dtype=torch.int64, device=device) if case.adam else None
+    ts = [Tensor(case, w, i, device, step_t) for i in range(len(w.tensors))]
     n_elem = sum(t.n for t in ts)
     esz = ts[0].x.element_size()
     stream = torch.cuda.current_stream(device)
     phases = case.phases()
     torch.cuda.synchronize(device)
 
+    def before(stage):
+        if step_t is not None and stage == "bwd":
+            step_t.add_(1)
+
     # eager warm-up (resolves launch configurations), then capture each phase
     for ph in phases:
+        before(ph)
         for t in ts:
             t.run(ph)
     torch.cuda.synchronize(device)
-    # one graph per phase (for the phase split) and one for the whole step
-    graphs = [(ph, BranchGraph(len(ts), lambda i, ph=ph: ts[i].run(ph), device)) for ph in phases]
-    step_graph = BranchGraph(len(ts), lambda i, ph: ts[i].run(ph), device, stages=phases)
+    # one graph per phase (for the phase split) and one for the whole step;
+    # with the optimizer, one of each per batch parity (alternating batches)
+    parities = (0, 1) if case.adam else (0,)
+    graphs = {ph: [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
+                               stages=(ph,), before=before) for par in parities]
+              for ph in phases}
+    step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
+                               stages=phases, before=before) for par in parities]
+    n_replay = [0]
 
     def step():
-        step_graph.replay()
+        step_graphs[n_replay[0] % len(parities)].replay()
+        n_replay[0] += 1
 
     for _ in range(args.warmup):
         step()
@@ -357,11 +417,11 @@ def gpu_arm(case, args, rank, world, device):
     # phase split: each phase graph replayed on its own, timed the same way
     phase_ms = {}
     n_split = max(1, min(args.steps, 100))
-    for name, gph in graphs:
+    for name, gph in graphs.items():
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for _ in range(n_split):
-            gph.replay()
+        for k in range(n_split):
+            gph[k % len(parities)].replay()
         b.record(stream)
         torch.cuda.synchronize(device)
         phase_ms[name] = a.elapsed_time(b) * args.steps / n_split
@@ -377,18 +437,24 @@ def gpu_arm(case, args, rank, world, device):
     # (tensor after tensor), a compute chain (tensor k's phases once its
     # inputs are in HBM) and a D2H chain (tensor k's outputs once computed),
     # so that tensor k's D2H overlaps tensor k+1's H2D on the full-duplex link.
-    host_in = [[a.cpu().pin_memory() for a in t.inputs()] for t in ts]
     host_out = [[torch.empty_like(a, device="cpu").pin_memory() for a in t.outputs()] for t in ts]
+    e2e_graphs = []
+    for par in parities:
+        host_in = [[a.cpu().pin_memory() for a in t.inputs(par)] for t in ts]
+        e2e_graphs.append(PipelineGraph(ts, host_in, host_out, phases, device, par,
+                                        before=lambda: before("bwd")))
     h2d = sum(a.numel() * a.element_size() for h in host_in for a in h)
     d2h = sum(a.numel() * a.element_size() for h in host_out for a in h)
-    e2e_graph = PipelineGraph(ts, host_in, host_out, phases, device)
     e2e_steps = max(3, min(args.steps, 20))
-    e2e_graph.replay()
+    e2e_steps += e2e_steps % len(parities)
+    e2e_graphs[0].replay()
+    if len(parities) > 1:
+        e2e_graphs[1].replay()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(e2e_steps):
-        e2e_graph.replay()
+    for k in range(e2e_steps):
+        e2e_graphs[k % len(parities)].replay()
     e1.record(stream)
     barrier()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
@@ -402,13 +468,21 @@ def gpu_arm(case, args, rank, world, device):
 # ----------------------------------------------------------------------------
 def oracle_step(case, samples):
     """One pass of the oracle's alpha, fwd, bwd, pack over host samples."""
+    import numpy as np
     import oracle as O
     fmt = O.NVFP4 if case.fmt == "nvfp4" else O.MXFP4
     for x, g, crs, dgs, sfp in samples:
         a = O.alpha(x) if fmt == O.NVFP4 else 0.0
         kw = dict(crs=crs, dgs=dgs, alpha=a, sub=case.sub, shared=case.shared, sfp=sfp)
         O.fwd(x, fmt, want_scales=False, **kw)
-        O.bwd(x, g, fmt, want_gsfp=sfp is not None, **kw)
+        if case.adam:
+            params = {k: v for k, v in (("crs", crs), ("dgs", dgs), ("sfp", sfp)) if v is not None}
+            moments = {k: (np.zeros(v.shape, np.float32), np.zeros(v.shape, np.float32))
+                       for k, v in params.items()}
+            O.bwd_adamw(x, g, fmt, params, moments, ADAMW_HP[case.fmt], 1, alpha=a, sub=case.sub,
+                        shared=case.shared)
+        else:
+            O.bwd(x, g, fmt, want_gsfp=sfp is not None, **kw)
         O.fwd(x, fmt, want_y=False, want_codes=True, **kw)
 
 
@@ -487,6 +561,7 @@ def reference_arm(case, args):
             "data": "synthetic",
             "config": {"workload": case.workload, "fmt": case.fmt, "sub_block": case.sub,
                        "shared_coefficients": case.shared, "learnable_sfp": case.sfp,
+                       "fused_adamw": case.adam,
                        "sample_rows_per_tensor": rows,
                        "elements_per_step": n},
             "cpu_baseline": {"value": round(value, 6), "unit": "GB/s", "cores": 1, "kind": "oracle",
@@ -509,10 +584,12 @@ def main():
     ap.add_argument("--shared", action="store_true", help="coefficients shared by all rows")
     ap.add_argument("--sfp", action="store_true",
                     help="learnable full-precision scales S^fp and their gradient")
+    ap.add_argument("--adam", action="store_true",
+                    help="backward fused with the AdamW step on the learned arrays")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
-    case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp)
+    case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp, args.adam)
     default_case = case == Case()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -569,7 +646,9 @@ def main():
                    "coefficients": ("shared by all rows" if case.shared else
                                     "per-block CRS + per-sub-block DGS"),
                    "scales": "learnable S^fp (+ dL/dS^fp)" if case.sfp else "absmax",
-                   "step": "+".join(case.phases()) + " over all tensors (bwd: gx + gcrs + gdgs)",
+                   "step": "+".join(case.phases()) + " over all tensors " +
+                           ("(bwd: gx + AdamW on the learned arrays)" if case.adam else
+                            "(bwd: gx + gcrs + gdgs)"),
                    "bytes_per_elem": round(sum(bpe.values()), 4),
                    "l2": f"inputs larger than L2: x+g = {r['n_elem'] * 2 * r['esz'] / 2**20:.0f} MiB"
                          " per step",

@@ -156,8 +156,9 @@ int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float* crs,
 /* Straight-through-estimator backward (Sec. 3.2) of focus_fq_fwd.
  * x, crs, dgs, alpha, sfp  as for focus_fq_fwd.
  * g      [rows, ld] upstream gradient dL/dy (dtype).
- * gx     optional [rows, ld] output dL/dx = mask * fl(fl(g * S^dq) / S^q);
- *        NULL skips it (frozen weights, Sec. 3.2).
+ * gx     optional [rows, ld] output dL/dx = mask * fl(g * fl(S^dq / S^q)), the
+ *        scale ratio rounded once per sub-block; NULL skips it (frozen
+ *        weights, Sec. 3.2).
  * gcrs   optional dL/dc_i    = -sum_k T_ik * c_i^k / (c_i c_i^k)^2
  * gdgs   optional dL/dc_i^k  = -T_ik * c_i / (c_i c_i^k)^2
  *        with T_ik = sum over sub-block (i,k) of mask * g * x; in shared mode
@@ -178,6 +179,59 @@ int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,
                  void* gx, float* gcrs, float* gdgs, float* gsfp, void* ws, size_t ws_bytes,
                  focus_stream_t stream);
 
+/* AdamW hyper-parameters (host memory, read during the call).  The paper
+ * trains with AdamW at a constant learning rate, one rate for the block
+ * scale S^fp and one for the relaxation coefficients (Sec. 4.1: MXFP4
+ * 2e-2 / 5e-2, NVFP4 5e-3 / 1e-3).  Requirements: learning rates and
+ * weight_decay finite and >= 0, 0 <= beta1, beta2 < 1, eps finite and > 0;
+ * otherwise FOCUS_ERR_INVALID_ARG. */
+typedef struct {
+    float lr_coef;        /* learning rate of c_i and c_i^k */
+    float lr_scale;       /* learning rate of S^fp */
+    float beta1;          /* first-moment decay (PyTorch default 0.9) */
+    float beta2;          /* second-moment decay (PyTorch default 0.999) */
+    float eps;            /* denominator guard (PyTorch default 1e-8) */
+    float weight_decay;   /* decoupled decay lambda (PyTorch AdamW default 0.01) */
+} focus_adamw_t;
+
+/* Optimizer state: fp32 moment arrays shaped and laid out exactly like the
+ * parameter they belong to (16-byte aligned, caller-owned device memory,
+ * zero before the first step).  Pairs of a parameter that is not learned
+ * (NULL in focus_fq_bwd_adamw) are ignored. */
+typedef struct {
+    float* m_crs;
+    float* v_crs;
+    float* m_dgs;
+    float* v_dgs;
+    float* m_sfp;
+    float* v_sfp;
+} focus_adamw_state_t;
+
+/* STE backward fused with one AdamW step on the learnable arrays (Sec. 3.2
+ * and Sec. 4.1).  Computes exactly what focus_fq_bwd computes, at the
+ * parameter values on entry, then, for each of crs, dgs and sfp that is
+ * non-NULL (the arrays being learned), replaces it in place by
+ *   p <- p * (1 - lr * weight_decay)
+ *   m <- beta1 * m + (1 - beta1) * grad,  v <- beta2 * v + (1 - beta2) * grad^2
+ *   p <- p - lr / (1 - beta1^t) * m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
+ * (PyTorch's AdamW) with lr = hp->lr_scale for sfp and hp->lr_coef for the
+ * coefficients, in binary32, and writes the new moments.  The gradients are
+ * not written to memory unless gcrs / gdgs / gsfp are given.
+ * crs, dgs, sfp  parameters as for focus_fq_bwd, updated in place; NULL: not
+ *        learned (coefficient 1 / absmax scale).  sfp only with per-row
+ *        coefficients.
+ * step   device pointer to an int64 t >= 1, the number of this update (the
+ *        caller advances it before each step; the library only reads it, so
+ *        a captured CUDA graph that advances it replays correctly).
+ * With coef_shared_rows = 1 the step is applied once the gradient summed
+ * over all rows is complete (an empty row set gives gradient 0, and the
+ * step still applies).  Other arguments as for focus_fq_bwd. */
+int focus_fq_bwd_adamw(const focus_desc_t* desc, const void* x, float* crs, float* dgs,
+                       const float* alpha, float* sfp, const void* g, void* gx,
+                       const focus_adamw_t* hp, const focus_adamw_state_t* state,
+                       const int64_t* step, float* gcrs, float* gdgs, float* gsfp, void* ws,
+                       size_t ws_bytes, focus_stream_t stream);
+
 /* Export (Fig. 3(d)): the FP4 codes of Q_E2M1(x / S^q) and the scale bytes
  * of S^dq -- what the deployed MXFP4 / NVFP4 model stores; S^q and the
  * coefficients are not part of it.  NVFP4 also needs the caller's alpha.
@@ -196,7 +250,7 @@ size_t focus_workspace_bytes(const focus_desc_t* desc, int which);
 /* Static, NUL-terminated description of a status code. */
 const char* focus_status_string(int status);
 
-/* ABI version of this library (major * 100 + minor): 200. */
+/* ABI version of this library (major * 100 + minor): 210. */
 int focus_version(void);
 
 #ifdef __cplusplus

@@ -97,6 +97,144 @@ int check_coef_ptrs(const float* a, const float* b, const float* c, const float*
     return FOCUS_OK;
 }
 
+size_t bwd_ws_bytes(const focus_desc_t* d);
+
+// Column finalisation of the shared-row backward alone (no rows to reduce).
+cudaError_t launch_shared_finalize(int fmt, int sub, const KParams& p, cudaStream_t st)
+{
+    if (fmt == 0) {
+        switch (sub) {
+        case 2: return run_shared_finalize<0, 2>(p, 0, st);
+        case 4: return run_shared_finalize<0, 4>(p, 0, st);
+        case 8: return run_shared_finalize<0, 8>(p, 0, st);
+        case 16: return run_shared_finalize<0, 16>(p, 0, st);
+        case 32: return run_shared_finalize<0, 32>(p, 0, st);
+        default: break;
+        }
+    } else {
+        switch (sub) {
+        case 2: return run_shared_finalize<1, 2>(p, 0, st);
+        case 4: return run_shared_finalize<1, 4>(p, 0, st);
+        case 8: return run_shared_finalize<1, 8>(p, 0, st);
+        case 16: return run_shared_finalize<1, 16>(p, 0, st);
+        default: break;
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+// The fused optimizer's arguments (null `hp` for the plain backward).
+struct OptArgs {
+    float* crs;
+    float* dgs;
+    float* sfp;
+    const focus_adamw_t* hp;
+    const focus_adamw_state_t* state;
+    const int64_t* step;
+};
+
+bool finite_ge0(float v) { return v >= 0.0f && v <= 3.4028234663852886e38f; }
+
+int check_opt(const OptArgs& o)
+{
+    if (!o.hp || !o.state || !o.step) return FOCUS_ERR_INVALID_ARG;
+    const focus_adamw_t& h = *o.hp;
+    if (!finite_ge0(h.lr_coef) || !finite_ge0(h.lr_scale) || !finite_ge0(h.weight_decay))
+        return FOCUS_ERR_INVALID_ARG;
+    if (!(h.beta1 >= 0.0f && h.beta1 < 1.0f) || !(h.beta2 >= 0.0f && h.beta2 < 1.0f))
+        return FOCUS_ERR_INVALID_ARG;
+    if (!(finite_ge0(h.eps) && h.eps > 0.0f)) return FOCUS_ERR_INVALID_ARG;
+    const focus_adamw_state_t& s = *o.state;
+    if ((o.crs && (!s.m_crs || !s.v_crs)) || (o.dgs && (!s.m_dgs || !s.v_dgs)) ||
+        (o.sfp && (!s.m_sfp || !s.v_sfp)))
+        return FOCUS_ERR_INVALID_ARG;
+    if (misaligned(o.step, 8)) return FOCUS_ERR_MISALIGNED;
+    if (o.crs && (misaligned(s.m_crs, 16) || misaligned(s.v_crs, 16))) return FOCUS_ERR_MISALIGNED;
+    if (o.dgs && (misaligned(s.m_dgs, 16) || misaligned(s.v_dgs, 16))) return FOCUS_ERR_MISALIGNED;
+    if (o.sfp && (misaligned(s.m_sfp, 16) || misaligned(s.v_sfp, 16))) return FOCUS_ERR_MISALIGNED;
+    return FOCUS_OK;
+}
+
+void set_opt(KParams& p, const OptArgs& o)
+{
+    const focus_adamw_t& h = *o.hp;
+    p.new_crs = o.crs;
+    p.new_dgs = o.dgs;
+    p.new_sfp = o.sfp;
+    p.opt_m[0] = o.crs ? o.state->m_crs : nullptr;
+    p.opt_v[0] = o.crs ? o.state->v_crs : nullptr;
+    p.opt_m[1] = o.dgs ? o.state->m_dgs : nullptr;
+    p.opt_v[1] = o.dgs ? o.state->v_dgs : nullptr;
+    p.opt_m[2] = o.sfp ? o.state->m_sfp : nullptr;
+    p.opt_v[2] = o.sfp ? o.state->v_sfp : nullptr;
+    p.step = reinterpret_cast<const long long*>(o.step);
+    p.lr_c = h.lr_coef;
+    p.lr_s = h.lr_scale;
+    p.beta1 = h.beta1;
+    p.beta2 = h.beta2;
+    p.eps = h.eps;
+    p.decay_c = static_cast<float>(1.0 - static_cast<double>(h.lr_coef) * h.weight_decay);
+    p.decay_s = static_cast<float>(1.0 - static_cast<double>(h.lr_scale) * h.weight_decay);
+}
+
+// The backward with or without the fused optimizer step.
+int run_bwd(const focus_desc_t* desc, const void* x, const float* crs, const float* dgs,
+            const float* alpha, const float* sfp, const void* g, void* gx, float* gcrs,
+            float* gdgs, float* gsfp, void* ws, size_t ws_bytes, cudaStream_t st,
+            const OptArgs* opt)
+{
+    int rc = check_desc(desc, true);
+    if (rc) return rc;
+    if ((sfp || gsfp) && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
+    if (opt && (rc = check_opt(*opt))) return rc;
+    const bool learn = opt && (opt->crs || opt->dgs || opt->sfp);
+    const bool want_T = gcrs != nullptr || gdgs != nullptr || (learn && (crs || dgs));
+    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4) ||
+        misaligned(sfp, 4) || misaligned(gsfp, 4))
+        return FOCUS_ERR_MISALIGNED;
+    if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
+    KParams p = make_params(desc);
+    p.x = x;
+    p.g = g;
+    p.gx = gx;
+    p.crs = crs;
+    p.dgs = dgs;
+    p.alpha = alpha;
+    p.sfp = sfp;
+    p.gcrs = gcrs;
+    p.gdgs = gdgs;
+    p.gsfp = gsfp;
+    if (learn) set_opt(p, *opt);
+    const int sub = effective_sub(desc, dgs, gdgs);
+    if (desc->rows == 0 || desc->cols == 0) {
+        // shared-row gradients of an empty row set are sums over nothing: zero
+        if (desc->coef_shared_rows && desc->cols > 0) {
+            if (learn) {
+                p.nsub = static_cast<uint32_t>(desc->cols / sub);
+                return map_cuda(launch_shared_finalize(desc->fmt, sub, p, st));
+            }
+            cudaError_t e = cudaSuccess;
+            if (gcrs) e = cudaMemsetAsync(gcrs, 0, sizeof(float) * (desc->cols / desc->block), st);
+            if (e == cudaSuccess && gdgs)
+                e = cudaMemsetAsync(gdgs, 0, sizeof(float) * (desc->cols / desc->sub_block), st);
+            return map_cuda(e);
+        }
+        return FOCUS_OK;
+    }
+    if (!x || !g || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
+    if (!gx && !want_T && !gsfp && !learn) return FOCUS_OK;
+    if (desc->coef_shared_rows && want_T) {
+        const size_t need = bwd_ws_bytes(desc);
+        if (!ws || ws_bytes < need) return FOCUS_ERR_WORKSPACE;
+        if (misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
+        p.ws = static_cast<float*>(ws);
+        p.nsub = static_cast<uint32_t>(desc->cols / sub);
+        const uint32_t ny = shared_row_groups(p.rows, p.bpr);
+        return map_cuda(launch_bwd_shared(desc->fmt, desc->dtype, sub, p, ny, st));
+    }
+    return map_cuda(launch_bwd(desc->fmt, desc->dtype, sub, p, st));
+}
+
 size_t bwd_ws_bytes(const focus_desc_t* d)
 {
     if (!d->coef_shared_rows || d->rows == 0 || d->cols == 0) return 0;
@@ -110,7 +248,7 @@ size_t bwd_ws_bytes(const focus_desc_t* d)
 
 using namespace focus;
 
-FOCUS_API int focus_version(void) { return 200; }
+FOCUS_API int focus_version(void) { return 210; }
 
 FOCUS_API const char* focus_status_string(int status)
 {
@@ -209,48 +347,17 @@ FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float*
                            void* gx, float* gcrs, float* gdgs, float* gsfp, void* ws,
                            size_t ws_bytes, focus_stream_t stream)
 {
-    int rc = check_desc(desc, true);
-    if (rc) return rc;
-    if ((sfp || gsfp) && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
-    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    const bool want_T = gcrs != nullptr || gdgs != nullptr;
-    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4) ||
-        misaligned(sfp, 4) || misaligned(gsfp, 4))
-        return FOCUS_ERR_MISALIGNED;
-    if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
-    if (desc->rows == 0 || desc->cols == 0) {
-        // shared-row gradients of an empty row set are sums over nothing: zero
-        if (desc->coef_shared_rows && desc->cols > 0) {
-            cudaError_t e = cudaSuccess;
-            if (gcrs) e = cudaMemsetAsync(gcrs, 0, sizeof(float) * (desc->cols / desc->block), st);
-            if (e == cudaSuccess && gdgs)
-                e = cudaMemsetAsync(gdgs, 0, sizeof(float) * (desc->cols / desc->sub_block), st);
-            return map_cuda(e);
-        }
-        return FOCUS_OK;
-    }
-    if (!x || !g || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
-    if (!gx && !want_T && !gsfp) return FOCUS_OK;
-    KParams p = make_params(desc);
-    p.x = x;
-    p.g = g;
-    p.gx = gx;
-    p.crs = crs;
-    p.dgs = dgs;
-    p.alpha = alpha;
-    p.sfp = sfp;
-    p.gcrs = gcrs;
-    p.gdgs = gdgs;
-    p.gsfp = gsfp;
-    const int sub = effective_sub(desc, dgs, gdgs);
-    if (desc->coef_shared_rows && want_T) {
-        const size_t need = bwd_ws_bytes(desc);
-        if (!ws || ws_bytes < need) return FOCUS_ERR_WORKSPACE;
-        if (misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
-        p.ws = static_cast<float*>(ws);
-        p.nsub = static_cast<uint32_t>(desc->cols / sub);
-        const uint32_t ny = shared_row_groups(p.rows, p.bpr);
-        return map_cuda(launch_bwd_shared(desc->fmt, desc->dtype, sub, p, ny, st));
-    }
-    return map_cuda(launch_bwd(desc->fmt, desc->dtype, sub, p, st));
+    return run_bwd(desc, x, crs, dgs, alpha, sfp, g, gx, gcrs, gdgs, gsfp, ws, ws_bytes,
+                   reinterpret_cast<cudaStream_t>(stream), nullptr);
+}
+
+FOCUS_API int focus_fq_bwd_adamw(const focus_desc_t* desc, const void* x, float* crs, float* dgs,
+                                 const float* alpha, float* sfp, const void* g, void* gx,
+                                 const focus_adamw_t* hp, const focus_adamw_state_t* state,
+                                 const int64_t* step, float* gcrs, float* gdgs, float* gsfp,
+                                 void* ws, size_t ws_bytes, focus_stream_t stream)
+{
+    const OptArgs opt = {crs, dgs, sfp, hp, state, step};
+    return run_bwd(desc, x, crs, dgs, alpha, sfp, g, gx, gcrs, gdgs, gsfp, ws, ws_bytes,
+                   reinterpret_cast<cudaStream_t>(stream), &opt);
 }

@@ -19,6 +19,8 @@
 //   gx     = mask * fl(g * rho),  rho = fl(S^dq / S^q) once per sub-block
 //   T_ik   = sum of mask * g * x over the sub-block (compensated, Sum2)
 //   dL/dc_i^k = -T_ik / (c_i (c_i^k)^2),  dL/dc_i = -(sum_k T_ik / c_i^k) / c_i^2
+// and, in the fused-optimizer modes, one AdamW step on every learned array
+// right after its gradient is known (Sec. 4.1: AdamW, constant learning rate).
 #pragma once
 
 #include "fq_device.cuh"
@@ -26,7 +28,8 @@
 namespace focus {
 
 constexpr int kThreads = 256;
-enum Mode { kFwd = 0, kPack = 1, kBwd = 2, kBwdS = 3 };  // kBwdS: backward + dL/dS^fp
+// kBwdS: backward + dL/dS^fp; kBwdA / kBwdSA: the same + AdamW in place
+enum Mode { kFwd = 0, kPack = 1, kBwd = 2, kBwdS = 3, kBwdA = 4, kBwdSA = 5 };
 
 struct KParams {
     const void* x;
@@ -57,6 +60,16 @@ struct KParams {
     int shared;           // one coefficient set for all rows
     int ste;              // 0 identity, 1 clipped
     int mx_rule;          // 0 ceiling, 1 OCP floor
+    // fused AdamW (modes kBwdA / kBwdSA and the shared-row finalisation)
+    float* new_crs;       // c_i updated in place (null: c_i not learned)
+    float* new_dgs;       // c_i^k updated in place
+    float* new_sfp;       // S^fp updated in place
+    float* opt_m[3];      // first moments of c_i, c_i^k, S^fp
+    float* opt_v[3];      // second moments
+    const long long* step;  // t >= 1 of this update (device); null: no optimizer step
+    float lr_c, lr_s;     // learning rates of the coefficients and of S^fp
+    float beta1, beta2, eps;
+    float decay_c, decay_s;  // 1 - lr * weight_decay (rounded once)
 };
 
 template <int FMT, int DT, int SUB>
@@ -509,6 +522,54 @@ __device__ __forceinline__ void block_coef_grads(const df (&T)[K], float c, cons
 }
 
 // ---------------------------------------------------------------------------
+// AdamW (decoupled weight decay) in binary32, PyTorch's formulation:
+//   w <- w (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
+//   w <- w - lr / (1 - b1^t) * m / (sqrt(v) / sqrt(1 - b2^t) + eps).
+// The bias corrections 1 - b^t = -expm1(t log1p(-(1 - b))) avoid the
+// cancellation of 1 - pow(b, t) at small t; they are evaluated per thread
+// from the device step counter, so a captured graph replays correctly.
+// ---------------------------------------------------------------------------
+struct AdamW {
+    float b1, o1, b2, o2, eps, rbc2, step_c, step_s, decay_c, decay_s;
+};
+
+__device__ __forceinline__ AdamW adamw_setup(const KParams& p)
+{
+    AdamW a;
+    const float t = static_cast<float>(__ldg(p.step));
+    a.b1 = p.beta1;
+    a.b2 = p.beta2;
+    a.o1 = __fsub_rn(1.0f, p.beta1);
+    a.o2 = __fsub_rn(1.0f, p.beta2);
+    a.eps = p.eps;
+    const float bc1 = -expm1f(__fmul_rn(t, log1pf(-a.o1)));
+    const float bc2 = -expm1f(__fmul_rn(t, log1pf(-a.o2)));
+    a.rbc2 = __frsqrt_rn(bc2);
+    a.step_c = __fdiv_rn(p.lr_c, bc1);
+    a.step_s = __fdiv_rn(p.lr_s, bc1);
+    a.decay_c = p.decay_c;
+    a.decay_s = p.decay_s;
+    return a;
+}
+
+// One update of parameter w with gradient gr; m and v are updated in place.
+__device__ __forceinline__ float adamw_update(float w, float gr, float& m, float& v, float step,
+                                              float decay, const AdamW& a)
+{
+    m = __fadd_rn(__fmul_rn(a.b1, m), __fmul_rn(a.o1, gr));
+    v = __fadd_rn(__fmul_rn(a.b2, v), __fmul_rn(a.o2, __fmul_rn(gr, gr)));
+    const float den = __fadd_rn(__fmul_rn(__fsqrt_rn(v), a.rbc2), a.eps);
+    return __fsub_rn(__fmul_rn(w, decay), __fmul_rn(step, __fdiv_rn(m, den)));
+}
+
+// Moments of one block's parameters, loaded with the block's other inputs.
+template <int K>
+struct BlockMoments {
+    float mc, vc, ms, vs;
+    float md[K], vd[K];
+};
+
+// ---------------------------------------------------------------------------
 // Forward / pack / per-row backward over a linear block index.
 // ---------------------------------------------------------------------------
 template <int FMT, int DT, int MODE>
@@ -535,10 +596,15 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
     constexpr int B = G::B, K = G::K, W = G::W;
     constexpr int U = Unroll<FMT, DT, MODE>::U;
     constexpr int ESZ = DT == 1 ? 2 : 4;
-    constexpr bool BWD = MODE == kBwd || MODE == kBwdS;
+    constexpr bool BWD = MODE >= kBwd;
+    constexpr bool SFPG = MODE == kBwdS || MODE == kBwdSA;
+    constexpr bool ADAM = MODE >= kBwdA;
     const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = BWD && p.gx != nullptr;
-    const bool want_T = (MODE == kBwdS) || (BWD && (p.gcrs != nullptr || p.gdgs != nullptr));
+    const bool want_T = SFPG || (BWD && (p.gcrs != nullptr || p.gdgs != nullptr)) ||
+                        (ADAM && (p.new_crs != nullptr || p.new_dgs != nullptr));
+    AdamW aw;
+    if constexpr (ADAM) aw = adamw_setup(p);
     const uint32_t span = U * kThreads;
 
     for (uint32_t base = blockIdx.x * span; base < p.n_blocks; base += gridDim.x * span) {
@@ -548,6 +614,7 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
         float cv[U];
         float dv[U][K];
         float sv[U];
+        BlockMoments<ADAM ? K : 1> mo[ADAM ? U : 1];
         // ---- issue every load of this step first ----
 #pragma unroll
         for (int j = 0; j < U; ++j) {
@@ -572,6 +639,20 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                 const uint32_t q = p.shared ? cb : blk;
                 if (p.crs) cv[j] = __ldg(p.crs + q);
                 if (p.dgs) load_coefs<K>(p.dgs + static_cast<size_t>(q) * K, dv[j]);
+                if constexpr (ADAM) {
+                    if (p.new_crs) {
+                        mo[j].mc = p.opt_m[0][blk];
+                        mo[j].vc = p.opt_v[0][blk];
+                    }
+                    if (p.new_dgs) {
+                        load_coefs<K>(p.opt_m[1] + static_cast<size_t>(blk) * K, mo[j].md);
+                        load_coefs<K>(p.opt_v[1] + static_cast<size_t>(blk) * K, mo[j].vd);
+                    }
+                    if (SFPG && p.new_sfp) {
+                        mo[j].ms = p.opt_m[2][blk];
+                        mo[j].vs = p.opt_v[2][blk];
+                    }
+                }
             } else {
 #pragma unroll
                 for (int i = 0; i < W; ++i) xr[j][i] = 0u;
@@ -628,17 +709,42 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                 if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
                 float gd[K], gc;
                 df T[K], gS;
-                block_bwd<DT, B, K, MODE == kBwdS>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], sdq,
-                                                   p.ste, want_gx, want_T, p.gx, off[j], gd, gc,
-                                                   T, gS);
+                block_bwd<DT, B, K, SFPG>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], sdq, p.ste,
+                                          want_gx, want_T, p.gx, off[j], gd, gc, T, gS);
                 if (want_T) {
                     if (p.gdgs) store_coefs<K>(p.gdgs + static_cast<size_t>(blk) * K, gd);
                     if (p.gcrs) p.gcrs[blk] = gc;
                 }
-                if constexpr (MODE == kBwdS) {
+                float gs = 0.0f;
+                if constexpr (SFPG) {
                     // STE through Q_fmt: dS^dq/dS^fp = 1 (MXFP4), alpha (NVFP4)
                     const float v = df_to_f(gS);
-                    p.gsfp[blk] = (FMT == 1) ? __fmul_rn(v, ts.alpha) : v;
+                    gs = (FMT == 1) ? __fmul_rn(v, ts.alpha) : v;
+                    if (p.gsfp) p.gsfp[blk] = gs;
+                }
+                if constexpr (ADAM) {
+                    BlockMoments<K>& o = mo[j];
+                    if (p.new_crs) {
+                        p.new_crs[blk] = adamw_update(cv[j], gc, o.mc, o.vc, aw.step_c, aw.decay_c, aw);
+                        p.opt_m[0][blk] = o.mc;
+                        p.opt_v[0][blk] = o.vc;
+                    }
+                    if (p.new_dgs) {
+                        float nd[K];
+#pragma unroll
+                        for (int k = 0; k < K; ++k)
+                            nd[k] = adamw_update(dv[j][k], gd[k], o.md[k], o.vd[k], aw.step_c,
+                                                 aw.decay_c, aw);
+                        const size_t q = static_cast<size_t>(blk) * K;
+                        store_coefs<K>(p.new_dgs + q, nd);
+                        store_coefs<K>(p.opt_m[1] + q, o.md);
+                        store_coefs<K>(p.opt_v[1] + q, o.vd);
+                    }
+                    if (SFPG && p.new_sfp) {
+                        p.new_sfp[blk] = adamw_update(sv[j], gs, o.ms, o.vs, aw.step_s, aw.decay_s, aw);
+                        p.opt_m[2][blk] = o.ms;
+                        p.opt_v[2][blk] = o.vs;
+                    }
                 }
             }
         }
@@ -767,6 +873,23 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams
     if (p.gdgs)
         for (int k = 0; k < K; ++k) p.gdgs[j * K + k] = gd[k];
     if (p.gcrs) p.gcrs[j] = gc;
+    if (p.step) {
+        // AdamW on the shared coefficients once their gradient is complete
+        const AdamW aw = adamw_setup(p);
+        if (p.new_crs) {
+            float m = p.opt_m[0][j], v = p.opt_v[0][j];
+            p.new_crs[j] = adamw_update(c, gc, m, v, aw.step_c, aw.decay_c, aw);
+            p.opt_m[0][j] = m;
+            p.opt_v[0][j] = v;
+        }
+        if (p.new_dgs)
+            for (int k = 0; k < K; ++k) {
+                float m = p.opt_m[1][j * K + k], v = p.opt_v[1][j * K + k];
+                p.new_dgs[j * K + k] = adamw_update(d[k], gd[k], m, v, aw.step_c, aw.decay_c, aw);
+                p.opt_m[1][j * K + k] = m;
+                p.opt_v[1][j * K + k] = v;
+            }
+    }
 }
 
 // ---------------------------------------------------------------------------

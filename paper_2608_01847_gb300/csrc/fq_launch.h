@@ -98,7 +98,44 @@ cudaError_t linear_by_sub(int sub, const KParams& p, cudaStream_t st)
     return cudaErrorInvalidValue;
 }
 
+// Shared-row backward: the row-group kernel, then (when coefficient
+// gradients or an optimizer step are wanted) the column finalisation.
+template <int FMT, int SUB>
+cudaError_t run_shared_finalize(const KParams& p, uint32_t ny, cudaStream_t st)
+{
+    fq_bwd_shared_finalize<FMT, SUB><<<p.bpr, kThreads, 0, st>>>(p, ny);
+    return cudaGetLastError();
+}
+
+template <int FMT, int DT, int SUB>
+cudaError_t run_bwd_shared(const KParams& p, uint32_t ny, cudaStream_t st)
+{
+    const dim3 grid(shared_col_ctas(p.bpr), ny);
+    fq_bwd_shared_kernel<FMT, DT, SUB><<<grid, kThreads, 0, st>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || (p.gcrs == nullptr && p.gdgs == nullptr && p.step == nullptr)) return e;
+    return run_shared_finalize<FMT, SUB>(p, ny, st);
+}
+
+template <int FMT, int DT>
+cudaError_t bwd_shared_by_sub(int sub, const KParams& p, uint32_t ny, cudaStream_t st)
+{
+    switch (sub) {
+    case 2: return run_bwd_shared<FMT, DT, 2>(p, ny, st);
+    case 4: return run_bwd_shared<FMT, DT, 4>(p, ny, st);
+    case 8: return run_bwd_shared<FMT, DT, 8>(p, ny, st);
+    case 16: return run_bwd_shared<FMT, DT, 16>(p, ny, st);
+    case 32:
+        if constexpr (FMT == 0) return run_bwd_shared<FMT, DT, 32>(p, ny, st);
+        break;
+    default: break;
+    }
+    return cudaErrorInvalidValue;
+}
+
 // Defined in the instantiation units.
+cudaError_t launch_bwd_adamw_mx(int dt, int sub, bool sfpg, const KParams& p, cudaStream_t st);
+cudaError_t launch_bwd_adamw_nv(int dt, int sub, bool sfpg, const KParams& p, cudaStream_t st);
 cudaError_t launch_fwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);
 cudaError_t launch_pack(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);
 cudaError_t launch_bwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st);

@@ -28,8 +28,9 @@ FOCUS_WS_ALPHA, FOCUS_WS_BWD = 0, 1
 STATUS = {0: "FOCUS_OK", -1: "FOCUS_ERR_INVALID_ARG", -2: "FOCUS_ERR_UNSUPPORTED",
           -3: "FOCUS_ERR_MISALIGNED", -4: "FOCUS_ERR_WORKSPACE", -5: "FOCUS_ERR_CUDA"}
 
-ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd", "focus_pack",
-                "focus_workspace_bytes", "focus_status_string", "focus_version")
+ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd",
+                "focus_fq_bwd_adamw", "focus_pack", "focus_workspace_bytes", "focus_status_string",
+                "focus_version")
 
 
 class FocusError(RuntimeError):
@@ -44,6 +45,16 @@ class focus_desc_t(ctypes.Structure):
                 ("dtype", ctypes.c_int32), ("fmt", ctypes.c_int32), ("block", ctypes.c_int32),
                 ("sub_block", ctypes.c_int32), ("coef_shared_rows", ctypes.c_int32),
                 ("ste", ctypes.c_int32), ("mx_rule", ctypes.c_int32)]
+
+
+class focus_adamw_t(ctypes.Structure):
+    _fields_ = [("lr_coef", ctypes.c_float), ("lr_scale", ctypes.c_float),
+                ("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
+                ("weight_decay", ctypes.c_float)]
+
+
+class focus_adamw_state_t(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("m_crs", "v_crs", "m_dgs", "v_dgs", "m_sfp", "v_sfp")]
 
 
 _lib: Optional[ctypes.CDLL] = None
@@ -62,13 +73,16 @@ def lib() -> ctypes.CDLL:
         L.focus_nvfp4_alpha_noalloc.argtypes = [D, P, P, P]
         L.focus_fq_fwd.argtypes = [D, P, P, P, P, P, P, P, P]
         L.focus_fq_bwd.argtypes = [D, P, P, P, P, P, P, P, P, P, P, P, SZ, P]
+        L.focus_fq_bwd_adamw.argtypes = [D, P, P, P, P, P, P, P, ctypes.POINTER(focus_adamw_t),
+                                         ctypes.POINTER(focus_adamw_state_t), P, P, P, P, P, SZ, P]
         L.focus_pack.argtypes = [D, P, P, P, P, P, P, P, P]
         L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
         L.focus_workspace_bytes.restype = SZ
         L.focus_status_string.argtypes = [ctypes.c_int]
         L.focus_status_string.restype = ctypes.c_char_p
         L.focus_version.restype = ctypes.c_int
-        for n in ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd", "focus_pack"):
+        for n in ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd",
+                  "focus_fq_bwd_adamw", "focus_pack"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -232,6 +246,50 @@ def focus_fq_bwd(x, g, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shar
     if want_gsfp:
         return gx, gcrs, gdgs, gsfp
     return gx, gcrs, gdgs
+
+
+def focus_fq_bwd_adamw(x, g, fmt, step, hp, crs=None, dgs=None, sfp=None, moments=None,
+                       alpha=None, *, sub_block=8, shared=False, ste=FOCUS_STE_IDENTITY,
+                       mx_rule=FOCUS_MX_CEIL, want_gx=True, gx=None, gcrs=None, gdgs=None,
+                       gsfp=None, ws=None):
+    """STE backward fused with one AdamW step (Sec. 3.2, Sec. 4.1).
+
+    crs / dgs / sfp: the learned arrays (fp32 CUDA tensors, updated in place;
+    None = not learned).  moments: dict name -> (m, v) tensors shaped like the
+    parameter ('crs', 'dgs', 'sfp'), updated in place.  step: int64 CUDA
+    tensor holding t >= 1 (read only).  hp: dict with lr_coef, lr_scale,
+    beta1, beta2, eps, weight_decay.  gcrs / gdgs / gsfp: optional gradient
+    outputs.  Returns gx (or None)."""
+    desc = make_desc(x, fmt, sub_block, shared, ste, mx_rule)
+    moments = moments or {}
+    _check_coefs(x, fmt, sub_block, shared, crs, dgs)
+    _check_coefs(x, fmt, sub_block, shared, gcrs, gdgs)
+    _check_sfp(x, fmt, sfp, "sfp")
+    _check_sfp(x, fmt, gsfp, "gsfp")
+    _same_layout(x, g, "g")
+    if gx is None and want_gx:
+        gx = _like_x(x)
+    _same_layout(x, gx, "gx")
+    if step.dtype != torch.int64 or step.numel() != 1 or step.device != x.device:
+        raise ValueError("step must be a one-element int64 tensor on x's device")
+    st = focus_adamw_state_t()
+    for name, param in (("crs", crs), ("dgs", dgs), ("sfp", sfp)):
+        if param is None:
+            continue
+        if name not in moments:
+            raise ValueError(f"moments for {name} are missing")
+        for k, t in zip("mv", moments[name]):
+            _dense(t, param.numel(), torch.float32, f"{k}_{name}")
+            setattr(st, f"{k}_{name}", t.data_ptr())
+    h = focus_adamw_t(*(float(hp[k]) for k in ("lr_coef", "lr_scale", "beta1", "beta2", "eps",
+                                                 "weight_decay")))
+    ws, nb = _workspace(desc, FOCUS_WS_BWD, x.device, ws)
+    _check(lib().focus_fq_bwd_adamw(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha),
+                                    _p(sfp), _p(g), _p(gx), ctypes.byref(h), ctypes.byref(st),
+                                    _p(step), _p(gcrs), _p(gdgs), _p(gsfp), _p(ws), nb,
+                                    _stream(x.device)),
+           "focus_fq_bwd_adamw")
+    return gx
 
 
 def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,

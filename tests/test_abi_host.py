@@ -47,7 +47,7 @@ def test_exports_exactly_the_declared_symbols(L):
 
 
 def test_version_and_status_strings(L):
-    assert F.focus_version() == 200
+    assert F.focus_version() == 210
     for code in (0, -1, -2, -3, -4, -5):
         assert L.focus_status_string(code)
     assert L.focus_status_string(42) == b"unknown status"
@@ -147,3 +147,54 @@ def test_fastdiv_magic_numbers():
         t = (n * np.uint64(m)) >> np.uint64(32)
         q = (t + n) >> np.uint64(l)
         assert np.array_equal(q, n // np.uint64(d)), d
+
+
+def adamw(L, d, hp, st, step=ALIGNED2, crs=ALIGNED, dgs=None, sfp=None, x=ALIGNED, g=ALIGNED2,
+          gx=None, ws=None, nb=0):
+    return L.focus_fq_bwd_adamw(ctypes.byref(d), x, crs, dgs, ALIGNED2, sfp, g, gx,
+                                ctypes.byref(hp) if hp is not None else None,
+                                ctypes.byref(st) if st is not None else None, step, None, None,
+                                None, ws, nb, None)
+
+
+def _hp(**kw):
+    v = dict(lr_coef=5e-2, lr_scale=2e-2, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+    v.update(kw)
+    return F.focus_adamw_t(*(v[k] for k in ("lr_coef", "lr_scale", "beta1", "beta2", "eps",
+                                            "weight_decay")))
+
+
+def _st(**kw):
+    st = F.focus_adamw_state_t()
+    for i, n in enumerate(("m_crs", "v_crs", "m_dgs", "v_dgs", "m_sfp", "v_sfp")):
+        setattr(st, n, kw.get(n, 0x300000 + 0x10000 * i))
+    return st
+
+
+@pytest.mark.parametrize("hp_kw,status", [
+    (dict(lr_coef=-1.0), -1), (dict(lr_scale=float("nan")), -1), (dict(beta1=1.0), -1),
+    (dict(beta2=-0.1), -1), (dict(eps=0.0), -1), (dict(eps=float("inf")), -1),
+    (dict(weight_decay=-1e-3), -1), (dict(lr_coef=float("inf")), -1),
+])
+def test_adamw_hyperparameter_rejections(L, hp_kw, status):
+    d = _desc(rows=0)      # nothing to compute: only the checks run
+    assert adamw(L, d, _hp(**hp_kw), _st()) == status
+    assert adamw(L, d, _hp(), _st()) == 0
+
+
+def test_adamw_argument_rejections(L):
+    d = _desc(rows=0)
+    assert adamw(L, d, None, _st()) == -1                          # hyper-parameters missing
+    assert adamw(L, d, _hp(), None) == -1                          # state missing
+    assert adamw(L, d, _hp(), _st(), step=None) == -1              # step counter missing
+    assert adamw(L, d, _hp(), _st(), step=P(0x100004)) == -3       # step is an int64
+    assert adamw(L, d, _hp(), _st(m_crs=0)) == -1                  # moments of a learned array
+    assert adamw(L, d, _hp(), _st(m_crs=0), crs=None) == 0         # ... not needed if not learned
+    assert adamw(L, d, _hp(), _st(v_dgs=0x300008), dgs=ALIGNED) == -3
+    assert adamw(L, d, _hp(), _st(m_sfp=0), sfp=ALIGNED) == -1
+    assert adamw(L, _desc(rows=0, shared=1), _hp(), _st(), sfp=ALIGNED) == -1   # S^fp is per row
+    assert adamw(L, _desc(), _hp(), _st(), x=ODD) == -3
+    assert adamw(L, _desc(), _hp(), _st(), g=None) == -1
+    assert adamw(L, _desc(fmt=1, block=32), _hp(), _st()) == -2
+    d = _desc(rows=64, cols=256, shared=1)
+    assert adamw(L, d, _hp(), _st()) == -4                         # shared rows need scratch
