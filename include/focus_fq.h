@@ -242,6 +242,48 @@ int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
                const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
                uint8_t* scale_bytes, focus_stream_t stream);
 
+/* Export for the Blackwell block-scaled tensor-core MMA (the deployment the
+ * paper targets: FP4 GEMMs on hardware that reads E2M1 codes with E8M0 /
+ * E4M3 block scales directly, Sec. 1 and Sec. 3.1).  Codes exactly as
+ * focus_pack writes them (row-major, K-major operand of the MMA).  The scale
+ * bytes go to scale_tiles in the MMA scale-factor layout: the [rows, C]
+ * scale matrix (C = cols / block) is cut into tiles of 128 rows x 4 columns
+ * of 512 bytes; tile (i, j) starts at byte (i * ceil(C / 4) + j) * 512, and
+ * inside it row r (0..127) and column c (0..3) are at byte
+ * (r % 32) * 16 + (r / 32) * 4 + c.  Bytes of the padding (rows beyond
+ * `rows`, columns beyond C) are written as 0.  scale_tiles: 16-byte aligned,
+ * focus_mma_scale_bytes(desc) bytes.  Other arguments as for focus_pack. */
+int focus_pack_mma(const focus_desc_t* desc, const void* x, const float* crs,
+                   const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
+                   uint8_t* scale_tiles, focus_stream_t stream);
+
+/* Size in bytes of focus_pack_mma's scale tiles for this descriptor
+ * (ceil(rows / 128) * ceil(cols / block / 4) * 512); 0 for an invalid
+ * descriptor. */
+size_t focus_mma_scale_bytes(const focus_desc_t* desc);
+
+/* W4A4 GEMM on the block-scaled FP4 tensor cores (tcgen05.mma
+ * .kind::mxf4 / .kind::mxf4nvf4) over two focus_pack_mma exports, the
+ * product a deployed FOCUS model computes with nothing but its export
+ * (Sec. 1, Sec. 3.1; Fig. 3(d)):
+ *   D[m, n] = sum_k A[m, k] * B[n, k]                       (MXFP4)
+ *   D[m, n] = fl(alpha_a * alpha_b) * sum_k A[m, k] * B[n, k]  (NVFP4)
+ * with A[m, k] = E2M1(code) * scale(m, k / block) (E8M0 / E4M3 scales).
+ * a_codes [M, K/2], b_codes [N, K/2]: row-major code bytes as written by
+ * focus_pack_mma (B is the second operand's rows, e.g. a weight [out, in]);
+ * a_scale_tiles / b_scale_tiles: their MMA-layout scale tiles; alpha_a,
+ * alpha_b: device fp32 per-tensor scales (NVFP4 only; ignored for MXFP4).
+ * d: [M, ldd] row-major fp32 output (ldd >= N), overwritten.  The products
+ * are exact and accumulate in fp32 inside the tensor core.
+ * Requirements: K % 64 == 0 (FOCUS_ERR_UNSUPPORTED otherwise); codes and
+ * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
+ * kernel whose wait for its MMAs gives up sets it to 1 (the output is then
+ * not written) instead of waiting for ever.  Enqueued on `stream`. */
+int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
+                   const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
+                   const uint8_t* b_scale_tiles, const float* alpha_b, float* d, int64_t ldd,
+                   int32_t* timeout_flag, focus_stream_t stream);
+
 /* Device scratch (bytes) that focus_nvfp4_alpha (which = FOCUS_WS_ALPHA) or
  * focus_fq_bwd (which = FOCUS_WS_BWD) needs for this descriptor on the
  * current device; 0 for an invalid descriptor. */

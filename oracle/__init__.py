@@ -318,3 +318,56 @@ def dequant(codes, scales, fmt, alpha=0.0, block=None, dtype=F32):
     _check(lib().focus_oracle_dequant(fmt, dtype, rows, cols, block, _ptr(codes),
                                       _ptr(scales), float(alpha), _ptr(y)))
     return y
+
+
+# --------------------------------------------------------------------------
+# Deployment view: the exported FP4 operands of a block-scaled tensor-core
+# GEMM (the hardware path the paper's "no inference overhead" rests on,
+# Sec. 1 and Sec. 3.1; the export of Fig. 3(d))
+# --------------------------------------------------------------------------
+def mma_scale_tiles(scales):
+    """Row-major scale bytes [R, C] -> the block-scaled MMA scale-factor
+    layout: tiles of 128 rows x 4 columns (512 bytes) over the matrix padded
+    with zero bytes to multiples of 128 x 4, tile (i, j) at (i * ceil(C/4) + j)
+    * 512, row r / column c of a tile at (r % 32) * 16 + (r // 32) * 4 + c.
+    Written out element by element."""
+    scales = np.asarray(scales, np.uint8)
+    R, C = scales.shape
+    tr, tc = (R + 127) // 128, (C + 3) // 4
+    out = np.zeros(tr * tc * 512, np.uint8)
+    for r in range(R):
+        for c in range(C):
+            i, j = r // 128, c // 4
+            rr, cc = r % 128, c % 4
+            out[(i * tc + j) * 512 + (rr % 32) * 16 + (rr // 32) * 4 + cc] = scales[r, c]
+    return out
+
+
+def fp4_gemm(codes_a, scales_a, codes_b, scales_b, fmt, alpha_a=1.0, alpha_b=1.0, block=None):
+    """D[m, n] = sum_k A[m, k] B[n, k] in binary64 for exported FP4 operands
+    (codes [rows, K/2], element 2t in the low nibble; row-major scale bytes
+    [rows, K/block]): A[m, k] = E2M1(code) * S(m, k / block) with S = 2^(byte
+    - 127) for MXFP4 and E4M3(byte) for NVFP4, and D scaled by alpha_a *
+    alpha_b for NVFP4 (the per-tensor scales, Eq. 2).  Dequantization
+    through the oracle's own decoders; the contraction is numpy's matmul."""
+    block = block or default_block(fmt)
+
+    def dense(codes, scales):
+        codes = np.asarray(codes, np.uint8)
+        rows, half = codes.shape
+        k = half * 2
+        nib = np.empty((rows, k), np.int64)
+        nib[:, 0::2] = codes & 15
+        nib[:, 1::2] = codes >> 4
+        val = np.array([e2m1_value(c) for c in range(16)], np.float64)[nib]
+        sb = np.asarray(scales, np.uint8)
+        if fmt == MXFP4:
+            s = np.ldexp(1.0, sb.astype(np.int64) - 127)
+        else:
+            s = np.array([e4m3_decode(b) for b in range(256)], np.float64)[sb]
+        return val * np.repeat(s, block, axis=1)
+
+    d = dense(codes_a, scales_a) @ dense(codes_b, scales_b).T
+    if fmt == NVFP4:
+        d = d * (float(np.float32(alpha_a)) * float(np.float32(alpha_b)))
+    return d

@@ -99,6 +99,14 @@ int check_coef_ptrs(const float* a, const float* b, const float* c, const float*
 
 size_t bwd_ws_bytes(const focus_desc_t* d);
 
+// Bytes of the scale tiles of the MMA layout: 128-row x 4-column tiles of
+// the [rows, cols/block] scale matrix, 512 bytes each.
+size_t mma_scale_bytes(const focus_desc_t* d)
+{
+    const int64_t sc = d->cols / d->block;
+    return static_cast<size_t>((d->rows + 127) / 128) * static_cast<size_t>((sc + 3) / 4) * 512;
+}
+
 // Column finalisation of the shared-row backward alone (no rows to reduce).
 cudaError_t launch_shared_finalize(int fmt, int sub, const KParams& p, cudaStream_t st)
 {
@@ -317,9 +325,12 @@ FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float*
                                reinterpret_cast<cudaStream_t>(stream)));
 }
 
-FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
-                         const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
-                         uint8_t* scale_bytes, focus_stream_t stream)
+namespace focus {
+namespace {
+
+int run_pack(const focus_desc_t* desc, const void* x, const float* crs, const float* dgs,
+             const float* alpha, const float* sfp, uint8_t* codes, uint8_t* scale_bytes,
+             bool mma_layout, cudaStream_t st)
 {
     int rc = check_desc(desc, true);
     if (rc) return rc;
@@ -329,6 +340,7 @@ FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* c
         return FOCUS_ERR_INVALID_ARG;
     if (misaligned(x, 32) || misaligned(codes, 16) || misaligned(alpha, 4) || misaligned(sfp, 4))
         return FOCUS_ERR_MISALIGNED;
+    if (mma_layout && misaligned(scale_bytes, 16)) return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
     p.x = x;
@@ -338,8 +350,41 @@ FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* c
     p.sfp = sfp;
     p.codes = codes;
     p.scales = scale_bytes;
-    return map_cuda(launch_pack(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p,
-                                reinterpret_cast<cudaStream_t>(stream)));
+    if (mma_layout) {
+        const int64_t sc = desc->cols / desc->block;
+        p.sf_tile_cols = static_cast<uint32_t>((sc + 3) / 4);
+        // padding of the last tile row / column: zero bytes
+        if (desc->rows % 128 != 0 || sc % 4 != 0) {
+            const cudaError_t e = cudaMemsetAsync(scale_bytes, 0, mma_scale_bytes(desc), st);
+            if (e != cudaSuccess) return FOCUS_ERR_CUDA;
+        }
+    }
+    return map_cuda(launch_pack(desc->fmt, desc->dtype, effective_sub(desc, dgs, nullptr), p, st));
+}
+
+}  // namespace
+}  // namespace focus
+
+FOCUS_API int focus_pack(const focus_desc_t* desc, const void* x, const float* crs,
+                         const float* dgs, const float* alpha, const float* sfp, uint8_t* codes,
+                         uint8_t* scale_bytes, focus_stream_t stream)
+{
+    return run_pack(desc, x, crs, dgs, alpha, sfp, codes, scale_bytes, false,
+                    reinterpret_cast<cudaStream_t>(stream));
+}
+
+FOCUS_API size_t focus_mma_scale_bytes(const focus_desc_t* desc)
+{
+    if (check_desc(desc, true) != FOCUS_OK) return 0;
+    return mma_scale_bytes(desc);
+}
+
+FOCUS_API int focus_pack_mma(const focus_desc_t* desc, const void* x, const float* crs,
+                             const float* dgs, const float* alpha, const float* sfp,
+                             uint8_t* codes, uint8_t* scale_tiles, focus_stream_t stream)
+{
+    return run_pack(desc, x, crs, dgs, alpha, sfp, codes, scale_tiles, true,
+                    reinterpret_cast<cudaStream_t>(stream));
 }
 
 FOCUS_API int focus_fq_bwd(const focus_desc_t* desc, const void* x, const float* crs,

@@ -60,6 +60,8 @@ struct KParams {
     int shared;           // one coefficient set for all rows
     int ste;              // 0 identity, 1 clipped
     int mx_rule;          // 0 ceiling, 1 OCP floor
+    uint32_t sf_tile_cols;  // export: 0 = row-major scale bytes; else the scale
+                            // bytes go to 128 x 4 MMA tiles, this many per tile row
     // fused AdamW (modes kBwdA / kBwdSA and the shared-row finalisation)
     float* new_crs;       // c_i updated in place (null: c_i not learned)
     float* new_dgs;       // c_i^k updated in place
@@ -522,6 +524,19 @@ __device__ __forceinline__ void block_coef_grads(const df (&T)[K], float c, cons
 }
 
 // ---------------------------------------------------------------------------
+// Scale bytes in the block-scaled MMA layout of the Blackwell tensor cores:
+// the [rows, cols/B] scale matrix is cut into tiles of 128 rows x 4 scale
+// columns (512 bytes, tile row-major over the padded matrix); inside a tile,
+// row r and column c sit at (r % 32) * 16 + (r / 32) * 4 + c, so that the 32
+// byte-quadruples of one 16-byte line hold rows r, r+32, r+64, r+96.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ size_t mma_scale_offset(uint32_t row, uint32_t col, uint32_t tile_cols)
+{
+    const size_t tile = static_cast<size_t>(row / 128) * tile_cols + col / 4;
+    return tile * 512 + (row % 32) * 16 + ((row % 128) / 32) * 4 + (col % 4);
+}
+
+// ---------------------------------------------------------------------------
 // AdamW (decoupled weight decay) in binary32, PyTorch's formulation:
 //   w <- w (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
 //   w <- w - lr / (1 - b1^t) * m / (sqrt(v) / sqrt(1 - b2^t) + eps).
@@ -703,7 +718,14 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                         __stcs(reinterpret_cast<uint2*>(dst), make_uint2(codes[0], codes[1]));
                     }
                 }
-                if (p.scales) p.scales[blk] = static_cast<uint8_t>(sbyte);
+                if (p.scales) {
+                    size_t at = blk;
+                    if (p.sf_tile_cols) {
+                        const uint32_t row = fast_div(blk, p.div_bpr);
+                        at = mma_scale_offset(row, blk - row * p.bpr, p.sf_tile_cols);
+                    }
+                    p.scales[at] = static_cast<uint8_t>(sbyte);
+                }
             } else {
                 float rho[K];
                 if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);

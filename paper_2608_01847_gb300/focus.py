@@ -29,8 +29,9 @@ STATUS = {0: "FOCUS_OK", -1: "FOCUS_ERR_INVALID_ARG", -2: "FOCUS_ERR_UNSUPPORTED
           -3: "FOCUS_ERR_MISALIGNED", -4: "FOCUS_ERR_WORKSPACE", -5: "FOCUS_ERR_CUDA"}
 
 ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd",
-                "focus_fq_bwd_adamw", "focus_pack", "focus_workspace_bytes", "focus_status_string",
-                "focus_version")
+                "focus_fq_bwd_adamw", "focus_pack", "focus_pack_mma", "focus_mma_scale_bytes",
+                "focus_fp4_gemm",
+                "focus_workspace_bytes", "focus_status_string", "focus_version")
 
 
 class FocusError(RuntimeError):
@@ -76,13 +77,18 @@ def lib() -> ctypes.CDLL:
         L.focus_fq_bwd_adamw.argtypes = [D, P, P, P, P, P, P, P, ctypes.POINTER(focus_adamw_t),
                                          ctypes.POINTER(focus_adamw_state_t), P, P, P, P, P, SZ, P]
         L.focus_pack.argtypes = [D, P, P, P, P, P, P, P, P]
+        L.focus_pack_mma.argtypes = [D, P, P, P, P, P, P, P, P]
+        L.focus_mma_scale_bytes.argtypes = [D]
+        L.focus_mma_scale_bytes.restype = SZ
+        I32, I64 = ctypes.c_int32, ctypes.c_int64
+        L.focus_fp4_gemm.argtypes = [I32, I64, I64, I64, P, P, P, P, P, P, P, I64, P, P]
         L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
         L.focus_workspace_bytes.restype = SZ
         L.focus_status_string.argtypes = [ctypes.c_int]
         L.focus_status_string.restype = ctypes.c_char_p
         L.focus_version.restype = ctypes.c_int
         for n in ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd",
-                  "focus_fq_bwd_adamw", "focus_pack"):
+                  "focus_fq_bwd_adamw", "focus_pack", "focus_pack_mma", "focus_fp4_gemm"):
             getattr(L, n).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -308,6 +314,55 @@ def focus_pack(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=Fa
     _check(lib().focus_pack(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(sfp),
                             _p(codes), _p(scale_bytes), _stream(x.device)), "focus_pack")
     return codes, scale_bytes
+
+
+def focus_mma_scale_bytes(desc: focus_desc_t) -> int:
+    return int(lib().focus_mma_scale_bytes(ctypes.byref(desc)))
+
+
+def focus_pack_mma(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, shared=False,
+                   mx_rule=FOCUS_MX_CEIL, codes=None, scale_tiles=None, sfp=None):
+    """Export for the block-scaled tensor-core MMA: returns (codes [rows, cols/2]
+    uint8, scale tiles: focus_mma_scale_bytes uint8 in the 128 x 4 tile layout)."""
+    desc = make_desc(x, fmt, sub_block, shared, FOCUS_STE_IDENTITY, mx_rule)
+    rows, cols = x.shape
+    n = focus_mma_scale_bytes(desc)
+    if codes is None:
+        codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device=x.device)
+    if scale_tiles is None:
+        scale_tiles = torch.empty(max(n, 16), dtype=torch.uint8, device=x.device)
+    _check_coefs(x, fmt, sub_block, shared, crs, dgs)
+    _dense(codes, rows * cols // 2, torch.uint8, "codes")
+    if not scale_tiles.is_contiguous() or scale_tiles.numel() < n or scale_tiles.dtype != torch.uint8:
+        raise ValueError(f"scale_tiles must be a contiguous uint8 tensor of at least {n} bytes")
+    _check_sfp(x, fmt, sfp, "sfp")
+    _check(lib().focus_pack_mma(ctypes.byref(desc), _p(x), _p(crs), _p(dgs), _p(alpha), _p(sfp),
+                                _p(codes), _p(scale_tiles), _stream(x.device)), "focus_pack_mma")
+    return codes, scale_tiles
+
+
+def focus_fp4_gemm(fmt, a_codes, a_tiles, b_codes, b_tiles, alpha_a=None, alpha_b=None, *, d=None,
+                   timeout_flag=None):
+    """D = A B^T on the block-scaled FP4 tensor cores from two focus_pack_mma
+    exports (codes [M, K/2] and [N, K/2] uint8, their scale tiles); returns
+    D [M, N] fp32.  alpha_a / alpha_b: NVFP4 per-tensor scales ([1] fp32)."""
+    M, kh = a_codes.shape
+    N, kh2 = b_codes.shape
+    if kh != kh2:
+        raise ValueError("A and B must have the same K")
+    K = 2 * kh
+    for t, name in ((a_codes, "a_codes"), (b_codes, "b_codes"), (a_tiles, "a_tiles"),
+                    (b_tiles, "b_tiles")):
+        if t.dtype != torch.uint8 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous uint8 tensor")
+    if d is None:
+        d = torch.empty((M, N), dtype=torch.float32, device=a_codes.device)
+    if d.dtype != torch.float32 or d.dim() != 2 or d.shape[0] != M or d.shape[1] != N or d.stride(1) != 1:
+        raise ValueError("d must be a [M, N] fp32 tensor with unit column stride")
+    _check(lib().focus_fp4_gemm(int(fmt), M, N, K, _p(a_codes), _p(a_tiles), _p(alpha_a),
+                                _p(b_codes), _p(b_tiles), _p(alpha_b), _p(d), d.stride(0),
+                                _p(timeout_flag), _stream(a_codes.device)), "focus_fp4_gemm")
+    return d
 
 
 def focus_version() -> int:

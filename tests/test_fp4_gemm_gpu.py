@@ -1,0 +1,138 @@
+"""GPU parity of the tensor-core FP4 GEMM over focus_pack_mma exports.
+
+Both operands are fake-quantized and exported on the GPU; the export must
+equal the oracle's bit for bit, and D must match the oracle's binary64
+contraction of the oracle's own export (oracle.fp4_gemm) within the fp32
+accumulation bound
+
+    |D - D_ref| <= (K / 16 + 8) * 2^-23 * sum_k |A[m, k] B[n, k]|  (+ 2^-23 |D_ref| for alpha)
+
+(every product is exact in fp32; each accumulation step rounds at most once
+by 2^-23 relative to the running magnitude).  A wrong scale, element or
+block shifts D by far more."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2608_01847_gb300 import build as B
+from paper_2608_01847_gb300 import focus as F
+from paper_2608_01847_gb300 import workloads as W
+from gpu_helpers import assert_bits_equal, dev, host
+
+pytestmark = pytest.mark.gpu
+
+FMT = {"mx": O.MXFP4, "nv": O.NVFP4}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    B.build()
+    F.lib()
+
+
+def operand(rows, k, seed, kind):
+    """Seeded host operand: an activation (N(0,1), a few outlier channels)
+    or a weight (Student-t(5) x 0.02), bf16."""
+    if kind == "act":
+        w = W.Workload("a", (W.TensorSpec("a", rows, k),), "bf16", ("nvfp4",), "activation", None, 1.0,
+                       "channels", 4, 30.0, (0.9, 1.1), seed)
+    else:
+        w = W.Workload("w", (W.TensorSpec("w", rows, k),), "bf16", ("nvfp4",), "weight", 5.0, 0.02,
+                       "entries", 0.001, 20.0, (0.9, 1.1), seed)
+    x, _ = W.host_tensor(w, 0)
+    return w, x
+
+
+def export_both(x, fmt, crs):
+    """GPU export (checked against the oracle's) and the oracle's export."""
+    a = O.alpha(x) if fmt == O.NVFP4 else 0.0
+    a_dev = torch.tensor([a], dtype=torch.float32, device="cuda")
+    cd = dev(crs) if crs is not None else None
+    codes, tiles = F.focus_pack_mma(dev(x), fmt, cd, None, a_dev)
+    ref = O.fwd(x, fmt, crs=crs, alpha=a, want_y=False, want_codes=True)
+    torch.cuda.synchronize()
+    assert_bits_equal(host(codes), ref["codes"], "codes")
+    assert_bits_equal(host(tiles), O.mma_scale_tiles(ref["scales"]), "scale tiles")
+    return codes, tiles, a_dev, ref, a
+
+
+def check_gemm(fmt, M, N, K, seed=0, crs=True):
+    block = 32 if fmt == O.MXFP4 else 16
+    wa, xa = operand(M, K, seed, "act")
+    wb, xb = operand(N, K, seed + 1, "weight")
+    ca = W.draw_coefs(wa, M * K // block, seed + 2).reshape(M, -1) if crs else None
+    cb = W.draw_coefs(wb, N * K // block, seed + 3).reshape(N, -1) if crs else None
+    ac, at, aa_dev, ra, aa = export_both(xa, fmt, ca)
+    bc, bt, ab_dev, rb, ab = export_both(xb, fmt, cb)
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    d = F.focus_fp4_gemm(fmt, ac, at, bc, bt, aa_dev, ab_dev, timeout_flag=flag)
+    torch.cuda.synchronize()
+    assert int(flag.item()) == 0, "MMA wait gave up"
+    ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], fmt, aa, ab)
+    mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], fmt, aa, ab)
+    got = host(d).astype(np.float64)
+    bound = (K / 16 + 8) * 2.0 ** -23 * mag + 2.0 ** -23 * np.abs(ref) + 1e-30
+    err = np.abs(got - ref)
+    bad = np.argwhere(~(err <= bound))
+    assert bad.size == 0, (f"{len(bad)} of {got.size} outside the bound; first {tuple(bad[0])}: "
+                           f"gpu {got[tuple(bad[0])]!r} ref {ref[tuple(bad[0])]!r}")
+    return d, ref
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+@pytest.mark.parametrize("M,N,K", [(128, 128, 64), (128, 128, 256), (256, 384, 512), (200, 130, 320),
+                                   (1, 1, 64), (129, 257, 1024), (384, 128, 2560)])
+def test_fp4_gemm_parity(fmt, M, N, K):
+    check_gemm(FMT[fmt], M, N, K, seed=M + N + K)
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_fp4_gemm_without_coefficients(fmt):
+    """c = 1: the export is plain RTN MXFP4 / NVFP4."""
+    check_gemm(FMT[fmt], 256, 256, 512, seed=5, crs=False)
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_fp4_gemm_degenerate_sizes(fmt):
+    f = FMT[fmt]
+    z = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    one = torch.ones(1, dtype=torch.float32, device="cuda")
+    d = F.focus_fp4_gemm(f, torch.zeros((3, 0), dtype=torch.uint8, device="cuda"), z,
+                         torch.zeros((5, 0), dtype=torch.uint8, device="cuda"), z, one, one,
+                         d=torch.full((3, 5), 7.0, device="cuda"))
+    torch.cuda.synchronize()
+    assert torch.equal(d, torch.zeros_like(d))                       # K = 0: empty sums
+    with pytest.raises(F.FocusError):
+        F.focus_fp4_gemm(f, torch.zeros((4, 16), dtype=torch.uint8, device="cuda"), z,
+                         torch.zeros((4, 16), dtype=torch.uint8, device="cuda"), z, one, one)  # K = 32
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_export_read_by_library_gemm(fmt):
+    """The export is what NVIDIA's own block-scaled FP4 GEMM (cuBLASLt,
+    through torch._scaled_mm) reads: same product within bf16 output
+    rounding.  Skipped where the installed torch has no FP4 path."""
+    f = FMT[fmt]
+    if not hasattr(torch, "float4_e2m1fn_x2"):
+        pytest.skip("torch without float4_e2m1fn_x2")
+    M, N, K = 256, 256, 512
+    wa, xa = operand(M, K, 11, "act")
+    wb, xb = operand(N, K, 12, "weight")
+    ac, at, aa_dev, ra, aa = export_both(xa, f, None)
+    bc, bt, ab_dev, rb, ab = export_both(xb, f, None)
+    sdt = torch.float8_e8m0fnu if f == O.MXFP4 else torch.float8_e4m3fn
+    try:
+        out = torch._scaled_mm(ac.view(torch.float4_e2m1fn_x2), bc.view(torch.float4_e2m1fn_x2).t(),
+                               at.view(sdt), bt.view(sdt), out_dtype=torch.bfloat16)
+        torch.cuda.synchronize()
+    except (RuntimeError, TypeError, NotImplementedError) as e:
+        pytest.skip(f"library FP4 GEMM unavailable here: {str(e).splitlines()[0][:120]}")
+    lib = out.float().cpu().numpy().astype(np.float64)
+    if f == O.NVFP4:
+        lib = lib * (float(np.float32(aa)) * float(np.float32(ab)))
+    ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], f, aa, ab)
+    mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], f, aa, ab)
+    assert np.all(np.abs(lib - ref) <= 2.0 ** -7 * np.abs(ref) + 2.0 ** -18 * mag)

@@ -733,3 +733,91 @@ def test_bwd_adamw_equals_autograd_and_torch_adamw(fmt):
     # arrays that are not learned are not in the result
     part = O.bwd_adamw(x, g, fmt, {"dgs": dgs}, {"dgs": moments["dgs"]}, HP, step, alpha=a)
     assert set(part) == {"gx", "dgs"}
+
+
+# ---------------------------------------------------------------------------
+# deployment view: MMA scale-factor tiles and the FP4 GEMM on the export
+# ---------------------------------------------------------------------------
+def test_mma_scale_tiles_hand_offsets():
+    R, C = 130, 5
+    s = np.zeros((R, C), np.uint8)
+    marks = {(0, 0): 1, (1, 0): 2, (31, 0): 3, (32, 0): 4, (64, 1): 5, (96, 3): 6, (0, 4): 7,
+             (128, 0): 8, (129, 4): 9, (127, 3): 10}
+    for (r, c), v in marks.items():
+        s[r, c] = v
+    t = O.mma_scale_tiles(s)
+    assert t.size == 2 * 2 * 512                       # 2 x 2 tiles (rows and columns padded)
+    where = {0: 1, 16: 2, 496: 3, 4: 4, 9: 5, 15: 6, 512: 7, 1024: 8, 1552: 9,
+             31 * 16 + 3 * 4 + 3: 10}
+    for off, v in where.items():
+        assert t[off] == v, (off, t[off], v)
+    assert np.count_nonzero(t) == len(marks)
+
+
+def test_mma_scale_tiles_is_a_permutation():
+    rng = np.random.default_rng(101)
+    R, C = 256, 8
+    s = rng.integers(1, 256, (R, C), dtype=np.uint8)
+    t = O.mma_scale_tiles(s)
+    assert t.size == R * C
+    assert np.array_equal(np.sort(t), np.sort(s.reshape(-1)))
+    # each 16-byte line of a tile holds rows r, r+32, r+64, r+96 (4 columns each)
+    line = t[:16].reshape(4, 4)
+    assert np.array_equal(line, s[[0, 32, 64, 96], :4])
+
+
+def _dequant_independent(codes, scales, fmt):
+    """Dense values of an export through torch's float8 decoders and the
+    pins' own E2M1 grid (nothing of the oracle)."""
+    k = codes.shape[1] * 2
+    nib = np.empty((codes.shape[0], k), np.int64)
+    nib[:, 0::2] = codes & 15
+    nib[:, 1::2] = codes >> 4
+    val = np.array([code_to_value(c) for c in range(16)])[nib]
+    block = 32 if fmt == O.MXFP4 else 16
+    if fmt == O.MXFP4:
+        s = torch.from_numpy(scales.copy()).view(torch.float8_e8m0fnu).double().numpy()
+    else:
+        s = torch.from_numpy(scales.copy()).view(torch.float8_e4m3fn).double().numpy()
+    return val * np.repeat(s, block, axis=1)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_fp4_gemm_matches_independent_dequant(fmt):
+    rng = np.random.default_rng(103)
+    M, N, K = 40, 24, 256
+    xa = (rng.standard_normal((M, K)) * 0.5).astype(np.float32)
+    xb = (rng.standard_t(4, (N, K)) * 0.02).astype(np.float32)
+    aa = O.alpha(xa) if fmt == O.NVFP4 else 0.0
+    ab = O.alpha(xb) if fmt == O.NVFP4 else 0.0
+    ea = O.fwd(xa, fmt, alpha=aa, want_y=False, want_codes=True)
+    eb = O.fwd(xb, fmt, alpha=ab, want_y=False, want_codes=True)
+    d = O.fp4_gemm(ea["codes"], ea["scales"], eb["codes"], eb["scales"], fmt, aa, ab)
+    ref = _dequant_independent(ea["codes"], ea["scales"], fmt) @ \
+        _dequant_independent(eb["codes"], eb["scales"], fmt).T
+    if fmt == O.NVFP4:
+        ref = ref * (float(np.float32(aa)) * float(np.float32(ab)))
+    np.testing.assert_allclose(d, ref, rtol=1e-14, atol=0)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_fp4_gemm_is_the_product_of_fake_quantized_operands(fmt):
+    """W4A4 on the export equals the product of the fake-quantized tensors:
+    exactly for MXFP4 (y = q 2^e has no rounding); for NVFP4 up to the
+    rounding of fl(alpha * Delta) in y (2^-23 relative per product)."""
+    rng = np.random.default_rng(107)
+    M, N, K = 32, 48, 512
+    xa = (rng.standard_normal((M, K))).astype(np.float32)
+    xb = (rng.standard_normal((N, K)) * 0.02).astype(np.float32)
+    ca = rng.uniform(0.9, 1.1, (M, K // O.default_block(fmt))).astype(np.float32)
+    aa = O.alpha(xa) if fmt == O.NVFP4 else 0.0
+    ab = O.alpha(xb) if fmt == O.NVFP4 else 0.0
+    fa = O.fwd(xa, fmt, crs=ca, alpha=aa, want_codes=True)
+    fb = O.fwd(xb, fmt, alpha=ab, want_codes=True)
+    d = O.fp4_gemm(fa["codes"], fa["scales"], fb["codes"], fb["scales"], fmt, aa, ab)
+    ya, yb = fa["y"].astype(np.float64), fb["y"].astype(np.float64)
+    if fmt == O.MXFP4:
+        np.testing.assert_allclose(d, ya @ yb.T, rtol=1e-13, atol=0)
+    else:
+        bound = 2.0 ** -22 * (np.abs(ya) @ np.abs(yb).T)
+        assert np.all(np.abs(d - ya @ yb.T) <= bound)

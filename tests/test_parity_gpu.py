@@ -340,3 +340,32 @@ def test_absmax_sfp_matches_absmax_path_on_gpu(fmt):
     assert torch.equal(r0[1], r1[1]) and torch.equal(r0[3], r1[3])
     rb = O.bwd(x, g, f, crs=crs, alpha=a, want_abs=True, want_gsfp=True)
     assert_grad_close(host(r0[3]), rb["gsfp"], rb["gsfp_abs"], FLOOR_ROW, "dL/dS^fp at absmax")
+
+
+# ---------------------------------------------------------------------------
+# export in the block-scaled MMA scale-factor layout
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("rows,cols", [(256, 512), (300, 96), (1, 48 * 2), (129, 1216)])
+def test_pack_mma_layout(fmt, dtype, rows, cols):
+    f = FMT[fmt]
+    block = 32 if f == O.MXFP4 else 16
+    if cols % block:
+        cols = cols * 2
+    w, x, g = seeded(rows, cols, dtype, seed=rows + cols)
+    crs = W.draw_coefs(w, rows * cols // block, 21).reshape(rows, -1)
+    dgs = W.draw_coefs(w, rows * cols // 8, 22).reshape(rows, -1)
+    xd, cd, dd = dev(x), dev(crs), dev(dgs)
+    a = O.alpha(x) if f == O.NVFP4 else 0.0
+    a_dev = torch.tensor([a], dtype=torch.float32, device="cuda") if f == O.NVFP4 else None
+    # poison the tile buffer: padding must come back as zeros
+    desc = F.make_desc(xd, f, 8)
+    tiles = torch.full((F.focus_mma_scale_bytes(desc),), 0xA5, dtype=torch.uint8, device="cuda")
+    codes, tiles = F.focus_pack_mma(xd, f, cd, dd, a_dev, scale_tiles=tiles)
+    codes_rm, scales_rm = F.focus_pack(xd, f, cd, dd, a_dev)
+    torch.cuda.synchronize()
+    ref = O.fwd(x, f, crs=crs, dgs=dgs, alpha=a, want_y=False, want_codes=True)
+    assert_bits_equal(host(codes), ref["codes"], "codes (mma export)")
+    assert_bits_equal(host(codes_rm), ref["codes"], "codes (row-major export)")
+    assert_bits_equal(host(tiles), O.mma_scale_tiles(ref["scales"]), "scale tiles")
