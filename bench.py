@@ -572,6 +572,94 @@ def reference_arm(case, args):
 
 
 # ----------------------------------------------------------------------------
+# ----------------------------------------------------------------------------
+# W4A4 GEMM on the exported operands (tensor cores)
+# ----------------------------------------------------------------------------
+GEMM_TOKENS = 8192          # activation rows: 4 sequences of 2048 tokens
+FP4_PER_BF16 = 13.5 / 2.25  # nominal dense FP4 / BF16 tensor rate of GB300
+
+
+def gemm_arm(args, device):
+    """One step = the layer's projections as W4A4 GEMMs on their exports:
+    D[T, out] = A[T, in] W[out, in]^T with A the activations and W the
+    weights, both exported by focus_pack_mma (timed region: the GEMMs only,
+    bf16 output)."""
+    import torch
+    from paper_2608_01847_gb300 import focus as F
+    from paper_2608_01847_gb300 import workloads as W
+    fmt = F.FOCUS_NVFP4 if args.fmt == "nvfp4" else F.FOCUS_MXFP4
+    w = W.WORKLOADS[args.workload]
+    gen = torch.Generator(device=device)
+    gen.manual_seed(4321)
+    acts, jobs, flops = {}, [], 0
+    for i, t in enumerate(w.tensors):
+        wx, _ = W.device_tensor(w, i, device)
+        K = t.cols
+        if K not in acts:
+            a = torch.randn((GEMM_TOKENS, K), generator=gen, device=device).to(torch.bfloat16)
+            aa = F.focus_nvfp4_alpha(a) if fmt == F.FOCUS_NVFP4 else None
+            acts[K] = (*F.focus_pack_mma(a, fmt, alpha=aa), aa)
+            del a
+        wa = F.focus_nvfp4_alpha(wx) if fmt == F.FOCUS_NVFP4 else None
+        wc, wt = F.focus_pack_mma(wx, fmt, alpha=wa)
+        del wx
+        d = torch.empty((GEMM_TOKENS, t.rows), dtype=torch.bfloat16, device=device)
+        jobs.append((acts[K], (wc, wt, wa), d))
+        flops += 2 * GEMM_TOKENS * t.rows * K
+    flag = torch.zeros(1, dtype=torch.int32, device=device)
+
+    def step():
+        for (ac, at, aa), (wc, wt, wa), d in jobs:
+            F.focus_fp4_gemm(fmt, ac, at, wc, wt, aa, wa, d=d, timeout_flag=flag)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(device)
+    stream = torch.cuda.current_stream(device)
+    per = []
+    with ClockSampler(device.index if device.index is not None else 0) as clk:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize(device)
+    ms = e0.elapsed_time(e1) / args.steps
+    # dominant launch: the largest projection alone
+    big = max(range(len(jobs)), key=lambda j: jobs[j][2].numel() * w.tensors[j].cols)
+    (ac, at, aa), (wc, wt, wa), d = jobs[big]
+    n_rep = max(3, min(args.steps, 50))
+    e0.record(stream)
+    for _ in range(n_rep):
+        F.focus_fp4_gemm(fmt, ac, at, wc, wt, aa, wa, d=d, timeout_flag=flag)
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    big_ms = e0.elapsed_time(e1) / n_rep
+    big_flops = 2 * GEMM_TOKENS * w.tensors[big].rows * w.tensors[big].cols
+    assert int(flag.item()) == 0, "a GEMM wait gave up"
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            bf16 = float(json.load(f)["bf16_tflops"])
+        peak_kind = "measured bf16 burst x nominal FP4/BF16 ratio 6"
+    except Exception:
+        bf16, peak_kind = 1900.0, "fallback bf16 x nominal FP4/BF16 ratio 6"
+    peak = bf16 * FP4_PER_BF16
+    tflops = flops / (ms * 1e-3) / 1e12
+    big_tflops = big_flops / (big_ms * 1e-3) / 1e12
+    return {
+        "metric": "W4A4 FP4 GEMM TFLOP/s on FOCUS exports", "value": round(tflops, 1), "unit": "TFLOP/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "e2m1", "data": "synthetic",
+        "config": {"workload": f"{args.workload} projections x {GEMM_TOKENS} tokens", "fmt": args.fmt,
+                   "gemms": [[GEMM_TOKENS, t.rows, t.cols] for t in w.tensors], "out": "bf16",
+                   "l2": "operands of one GEMM fit in L2 (weights <= 25 MB of codes); outputs stream"},
+        "roofline": {"bound": "tensor", "kernel": f"fp4_gemm_kernel ({w.tensors[big].name})",
+                     "achieved": round(big_tflops, 1), "peak": round(peak, 1), "peak_kind": peak_kind,
+                     "unit": "TFLOP/s", "frac": round(big_tflops / peak, 4), "traffic": None},
+        "clocks": clk.summary(), "gpu_launches": args.steps * len(jobs),
+    }
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -586,6 +674,8 @@ def main():
                     help="learnable full-precision scales S^fp and their gradient")
     ap.add_argument("--adam", action="store_true",
                     help="backward fused with the AdamW step on the learned arrays")
+    ap.add_argument("--gemm", action="store_true",
+                    help="time the W4A4 FP4 GEMMs of the workload's projections on their exports")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
@@ -616,6 +706,10 @@ def main():
         dist.barrier()
         build()
 
+    if args.gemm:
+        if rank == 0:
+            print(json.dumps(gemm_arm(args, device)))
+        return
     r = gpu_arm(case, args, rank, world, device)
     if rank != 0:
         if world > 1:

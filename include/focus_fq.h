@@ -273,16 +273,18 @@ size_t focus_mma_scale_bytes(const focus_desc_t* desc);
  * focus_pack_mma (B is the second operand's rows, e.g. a weight [out, in]);
  * a_scale_tiles / b_scale_tiles: their MMA-layout scale tiles; alpha_a,
  * alpha_b: device fp32 per-tensor scales (NVFP4 only; ignored for MXFP4).
- * d: [M, ldd] row-major fp32 output (ldd >= N), overwritten.  The products
- * are exact and accumulate in fp32 inside the tensor core.
+ * d: [M, ldd] row-major output (ldd >= N) of d_dtype (FOCUS_F32, or
+ * FOCUS_BF16 rounded to nearest even), overwritten.  The products are exact
+ * and accumulate in fp32 inside the tensor core; alpha is applied to the
+ * fp32 sum before the output rounding.
  * Requirements: K % 64 == 0 (FOCUS_ERR_UNSUPPORTED otherwise); codes and
  * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
  * kernel whose wait for its MMAs gives up sets it to 1 (the output is then
  * not written) instead of waiting for ever.  Enqueued on `stream`. */
 int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
                    const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
-                   const uint8_t* b_scale_tiles, const float* alpha_b, float* d, int64_t ldd,
-                   int32_t* timeout_flag, focus_stream_t stream);
+                   const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,
+                   int64_t ldd, int32_t* timeout_flag, focus_stream_t stream);
 
 /* Device scratch (bytes) that focus_nvfp4_alpha (which = FOCUS_WS_ALPHA) or
  * focus_fq_bwd (which = FOCUS_WS_BWD) needs for this descriptor on the

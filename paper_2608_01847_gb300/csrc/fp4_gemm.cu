@@ -6,23 +6,33 @@
 // the paper's "no inference overhead" refers to (Sec. 1, Sec. 3.1): only the
 // exported codes and hardware scales enter the product.
 //
-// One CTA (4 warps) per 128 x 128 tile of D; K in chunks of 256 elements
-// (128 bytes of codes per row = four K = 64 MMA steps).  Per chunk the CTA
-// stages the A and B code tiles in shared memory (K-major, 8 x 16-byte core
-// matrices), writes the four steps' scale words to tensor memory, and one
-// thread issues the MMAs; the accumulator lives in tensor memory and is read
-// back once at the end.
+// Persistent, warp-specialised kernel, one CTA per SM, 128 x 128 tiles of D:
+//   warp 0     TMA producer: per K chunk of 256 elements (128 bytes of codes
+//              per row) the A and B code tiles (2D TMA, 128-byte swizzle)
+//              and their scale tiles (1D bulk copies) into a ring of stages;
+//   warp 1     MMA issuer: scale tiles shared -> tensor memory (tcgen05.cp),
+//              four K = 64 block-scaled MMAs per chunk into an accumulator
+//              in tensor memory, commit to free the stage;
+//   warps 2-5  epilogue: accumulator -> registers (one lane quarter each),
+//              alpha scaling, fp32 or bf16 stores.
+// Two accumulators in tensor memory let the epilogue of one tile overlap
+// the main loop of the next.
 //
-// Scale factors in tensor memory (M = N = 128, one CTA): an MMA step reads a
+// Scale factors in tensor memory (M = N = 128): one MMA step reads a
 // 4-column region; row m of A takes lane m, column m / 32; column n of B is
-// read by each 32-lane quarter of the data path from its own quarter, lane
-// n % 32, column n / 32.  So lane l of every quarter holds, in the region's
-// four columns, the scale words of rows l, l + 32, l + 64, l + 96 -- which is
-// exactly 16-byte line l of a 128 x 4 export tile.  Each word holds the
-// scales of consecutive K blocks in byte order (NVFP4: four 16-element
-// blocks; MXFP4: two 32-element blocks in bytes 0-1).
+// read by each 32-lane quarter from its own quarter, lane n % 32, column
+// n / 32.  Lane l of every quarter must therefore hold, in the four
+// columns, the scale words of rows l, l + 32, l + 64, l + 96: exactly line l
+// of a 128 x 4 export tile, which tcgen05.cp .32x128b.warpx4 broadcasts to
+// all four quarters.  A word holds consecutive K blocks in byte order: one
+// NVFP4 step uses all four bytes, an MXFP4 tile feeds two steps (bytes 0-1,
+// then bytes 2-3 through the scale data id).
 #include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <algorithm>
+#include <mutex>
 
 #include "../../include/focus_fq.h"
 #include "tc_ptx.cuh"
@@ -32,143 +42,235 @@
 namespace focus {
 namespace {
 
-constexpr int kGemmThreads = 128;
-constexpr int kTile = 128;          // M and N of one CTA
-constexpr int kChunkBytes = 128;    // K bytes (256 FP4) per chunk
-// tensor memory: D in columns 0-127; the scale regions of the chunk's four
-// MMA steps at 128 + 16 kk (A) and 192 + 16 kk (B), each 4 columns.  An
-// MMA's scale address must be aligned (a region starting at an odd column
-// raises a misaligned-address error); 16-column steps keep every region on
-// a 16-column boundary.
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kSfa = 128, kSfb = 192, kSfStep = 16;
+constexpr int kTile = 128;            // M and N of a CTA tile
+constexpr int kChunk = 128;           // K bytes (256 FP4) per stage
+constexpr int kStages = 5;
+constexpr int kTileBytes = kTile * kChunk;          // 16 KB of codes per operand
+constexpr int kSfBytes = 4 * 512;                   // up to four scale tiles per operand
+constexpr int kStageBytes = 2 * kTileBytes + 2 * kSfBytes;
+constexpr int kSmemBytes = kStages * kStageBytes + 1024;   // + alignment slack
+constexpr int kThreads = 192;         // producer, MMA, four epilogue warps
+// tensor memory: accumulators in columns 0-127 and 128-255; scale regions
+// for the four steps of a chunk at 256 + 16 j (A) and 320 + 16 j (B), each
+// 4 columns (every region on a 16-column boundary).
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kSfa = 256, kSfb = 320, kSfStep = 16;
 constexpr uint32_t kWaitLimit = 1u << 22;
 
 struct GemmParams {
-    const uint8_t* a;      // [M, K/2] codes
     const uint8_t* sfa;    // scale tiles of A
-    const uint8_t* b;      // [N, K/2] codes
     const uint8_t* sfb;    // scale tiles of B
-    const float* alpha_a;  // NVFP4 per-tensor scales (device), else null
+    const float* alpha_a;  // NVFP4 per-tensor scales (device)
     const float* alpha_b;
-    float* d;              // [M, ldd] fp32
-    int32_t* flag;         // set to 1 if an MMA completion wait gave up
-    int64_t M, N, K, ldd;
+    void* d;               // [M, ldd] fp32 or bf16
+    int32_t* flag;         // set to 1 if a wait gave up
+    int64_t M, N, ldd;
     uint32_t tiles_k;      // scale tiles per 128-row tile row: ceil(K / block / 4)
+    uint32_t tiles_m, tiles_n;
+    uint32_t n_steps;      // K / 64
+    int d_bf16;
+    int d_vec;             // rows of D start on 16-byte boundaries (vector stores)
 };
 
-template <int FMT>
-__global__ void __launch_bounds__(kGemmThreads) fp4_gemm_kernel(const GemmParams p)
+__device__ __forceinline__ void give_up(const GemmParams& p)
 {
-    __shared__ __align__(1024) uint8_t sA[kTile * kChunkBytes];
-    __shared__ __align__(1024) uint8_t sB[kTile * kChunkBytes];
-    __shared__ __align__(8) uint64_t bar;
+    if (p.flag) atomicOr(p.flag, 1);
+}
+
+template <int FMT>
+__global__ void __launch_bounds__(kThreads, 1)
+    fp4_gemm_kernel(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
+                    const GemmParams p)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2];
     __shared__ uint32_t tbase;
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    auto stage_a = [&](uint32_t s) { return smem + s * kStageBytes; };
+    auto stage_b = [&](uint32_t s) { return smem + s * kStageBytes + kTileBytes; };
+    auto stage_sfa = [&](uint32_t s) { return smem + s * kStageBytes + 2 * kTileBytes; };
+    auto stage_sfb = [&](uint32_t s) { return smem + s * kStageBytes + 2 * kTileBytes + kSfBytes; };
 
-    const int t = threadIdx.x, warp = t / 32, lane = t % 32;
-    const int64_t m0 = static_cast<int64_t>(blockIdx.y) * kTile;
-    const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kTile;
-    const int64_t row_bytes = p.K / 2;
-
-    if (t == 0) tc::mbar_init(&bar, 1);
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            tc::mbar_init(&acc_full[b], 1);
+            tc::mbar_init(&acc_empty[b], 128);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
     if (warp == 0) {
         tc::tmem_alloc(&tbase, kTmemCols);
         tc::tmem_relinquish();
     }
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = tbase;
-    const uint32_t lane_addr = tb + (static_cast<uint32_t>(warp * 32) << 16);
-    constexpr uint32_t idesc = tc::idesc_fp4(kTile, kTile, FMT == 0);
 
-    const int64_t n_chunks = (row_bytes + kChunkBytes - 1) / kChunkBytes;
-    bool ok = true;
-    for (int64_t c = 0; c < n_chunks && ok; ++c) {
-        const int64_t kb0 = c * kChunkBytes;
-        const int64_t left = row_bytes - kb0;
-        const int n_mma = static_cast<int>((left < kChunkBytes ? left : kChunkBytes) / 32);
-        // ---- code tiles: thread t stages row t of A and of B ----
-#pragma unroll
-        for (int j = 0; j < kChunkBytes / 16; ++j) {
-            uint4 va = make_uint4(0u, 0u, 0u, 0u), vb = va;
-            if (j < 2 * n_mma) {
-                if (m0 + t < p.M)
-                    va = __ldg(reinterpret_cast<const uint4*>(p.a + (m0 + t) * row_bytes + kb0) + j);
-                if (n0 + t < p.N)
-                    vb = __ldg(reinterpret_cast<const uint4*>(p.b + (n0 + t) * row_bytes + kb0) + j);
-            }
-            const int off = (t / 8) * 1024 + j * 128 + (t % 8) * 16;
-            *reinterpret_cast<uint4*>(sA + off) = va;
-            *reinterpret_cast<uint4*>(sB + off) = vb;
-        }
-        // ---- scale words: line `lane` of the step's export tile, all quarters ----
-        for (int kk = 0; kk < n_mma; ++kk) {
-            const int64_t g = c * 4 + kk;                  // global K = 64 step
-            const int64_t tj = FMT == 0 ? g / 2 : g;       // tile column (4 scale columns)
-            const int shift = FMT == 0 ? 16 * static_cast<int>(g % 2) : 0;
-            const uint4 la = __ldg(reinterpret_cast<const uint4*>(
-                p.sfa + ((m0 / kTile) * p.tiles_k + tj) * 512 + 16 * lane));
-            const uint4 lb = __ldg(reinterpret_cast<const uint4*>(
-                p.sfb + ((n0 / kTile) * p.tiles_k + tj) * 512 + 16 * lane));
-            tc::tmem_st_x4(lane_addr + kSfa + kSfStep * kk, la.x >> shift, la.y >> shift,
-                           la.z >> shift, la.w >> shift);
-            tc::tmem_st_x4(lane_addr + kSfb + kSfStep * kk, lb.x >> shift, lb.y >> shift,
-                           lb.z >> shift, lb.w >> shift);
-        }
-        tc::tmem_wait_st();
-        tc::fence_async_smem();
-        tc::tc_fence_before();
-        __syncthreads();
-        tc::tc_fence_after();
-        if (t == 0) {
-            const uint32_t a0 = tc::smem_u32(sA), b0 = tc::smem_u32(sB);
-            for (int kk = 0; kk < n_mma; ++kk) {
-                const uint64_t ad = tc::smem_desc_kmajor(a0 + 256 * kk, 128, 1024);
-                const uint64_t bd = tc::smem_desc_kmajor(b0 + 256 * kk, 128, 1024);
-                const uint32_t acc = (c > 0 || kk > 0) ? 1u : 0u;
-                const uint32_t sfa = tb + kSfa + kSfStep * kk, sfb = tb + kSfb + kSfStep * kk;
-                if (FMT == 0)
-                    tc::mma_mxf4(tb, ad, bd, idesc, sfa, sfb, acc);
-                else
-                    tc::mma_nvf4(tb, ad, bd, idesc, sfa, sfb, acc);
-            }
-            tc::mma_commit(&bar);
-        }
-        // every thread takes the same branch afterwards
-        ok = __syncthreads_and(tc::mbar_wait(&bar, static_cast<uint32_t>(c & 1), kWaitLimit)) != 0;
-        tc::tc_fence_after();
-        if (!ok) {
-            // give the MMAs in flight a second bounded chance to finish before
-            // tensor memory is released
-            tc::mbar_wait(&bar, static_cast<uint32_t>(c & 1), kWaitLimit);
-            if (t == 0 && p.flag) atomicOr(p.flag, 1);
-        }
-    }
+    const uint32_t n_tiles = p.tiles_m * p.tiles_n;
+    const uint32_t n_chunks = (p.n_steps + 3) / 4;
+    constexpr uint32_t steps_per_tile = FMT == 0 ? 2 : 1;   // K steps one scale tile covers
 
-    // ---- epilogue: lane = row, column = n ----
-    if (ok && n_chunks > 0) {
+    if (warp == 0) {
+        // ---------------- TMA producer ----------------
+        if (lane == 0) {
+            uint32_t s = 0, ph = 0;
+            bool ok = true;
+            for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
+                for (uint32_t c = 0; c < n_chunks; ++c) {
+                    if (!tc::mbar_wait(&empty[s], ph ^ 1, kWaitLimit)) {
+                        ok = false;
+                        give_up(p);
+                        break;
+                    }
+                    const uint32_t steps = min(4u, p.n_steps - 4 * c);
+                    const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
+                    const uint32_t tile0 = (4 * c) / steps_per_tile;
+                    tc::mbar_arrive_expect_tx(&full[s], 2 * kTileBytes + 2 * sf_tiles * 512);
+                    tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
+                                    static_cast<int32_t>(tm * kTile), &full[s]);
+                    tc::tma_load_2d(stage_b(s), &tma_b, static_cast<int32_t>(c * kChunk),
+                                    static_cast<int32_t>(tn * kTile), &full[s]);
+                    tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
+                                  sf_tiles * 512, &full[s]);
+                    tc::bulk_load(stage_sfb(s), p.sfb + (static_cast<size_t>(tn) * p.tiles_k + tile0) * 512,
+                                  sf_tiles * 512, &full[s]);
+                    if (++s == kStages) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------- MMA issuer ----------------
+        if (lane == 0) {
+            uint32_t s = 0, ph = 0, acc = 0, acc_ph = 0;
+            bool ok = true;
+            for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                if (!tc::mbar_wait(&acc_empty[acc], acc_ph ^ 1, kWaitLimit)) {
+                    give_up(p);
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t d_tmem = tb + acc * kTile;
+                for (uint32_t c = 0; c < n_chunks; ++c) {
+                    if (!tc::mbar_wait(&full[s], ph, kWaitLimit)) {
+                        ok = false;
+                        give_up(p);
+                        break;
+                    }
+                    tc::tc_fence_after();
+                    const uint32_t steps = min(4u, p.n_steps - 4 * c);
+                    const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
+                    const uint32_t sa = tc::smem_u32(stage_sfa(s)), sb = tc::smem_u32(stage_sfb(s));
+                    for (uint32_t j = 0; j < sf_tiles; ++j) {
+                        tc::tmem_cp_32x128b_x4(tb + kSfa + kSfStep * j, sa + 512 * j);
+                        tc::tmem_cp_32x128b_x4(tb + kSfb + kSfStep * j, sb + 512 * j);
+                    }
+                    const uint32_t a0 = tc::smem_u32(stage_a(s)), b0 = tc::smem_u32(stage_b(s));
+                    for (uint32_t kk = 0; kk < steps; ++kk) {
+                        const uint64_t ad = tc::smem_desc_sw128(a0 + 32 * kk);
+                        const uint64_t bd = tc::smem_desc_sw128(b0 + 32 * kk);
+                        const uint32_t j = kk / steps_per_tile;
+                        const uint32_t sfa = tb + kSfa + kSfStep * j, sfb = tb + kSfb + kSfStep * j;
+                        const uint32_t accumulate = (c > 0 || kk > 0) ? 1u : 0u;
+                        if (FMT == 0)
+                            tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTile, true, 2 * (kk % 2)), sfa, sfb,
+                                         accumulate);
+                        else
+                            tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTile, false), sfa, sfb,
+                                         accumulate);
+                    }
+                    tc::mma_commit(&empty[s]);
+                    if (++s == kStages) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                }
+                if (!ok) break;
+                tc::mma_commit(&acc_full[acc]);
+                if (++acc == 2) {
+                    acc = 0;
+                    acc_ph ^= 1;
+                }
+            }
+        }
+    } else {
+        // ---------------- epilogue (warps 2-5: lane quarters 2, 3, 0, 1) ----------------
+        const uint32_t q = warp % 4;
+        const uint32_t lane_addr = tb + ((q * 32) << 16);
         const float scale = FMT == 1 ? __fmul_rn(__ldg(p.alpha_a), __ldg(p.alpha_b)) : 1.0f;
-        const int64_t m = m0 + warp * 32 + lane;
+        uint32_t acc = 0, acc_ph = 0;
+        for (uint32_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
+            const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
+            const bool got = __all_sync(0xffffffffu, tc::mbar_wait(&acc_full[acc], acc_ph, kWaitLimit));
+            if (!got) {
+                if (lane == 0) give_up(p);
+                break;
+            }
+            tc::tc_fence_after();
+            const int64_t m = static_cast<int64_t>(tm) * kTile + q * 32 + lane;
+            const int64_t n0 = static_cast<int64_t>(tn) * kTile;
 #pragma unroll 1
-        for (int q = 0; q < kTile / 32; ++q) {
-            uint32_t r[32];
-            tc::tmem_ld_x32(lane_addr + 32 * q, r);
-            tc::tmem_wait_ld();
-            if (m < p.M) {
-                float* dst = p.d + m * p.ldd + n0 + 32 * q;
+            for (int cb = 0; cb < kTile / 32; ++cb) {
+                uint32_t r[32];
+                tc::tmem_ld_x32(lane_addr + acc * kTile + 32 * cb, r);
+                tc::tmem_wait_ld();
+                if (cb == kTile / 32 - 1) {
+                    // the accumulator is free once its last columns are in registers
+                    tc::tc_fence_before();
+                    tc::mbar_arrive(&acc_empty[acc]);
+                }
+                if (m < p.M) {
+                    const int64_t nb = n0 + 32 * cb;
+                    if (p.d_bf16) {
+                        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.d) + m * p.ldd + nb;
+                        if (nb + 32 <= p.N && p.d_vec) {
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (n0 + 32 * q + i < p.N) dst[i] = __fmul_rn(__uint_as_float(r[i]), scale);
+                            for (int i = 0; i < 32; i += 8) {
+                                uint32_t w[4];
+#pragma unroll
+                                for (int e = 0; e < 4; ++e) {
+                                    const __nv_bfloat162 h = __floats2bfloat162_rn(
+                                        __fmul_rn(__uint_as_float(r[i + 2 * e]), scale),
+                                        __fmul_rn(__uint_as_float(r[i + 2 * e + 1]), scale));
+                                    w[e] = *reinterpret_cast<const uint32_t*>(&h);
+                                }
+                                *reinterpret_cast<uint4*>(dst + i) = make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                        } else {
+                            for (int i = 0; i < 32 && nb + i < p.N; ++i)
+                                dst[i] = __float2bfloat16_rn(__fmul_rn(__uint_as_float(r[i]), scale));
+                        }
+                    } else {
+                        float* dst = static_cast<float*>(p.d) + m * p.ldd + nb;
+                        if (nb + 32 <= p.N && p.d_vec) {
+#pragma unroll
+                            for (int i = 0; i < 32; i += 4)
+                                *reinterpret_cast<float4*>(dst + i) =
+                                    make_float4(__fmul_rn(__uint_as_float(r[i]), scale),
+                                                __fmul_rn(__uint_as_float(r[i + 1]), scale),
+                                                __fmul_rn(__uint_as_float(r[i + 2]), scale),
+                                                __fmul_rn(__uint_as_float(r[i + 3]), scale));
+                        } else {
+                            for (int i = 0; i < 32 && nb + i < p.N; ++i)
+                                dst[i] = __fmul_rn(__uint_as_float(r[i]), scale);
+                        }
+                    }
+                }
+            }
+            if (++acc == 2) {
+                acc = 0;
+                acc_ph ^= 1;
             }
         }
-    } else if (n_chunks == 0) {
-        // K = 0: D = 0
-        const int64_t m = m0 + warp * 32 + lane;
-        if (m < p.M)
-            for (int i = 0; i < kTile; ++i)
-                if (n0 + i < p.N) p.d[m * p.ldd + n0 + i] = 0.0f;
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -176,7 +278,76 @@ __global__ void __launch_bounds__(kGemmThreads) fp4_gemm_kernel(const GemmParams
     if (warp == 0) tc::tmem_dealloc(tb, kTmemCols);
 }
 
+// D = 0 (K = 0: every sum is empty).
+__global__ void zero_kernel(void* d, int64_t M, int64_t N, int64_t ldd, int bf16)
+{
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (i >= M * N) return;
+    const int64_t m = i / N, n = i % N;
+    if (bf16)
+        static_cast<__nv_bfloat16*>(d)[m * ldd + n] = __float2bfloat16_rn(0.0f);
+    else
+        static_cast<float*>(d)[m * ldd + n] = 0.0f;
+}
+
 bool misaligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; }
+
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encode_fn()
+{
+    static EncodeTiled fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiled>(f);
+    });
+    return fn;
+}
+
+// Tensor map of a [rows, row_bytes] code matrix, boxes of 128 rows x 128
+// bytes, 128-byte swizzle, zero fill outside.
+bool make_map(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t row_bytes)
+{
+    EncodeTiled fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(row_bytes), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
+    const cuuint32_t box[2] = {kChunk, kTile};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(codes), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int device_sm_count()
+{
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 1;
+    return n;
+}
+
+template <int FMT>
+cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, cudaStream_t st)
+{
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(fp4_gemm_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    });
+    if (attr != cudaSuccess) return attr;
+    const uint32_t tiles = p.tiles_m * p.tiles_n;
+    const uint32_t grid = std::min<uint32_t>(tiles, static_cast<uint32_t>(device_sm_count()));
+    fp4_gemm_kernel<FMT><<<grid, kThreads, kSmemBytes, st>>>(ma, mb, p);
+    return cudaGetLastError();
+}
 
 }  // namespace
 }  // namespace focus
@@ -185,25 +356,34 @@ using namespace focus;
 
 FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
                              const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
-                             const uint8_t* b_scale_tiles, const float* alpha_b, float* d, int64_t ldd,
-                             int32_t* timeout_flag, focus_stream_t stream)
+                             const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,
+                             int64_t ldd, int32_t* timeout_flag, focus_stream_t stream)
 {
     if (fmt != FOCUS_MXFP4 && fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;
+    if (d_dtype != FOCUS_F32 && d_dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
     if (M < 0 || N < 0 || K < 0 || ldd < N) return FOCUS_ERR_INVALID_ARG;
     if (K % 64 != 0) return FOCUS_ERR_UNSUPPORTED;
-    if (M > (int64_t(1) << 31) - kTile || N > (int64_t(65535) * kTile)) return FOCUS_ERR_UNSUPPORTED;
+    if (M > (int64_t(1) << 31) - kTile || N > (int64_t(1) << 31) - kTile || K > (int64_t(1) << 31))
+        return FOCUS_ERR_UNSUPPORTED;
     if (M == 0 || N == 0) return FOCUS_OK;
-    if (!d || (K > 0 && (!a_codes || !b_codes || !a_scale_tiles || !b_scale_tiles)))
-        return FOCUS_ERR_INVALID_ARG;
+    if (!d) return FOCUS_ERR_INVALID_ARG;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const int bf16 = d_dtype == FOCUS_BF16;
+    if (misaligned(d, bf16 ? 2 : 4) || misaligned(timeout_flag, 4)) return FOCUS_ERR_MISALIGNED;
+    if (K == 0) {
+        const int64_t n = M * N;
+        zero_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, st>>>(d, M, N, ldd, bf16);
+        return cudaGetLastError() == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA;
+    }
+    if (!a_codes || !b_codes || !a_scale_tiles || !b_scale_tiles) return FOCUS_ERR_INVALID_ARG;
     if (fmt == FOCUS_NVFP4 && (!alpha_a || !alpha_b)) return FOCUS_ERR_INVALID_ARG;
     if (misaligned(a_codes, 16) || misaligned(b_codes, 16) || misaligned(a_scale_tiles, 16) ||
-        misaligned(b_scale_tiles, 16) || misaligned(d, 4) || misaligned(alpha_a, 4) ||
-        misaligned(alpha_b, 4) || misaligned(timeout_flag, 4))
+        misaligned(b_scale_tiles, 16) || misaligned(alpha_a, 4) || misaligned(alpha_b, 4))
         return FOCUS_ERR_MISALIGNED;
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, a_codes, M, K / 2) || !make_map(&mb, b_codes, N, K / 2)) return FOCUS_ERR_CUDA;
     GemmParams p;
-    p.a = a_codes;
     p.sfa = a_scale_tiles;
-    p.b = b_codes;
     p.sfb = b_scale_tiles;
     p.alpha_a = alpha_a;
     p.alpha_b = alpha_b;
@@ -211,15 +391,14 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
     p.flag = timeout_flag;
     p.M = M;
     p.N = N;
-    p.K = K;
     p.ldd = ldd;
     const int64_t block = fmt == FOCUS_MXFP4 ? 32 : 16;
     p.tiles_k = static_cast<uint32_t>((K / block + 3) / 4);
-    const dim3 grid(static_cast<uint32_t>((N + kTile - 1) / kTile), static_cast<uint32_t>((M + kTile - 1) / kTile));
-    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    if (fmt == FOCUS_MXFP4)
-        fp4_gemm_kernel<0><<<grid, kGemmThreads, 0, st>>>(p);
-    else
-        fp4_gemm_kernel<1><<<grid, kGemmThreads, 0, st>>>(p);
-    return cudaGetLastError() == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA;
+    p.tiles_m = static_cast<uint32_t>((M + kTile - 1) / kTile);
+    p.tiles_n = static_cast<uint32_t>((N + kTile - 1) / kTile);
+    p.n_steps = static_cast<uint32_t>(K / 64);
+    p.d_bf16 = bf16;
+    p.d_vec = !misaligned(d, 16) && (ldd * (bf16 ? 2 : 4)) % 16 == 0;
+    const cudaError_t e = fmt == FOCUS_MXFP4 ? launch<0>(ma, mb, p, st) : launch<1>(ma, mb, p, st);
+    return e == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA;
 }

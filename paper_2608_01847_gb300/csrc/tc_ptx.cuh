@@ -44,6 +44,40 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
     return false;
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Arrive once and expect `bytes` of asynchronous copies on this phase.
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+// ---- TMA ------------------------------------------------------------------------
+// 2D tile of a tensor map into shared memory; completes `bytes` on `bar`.
+// x (innermost coordinate, in elements of the map) must be a multiple of 16
+// bytes.
+__device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, int32_t x, int32_t y, uint64_t* bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Contiguous bulk copy global -> shared (16-byte aligned, size % 16 == 0).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+
 // ---- proxy / tcgen05 ordering -----------------------------------------------
 // generic-proxy writes to shared memory -> visible to the tensor core (async proxy)
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
@@ -111,16 +145,44 @@ __device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t saddr, uint32_t lb
     return d;
 }
 
+// K-major operand in 128-byte swizzled rows (as a TMA SWIZZLE_128B load
+// writes them): 8-row groups 1024 bytes apart; the tile must be 1024-byte
+// aligned, and a K offset inside the 128-byte row is added to the start.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);          // start address
+    d |= static_cast<uint64_t>(1) << 16;                          // leading offset (unused)
+    d |= static_cast<uint64_t>(1024 >> 4) << 32;                  // stride: 8 rows x 128 B
+    d |= static_cast<uint64_t>(1) << 46;                          // descriptor version 1
+    d |= static_cast<uint64_t>(2) << 61;                          // 128-byte swizzle
+    return d;
+}
+
+// Scale factors: shared memory -> tensor memory, 32 rows x 16 bytes (one
+// 128 x 4 export tile, line l = row l), copied to lane l of all four lane
+// quarters, columns taddr .. taddr + 3.  Ordered before later MMAs issued
+// by the same thread.
+__device__ __forceinline__ void tmem_cp_32x128b_x4(uint32_t taddr, uint32_t saddr)
+{
+    const uint64_t desc = smem_desc_kmajor(saddr, 16, 128);
+    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
+}
+
 // Instruction descriptor of the block-scaled FP4 MMA (.kind::mxf4 and
 // .kind::mxf4nvf4): both operands E2M1 (format 1), K-major, dense, scale
 // factor data ids 0; `ue8m0` selects E8M0 (MXFP4) over E4M3 (NVFP4) scales.
-__host__ __device__ constexpr uint32_t idesc_fp4(uint32_t m, uint32_t n, bool ue8m0)
+// `sf_id` picks the scale bytes inside each 32-bit scale word (0, or 2 for
+// the second K step of an MXFP4 tile).
+__host__ __device__ constexpr uint32_t idesc_fp4(uint32_t m, uint32_t n, bool ue8m0, uint32_t sf_id = 0)
 {
-    return (1u << 7)                       // bits 7-9: A format E2M1
+    return (sf_id << 4)                    // bits 4-5: B scale factor data id
+           | (1u << 7)                     // bits 7-9: A format E2M1
            | (1u << 10)                    // bits 10-12: B format E2M1
            | ((n >> 3) << 17)              // bits 17-22: N / 8
            | ((ue8m0 ? 1u : 0u) << 23)     // bit 23: scale type (0 UE4M3, 1 UE8M0)
-           | ((m >> 4) << 24);             // bits 24-28: M / 16
+           | ((m >> 4) << 24)              // bits 24-28: M / 16
+           | (sf_id << 29);                // bits 29-30: A scale factor data id
 }
 
 // D[tmem] (+)= (A * SFA) x (B * SFB)^T for one K = 64 step.

@@ -81,7 +81,7 @@ def lib() -> ctypes.CDLL:
         L.focus_mma_scale_bytes.argtypes = [D]
         L.focus_mma_scale_bytes.restype = SZ
         I32, I64 = ctypes.c_int32, ctypes.c_int64
-        L.focus_fp4_gemm.argtypes = [I32, I64, I64, I64, P, P, P, P, P, P, P, I64, P, P]
+        L.focus_fp4_gemm.argtypes = [I32, I64, I64, I64, P, P, P, P, P, P, P, I32, I64, P, P]
         L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
         L.focus_workspace_bytes.restype = SZ
         L.focus_status_string.argtypes = [ctypes.c_int]
@@ -342,10 +342,11 @@ def focus_pack_mma(x, fmt, crs=None, dgs=None, alpha=None, *, sub_block=8, share
 
 
 def focus_fp4_gemm(fmt, a_codes, a_tiles, b_codes, b_tiles, alpha_a=None, alpha_b=None, *, d=None,
-                   timeout_flag=None):
+                   out_dtype=torch.float32, timeout_flag=None):
     """D = A B^T on the block-scaled FP4 tensor cores from two focus_pack_mma
     exports (codes [M, K/2] and [N, K/2] uint8, their scale tiles); returns
-    D [M, N] fp32.  alpha_a / alpha_b: NVFP4 per-tensor scales ([1] fp32)."""
+    D [M, N] (fp32 or bf16).  alpha_a / alpha_b: NVFP4 per-tensor scales
+    ([1] fp32)."""
     M, kh = a_codes.shape
     N, kh2 = b_codes.shape
     if kh != kh2:
@@ -356,11 +357,13 @@ def focus_fp4_gemm(fmt, a_codes, a_tiles, b_codes, b_tiles, alpha_a=None, alpha_
         if t.dtype != torch.uint8 or not t.is_contiguous():
             raise ValueError(f"{name} must be a contiguous uint8 tensor")
     if d is None:
-        d = torch.empty((M, N), dtype=torch.float32, device=a_codes.device)
-    if d.dtype != torch.float32 or d.dim() != 2 or d.shape[0] != M or d.shape[1] != N or d.stride(1) != 1:
-        raise ValueError("d must be a [M, N] fp32 tensor with unit column stride")
+        d = torch.empty((M, N), dtype=out_dtype, device=a_codes.device)
+    if d.dtype not in (torch.float32, torch.bfloat16) or d.dim() != 2 or d.shape[0] != M or \
+            d.shape[1] != N or (M > 0 and N > 0 and d.stride(1) != 1):
+        raise ValueError("d must be a [M, N] fp32 or bf16 tensor with unit column stride")
+    dt = FOCUS_BF16 if d.dtype == torch.bfloat16 else FOCUS_F32
     _check(lib().focus_fp4_gemm(int(fmt), M, N, K, _p(a_codes), _p(a_tiles), _p(alpha_a),
-                                _p(b_codes), _p(b_tiles), _p(alpha_b), _p(d), d.stride(0),
+                                _p(b_codes), _p(b_tiles), _p(alpha_b), _p(d), dt, max(d.stride(0), N),
                                 _p(timeout_flag), _stream(a_codes.device)), "focus_fp4_gemm")
     return d
 

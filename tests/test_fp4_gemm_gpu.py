@@ -136,3 +136,23 @@ def test_export_read_by_library_gemm(fmt):
     ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], f, aa, ab)
     mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], f, aa, ab)
     assert np.all(np.abs(lib - ref) <= 2.0 ** -7 * np.abs(ref) + 2.0 ** -18 * mag)
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_fp4_gemm_bf16_output(fmt):
+    """bf16 output: the fp32 result rounded to nearest even (within one bf16
+    rounding of the fp32 bound), and odd row pitches take the scalar path."""
+    f = FMT[fmt]
+    M, N, K = 192, 200, 768
+    wa, xa = operand(M, K, 31, "act")
+    wb, xb = operand(N, K, 32, "weight")
+    ac, at, aa_dev, ra, aa = export_both(xa, f, None)
+    bc, bt, ab_dev, rb, ab = export_both(xb, f, None)
+    d32 = F.focus_fp4_gemm(f, ac, at, bc, bt, aa_dev, ab_dev)
+    d16 = F.focus_fp4_gemm(f, ac, at, bc, bt, aa_dev, ab_dev, out_dtype=torch.bfloat16)
+    wide = torch.zeros((M, N + 3), dtype=torch.bfloat16, device="cuda")
+    F.focus_fp4_gemm(f, ac, at, bc, bt, aa_dev, ab_dev, d=wide[:, :N])
+    torch.cuda.synchronize()
+    assert torch.equal(d16, d32.to(torch.bfloat16))
+    assert torch.equal(wide[:, :N], d16)
+    assert torch.count_nonzero(wide[:, N:]) == 0
