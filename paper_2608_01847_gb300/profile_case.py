@@ -36,7 +36,8 @@ def main():
     from paper_2608_01847_gb300 import workloads as W
 
     ap = argparse.ArgumentParser()
-    ap.add_argument("--phase", choices=["alpha", "fwd", "bwd", "pack"], default="bwd")
+    ap.add_argument("--phase", choices=["alpha", "fwd", "bwd", "pack", "gemm"], default="bwd")
+    ap.add_argument("--tokens", type=int, default=8192, help="gemm: activation rows")
     ap.add_argument("--workload", default="qwen3_4b_layer")
     ap.add_argument("--tensor", default="gate_proj")
     ap.add_argument("--fmt", choices=["mxfp4", "nvfp4"], default="nvfp4")
@@ -66,8 +67,21 @@ def main():
                          F.focus_workspace_bytes(desc, F.FOCUS_WS_ALPHA)),
                      dtype=torch.uint8, device="cuda")
 
+    if a.phase == "gemm":
+        # W4A4 GEMM D[tokens, rows] = A[tokens, cols] W[rows, cols]^T on exports
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(4321)
+        act = torch.randn((a.tokens, cols), generator=gen, device="cuda").to(torch.bfloat16)
+        act_alpha = F.focus_nvfp4_alpha(act)
+        ac, at = F.focus_pack_mma(act, fmt, alpha=act_alpha)
+        wc, wt = F.focus_pack_mma(x, fmt, alpha=alpha)
+        dmat = torch.empty((a.tokens, rows), dtype=torch.bfloat16, device="cuda")
+        del act, g, gx, y
+
     def run():
-        if a.phase == "alpha":
+        if a.phase == "gemm":
+            F.focus_fp4_gemm(fmt, ac, at, wc, wt, act_alpha, alpha, d=dmat)
+        elif a.phase == "alpha":
             F.focus_nvfp4_alpha(x, alpha, ws)
         elif a.phase == "fwd":
             F.focus_fq_fwd(x, fmt, crs, dgs, alpha, sub_block=a.sub, shared=a.shared, y=y)
@@ -87,6 +101,12 @@ def main():
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
+    if a.phase == "gemm":
+        flops = 2 * a.tokens * rows * cols
+        print(json.dumps({"phase": "gemm", "tensor": f"{a.workload}/{a.tensor}",
+                          "shape": [a.tokens, rows, cols], "fmt": a.fmt, "ms": times,
+                          "tflops_last": flops / (times[-1] * 1e-3) / 1e12}))
+        return
     n = rows * cols
     bpe = bytes_per_elem(a.phase, a.fmt, a.sub, a.shared, not a.no_gx)
     print(json.dumps({"phase": a.phase, "tensor": f"{a.workload}/{a.tensor}", "shape": [rows, cols],
