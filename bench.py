@@ -49,6 +49,7 @@ class Case:
     shared: bool = False       # one coefficient set for all rows (activations)
     sfp: bool = False          # learnable full-precision scales S^fp (Eq. 4) and dL/dS^fp
     adam: bool = False         # backward fused with the AdamW step on c, c^k (and S^fp)
+    io: str = ""               # element type of x, y, g, gx ("" = the workload's own)
 
     @property
     def block(self) -> int:
@@ -361,6 +362,8 @@ def gpu_arm(case, args, rank, world, device):
     F.lib()
     w = W.WORKLOADS[case.workload] if case.workload in W.WORKLOADS else W.sweep_workload(
         int(case.workload.split("_")[-1]))
+    if case.io:
+        w = dataclasses.replace(w, dtype=case.io)
     # the fused optimizer's step counter t, advanced on the device before
     # every backward phase (inside the captured graphs)
     step_t = torch.zeros(1, dtype=torch.int64, device=device) if case.adam else None
@@ -490,6 +493,8 @@ def oracle_samples(case, rows_per_tensor):
     import numpy as np
     from paper_2608_01847_gb300 import workloads as W
     w = W.WORKLOADS[case.workload]
+    if case.io:
+        w = dataclasses.replace(w, dtype=case.io)
     out = []
     for i in range(len(w.tensors)):
         x, g = W.host_tensor(w, i, rows=rows_per_tensor)
@@ -498,8 +503,8 @@ def oracle_samples(case, rows_per_tensor):
         sfp = None
         if case.sfp:
             # absmax initialisation moved by U(0.9, 1.1), as on the device
-            xf = x.astype(np.uint32) << 16 if x.dtype == np.uint16 else x
-            m = np.abs(xf.view(np.float32)).reshape(x.shape[0], -1, case.block).max(-1)
+            xf = W.bf16_bits_to_f32(x) if x.dtype == np.uint16 else x.astype(np.float32)
+            m = np.abs(xf).reshape(x.shape[0], -1, case.block).max(-1)
             den = np.float32(6.0)
             if case.fmt == "nvfp4":
                 den = np.float32(m.max() / np.float32(2688.0)) * np.float32(6.0)
@@ -674,12 +679,14 @@ def main():
                     help="learnable full-precision scales S^fp and their gradient")
     ap.add_argument("--adam", action="store_true",
                     help="backward fused with the AdamW step on the learned arrays")
+    ap.add_argument("--io", default="", choices=["", "bf16", "f16", "f32"],
+                    help="element type of x, y, g, gx (default: the workload's)")
     ap.add_argument("--gemm", action="store_true",
                     help="time the W4A4 FP4 GEMMs of the workload's projections on their exports")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
-    case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp, args.adam)
+    case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp, args.adam, args.io)
     default_case = case == Case()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -735,7 +742,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": case.workload, "tensors": r["ntensors"], "elements": r["n_elem"],
-                   "fmt": case.fmt, "io_dtype": "bf16" if r["esz"] == 2 else "f32",
+                   "fmt": case.fmt, "io_dtype": case.io or ("bf16" if r["esz"] == 2 else "f32"),
                    "sub_block": case.sub,
                    "coefficients": ("shared by all rows" if case.shared else
                                     "per-block CRS + per-sub-block DGS"),

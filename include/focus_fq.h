@@ -68,14 +68,16 @@ typedef enum {
 } focus_status_t;
 
 typedef enum { FOCUS_MXFP4 = 0, FOCUS_NVFP4 = 1 } focus_format_t;
-typedef enum { FOCUS_F32 = 0, FOCUS_BF16 = 1 } focus_dtype_t;
+typedef enum { FOCUS_F32 = 0, FOCUS_BF16 = 1, FOCUS_F16 = 2 } focus_dtype_t;
 typedef enum { FOCUS_STE_IDENTITY = 0, FOCUS_STE_CLIPPED = 1 } focus_ste_t;
 typedef enum { FOCUS_MX_CEIL = 0, FOCUS_MX_FLOOR = 1 } focus_mx_rule_t;
 
 /* Tensor and method descriptor (host memory, read during the call only).
  *   rows, cols, ld    x is [rows, ld] row-major, blocks run along cols;
  *                     cols % block == 0; rows * cols / 8 < 2^31.
- *   dtype             focus_dtype_t of x, y, g and gx.
+ *   dtype             focus_dtype_t of x, y, g and gx (binary32, bfloat16 or
+ *                     IEEE binary16; 16-bit outputs are rounded to nearest
+ *                     even, binary16 overflowing to infinity).
  *   fmt               focus_format_t.
  *   block             32 for FOCUS_MXFP4, 16 for FOCUS_NVFP4 (Sec. 3.1).
  *   sub_block         DGS sub-block size b (Sec. 3.4): one of 2, 4, 8, 16,

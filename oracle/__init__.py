@@ -10,7 +10,8 @@ it follows: FOCUS Sec. 3.1 Eq. 1-3, Sec. 3.2 Eq. 4-5, Sec. 3.3 Eq. 6-7,
 Sec. 3.4 Eq. 8, Fig. 3(d)).  This module only builds it with gcc and marshals
 numpy arrays into it.
 
-Dtype codes: 0 = float32, 1 = bfloat16 (stored as uint16 bit patterns).
+Dtype codes: 0 = float32, 1 = bfloat16 (stored as uint16 bit patterns),
+2 = IEEE binary16 (numpy float16).
 Format codes: 0 = MXFP4 (block 32, E8M0), 1 = NVFP4 (block 16, E4M3 + alpha).
 """
 from __future__ import annotations
@@ -26,7 +27,7 @@ _SRC = os.path.join(_HERE, "focus_oracle.c")
 _LIB = os.path.join(_HERE, "_build", "libfocus_oracle.so")
 
 MXFP4, NVFP4 = 0, 1
-F32, BF16 = 0, 1
+F32, BF16, F16 = 0, 1, 2
 STE_IDENTITY, STE_CLIPPED = 0, 1
 MX_CEIL, MX_FLOOR = 0, 1
 
@@ -74,6 +75,8 @@ def lib() -> ctypes.CDLL:
         L.focus_oracle_e4m3_encodes.argtypes = [p, i64, p]
         L.focus_oracle_e8m0_exponents.argtypes = [p, i64, i32, p]
         L.focus_oracle_bf16_rnes.argtypes = [p, i64, p]
+        L.focus_oracle_f16_rnes.argtypes = [p, i64, p]
+        L.focus_oracle_f16_decodes.argtypes = [p, i64, p]
         _lib = L
     return _lib
 
@@ -100,7 +103,9 @@ def _dtype_code(x: np.ndarray) -> int:
         return F32
     if x.dtype == np.uint16:
         return BF16
-    raise TypeError("oracle inputs are float32 or uint16 (bfloat16 bit patterns)")
+    if x.dtype == np.float16:
+        return F16
+    raise TypeError("oracle inputs are float32, float16 or uint16 (bfloat16 bit patterns)")
 
 
 def _c32(a):
@@ -147,6 +152,22 @@ def bf16_rne(f) -> np.ndarray:
     f = np.ascontiguousarray(f, dtype=np.float32)
     out = np.empty(f.shape, np.uint16)
     lib().focus_oracle_bf16_rnes(_ptr(f), f.size, _ptr(out))
+    return out
+
+
+def f16_rne(f) -> np.ndarray:
+    """binary32 -> binary16 bit patterns (round to nearest even)."""
+    f = np.ascontiguousarray(f, dtype=np.float32)
+    out = np.empty(f.shape, np.uint16)
+    lib().focus_oracle_f16_rnes(_ptr(f), f.size, _ptr(out))
+    return out
+
+
+def f16_decode(h) -> np.ndarray:
+    """binary16 bit patterns -> binary32 values."""
+    h = np.ascontiguousarray(h, dtype=np.uint16)
+    out = np.empty(h.shape, np.float32)
+    lib().focus_oracle_f16_decodes(_ptr(h), h.size, _ptr(out))
     return out
 
 
@@ -314,7 +335,7 @@ def dequant(codes, scales, fmt, alpha=0.0, block=None, dtype=F32):
     rows = codes.shape[0]
     cols = codes.shape[1] * 2
     block = block or default_block(fmt)
-    y = np.empty((rows, cols), np.float32 if dtype == F32 else np.uint16)
+    y = np.empty((rows, cols), {F32: np.float32, BF16: np.uint16, F16: np.float16}[dtype])
     _check(lib().focus_oracle_dequant(fmt, dtype, rows, cols, block, _ptr(codes),
                                       _ptr(scales), float(alpha), _ptr(y)))
     return y

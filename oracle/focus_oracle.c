@@ -52,7 +52,7 @@
 #include <string.h>
 
 enum { OR_MXFP4 = 0, OR_NVFP4 = 1 };
-enum { OR_F32 = 0, OR_BF16 = 1 };
+enum { OR_F32 = 0, OR_BF16 = 1, OR_F16 = 2 };
 enum { OR_STE_IDENTITY = 0, OR_STE_CLIPPED = 1 };
 enum { OR_MX_CEIL = 0, OR_MX_FLOOR = 1 };
 
@@ -73,6 +73,51 @@ uint16_t focus_oracle_bf16_rne(float f)
     if (isnan(f)) return (uint16_t)(((b >> 16) & 0x8000u) | 0x7FC0u);
     uint32_t lsb = (b >> 16) & 1u;
     return (uint16_t)((b + 0x7FFFu + lsb) >> 16);
+}
+
+/* Round a non-negative binary64 value to the nearest integer, ties to the
+ * even integer (no dependence on the floating-point environment). */
+static double rne_int(double q)
+{
+    double f = floor(q), d = q - f;
+    if (d > 0.5) return f + 1.0;
+    if (d < 0.5) return f;
+    return fmod(f, 2.0) != 0.0 ? f + 1.0 : f;
+}
+
+/* IEEE 754 binary16 -> binary32 (exact): sign, 5-bit exponent (bias 15),
+ * 10-bit fraction; exponent 0 = subnormal m * 2^-24; 31 = inf / NaN. */
+float focus_oracle_f16_decode(uint16_t h)
+{
+    int s = h >> 15, e = (h >> 10) & 31, m = h & 1023;
+    float v;
+    if (e == 0) v = ldexpf((float)m, -24);
+    else if (e == 31) v = m ? NAN : INFINITY;
+    else v = ldexpf((float)(1024 + m), e - 25);
+    return s ? -v : v;
+}
+
+/* binary32 -> binary16, round to nearest, ties to even; magnitudes from
+ * 65520 up (the midpoint above the largest finite 65504) become infinity;
+ * NaN -> quiet NaN. */
+uint16_t focus_oracle_f16_rne(float f)
+{
+    uint16_t sign = signbit(f) ? 0x8000u : 0u;
+    if (isnan(f)) return (uint16_t)(sign | 0x7E00u);
+    double a = fabs((double)f);
+    if (a >= 65520.0) return (uint16_t)(sign | 0x7C00u);
+    if (a < ldexp(1.0, -14)) {
+        /* subnormal range: multiples of 2^-24 (1024 * 2^-24 is the
+         * smallest normal, whose encoding 0x400 the sum below produces) */
+        return (uint16_t)(sign | (uint16_t)rne_int(a * ldexp(1.0, 24)));
+    }
+    int ex;
+    frexp(a, &ex);                          /* a in [2^(ex-1), 2^ex) */
+    int E = ex - 1;
+    double m = rne_int(a * ldexp(1.0, 10 - E));   /* in [1024, 2048] */
+    if (m == 2048.0) { m = 1024.0; E += 1; }
+    if (E + 15 >= 31) return (uint16_t)(sign | 0x7C00u);
+    return (uint16_t)(sign | ((E + 15) << 10) | ((int)m - 1024));
 }
 
 /* ------------------------------------------------------------------ */
@@ -225,12 +270,14 @@ static float block_scale_fp(int fmt, float sfp, float alpha, uint8_t* byte)
 static float load_elem(int dtype, const void* p, int64_t idx)
 {
     if (dtype == OR_F32) return ((const float*)p)[idx];
+    if (dtype == OR_F16) return focus_oracle_f16_decode(((const uint16_t*)p)[idx]);
     return bf16_to_f32(((const uint16_t*)p)[idx]);
 }
 
 static void store_elem(int dtype, void* p, int64_t idx, float v)
 {
     if (dtype == OR_F32) ((float*)p)[idx] = v;
+    else if (dtype == OR_F16) ((uint16_t*)p)[idx] = focus_oracle_f16_rne(v);
     else ((uint16_t*)p)[idx] = focus_oracle_bf16_rne(v);
 }
 
@@ -252,7 +299,7 @@ static int check_shape(int64_t rows, int64_t cols, int64_t ld, int block, int su
     if (rows < 0 || cols < 0 || ld < cols) return -1;
     if (block <= 0 || sub <= 0 || block % sub != 0) return -1;
     if (cols % block != 0) return -1;
-    if (dtype != OR_F32 && dtype != OR_BF16) return -1;
+    if (dtype != OR_F32 && dtype != OR_BF16 && dtype != OR_F16) return -1;
     return 0;
 }
 
@@ -563,4 +610,14 @@ void focus_oracle_e8m0_exponents(const float* m, int64_t n, int rule, int32_t* o
 void focus_oracle_bf16_rnes(const float* f, int64_t n, uint16_t* out)
 {
     for (int64_t i = 0; i < n; i++) out[i] = focus_oracle_bf16_rne(f[i]);
+}
+
+void focus_oracle_f16_rnes(const float* f, int64_t n, uint16_t* out)
+{
+    for (int64_t i = 0; i < n; i++) out[i] = focus_oracle_f16_rne(f[i]);
+}
+
+void focus_oracle_f16_decodes(const uint16_t* h, int64_t n, float* out)
+{
+    for (int64_t i = 0; i < n; i++) out[i] = focus_oracle_f16_decode(h[i]);
 }

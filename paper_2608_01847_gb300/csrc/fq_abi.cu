@@ -40,10 +40,10 @@ int check_desc(const focus_desc_t* d, bool method)
 {
     if (!d) return FOCUS_ERR_INVALID_ARG;
     if (d->rows < 0 || d->cols < 0 || d->ld < d->cols || d->ld < 0) return FOCUS_ERR_INVALID_ARG;
-    if (d->dtype != FOCUS_F32 && d->dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
+    if (d->dtype != FOCUS_F32 && d->dtype != FOCUS_BF16 && d->dtype != FOCUS_F16) return FOCUS_ERR_INVALID_ARG;
     if (d->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
     // rows start on 32-byte boundaries (256-bit accesses)
-    if ((d->ld * (d->dtype == FOCUS_BF16 ? 2 : 4)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
+    if ((d->ld * (d->dtype == FOCUS_F32 ? 4 : 2)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
     if (d->rows > 0 && d->cols > 0 && d->rows > kMaxChunks / (d->cols / 8)) return FOCUS_ERR_UNSUPPORTED;
     if (!method) return FOCUS_OK;
     if (d->fmt != FOCUS_MXFP4 && d->fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;

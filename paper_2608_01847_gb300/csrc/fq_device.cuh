@@ -53,6 +53,18 @@ __device__ __forceinline__ uint32_t fast_div(uint32_t n, const FastDiv& f)
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
+// IEEE binary16 halves of a 32-bit word (exact widening) and the
+// round-to-nearest-even narrowing of two floats into one word.
+__device__ __forceinline__ float2 f16x2_to_float2(uint32_t w)
+{
+    return __half22float2(*reinterpret_cast<const __half2*>(&w));
+}
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi)
+{
+    const __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
 // Two binary32 values -> bf16x2 (round to nearest even); `lo` in bits 0-15.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 {
@@ -388,19 +400,20 @@ __device__ __forceinline__ void st_v8(void* p, const uint32_t (&w)[8])
 }
 
 // ---------------------------------------------------------------------------
-// Global memory: one "chunk" is 8 consecutive elements of a row (16 B bf16,
-// 32 B fp32), read with 128-bit non-coherent loads.
+// Global memory: one "chunk" is 8 consecutive elements of a row (16 B bf16
+// or fp16, 32 B fp32), read with 128-bit non-coherent loads.
+// DT: 0 binary32, 1 bfloat16, 2 binary16.
 // ---------------------------------------------------------------------------
 template <int DT>
 struct ChunkRaw {
-    uint4 w[DT == 1 ? 1 : 2];
+    uint4 w[DT != 0 ? 1 : 2];
 };
 
 template <int DT>
 __device__ __forceinline__ void load_chunk(ChunkRaw<DT>& c, const void* base, uint64_t off)
 {
     const uint4* p = reinterpret_cast<const uint4*>(static_cast<const char*>(base) +
-                                                    off * (DT == 1 ? 2u : 4u));
+                                                    off * (DT != 0 ? 2u : 4u));
     c.w[0] = __ldg(p);
     if (DT == 0) c.w[1] = __ldg(p + 1);
 }
@@ -422,6 +435,14 @@ __device__ __forceinline__ void unpack_chunk(const ChunkRaw<DT>& c, float (&v)[8
             v[2 * i] = bf16_lo(w[i]);
             v[2 * i + 1] = bf16_hi(w[i]);
         }
+    } else if (DT == 2) {
+        const uint32_t w[4] = {c.w[0].x, c.w[0].y, c.w[0].z, c.w[0].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = f16x2_to_float2(w[i]);
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
     } else {
 #pragma unroll
         for (int i = 0; i < 2; ++i) {
@@ -436,10 +457,13 @@ __device__ __forceinline__ void unpack_chunk(const ChunkRaw<DT>& c, float (&v)[8
 template <int DT>
 __device__ __forceinline__ void store_chunk(void* base, uint64_t off, const float (&v)[8])
 {
-    uint4* p = reinterpret_cast<uint4*>(static_cast<char*>(base) + off * (DT == 1 ? 2u : 4u));
+    uint4* p = reinterpret_cast<uint4*>(static_cast<char*>(base) + off * (DT != 0 ? 2u : 4u));
     if (DT == 1) {
         __stcs(p, make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
                              pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7])));
+    } else if (DT == 2) {
+        __stcs(p, make_uint4(pack_f16x2(v[0], v[1]), pack_f16x2(v[2], v[3]),
+                             pack_f16x2(v[4], v[5]), pack_f16x2(v[6], v[7])));
     } else {
         __stcs(p, make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]),
                              __float_as_uint(v[2]), __float_as_uint(v[3])));

@@ -5,8 +5,8 @@ namespace focus {
 
 cudaError_t launch_bwd_adamw_nv(int dt, int sub, bool sfpg, const KParams& p, cudaStream_t st)
 {
-    if (sfpg) return dt ? linear_by_sub<1, 1, kBwdSA>(sub, p, st) : linear_by_sub<1, 0, kBwdSA>(sub, p, st);
-    return dt ? linear_by_sub<1, 1, kBwdA>(sub, p, st) : linear_by_sub<1, 0, kBwdA>(sub, p, st);
+    if (sfpg) return linear_by_dt<1, kBwdSA>(dt, sub, p, st);
+    return linear_by_dt<1, kBwdA>(dt, sub, p, st);
 }
 
 }  // namespace focus

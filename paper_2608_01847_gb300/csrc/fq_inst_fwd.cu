@@ -5,8 +5,8 @@ namespace focus {
 
 cudaError_t launch_fwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
 {
-    if (fmt == 0) return dt ? linear_by_sub<0, 1, kFwd>(sub, p, st) : linear_by_sub<0, 0, kFwd>(sub, p, st);
-    return dt ? linear_by_sub<1, 1, kFwd>(sub, p, st) : linear_by_sub<1, 0, kFwd>(sub, p, st);
+    if (fmt == 0) return linear_by_dt<0, kFwd>(dt, sub, p, st);
+    return linear_by_dt<1, kFwd>(dt, sub, p, st);
 }
 
 }  // namespace focus

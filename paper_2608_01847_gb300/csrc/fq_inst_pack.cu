@@ -24,15 +24,16 @@ __global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* part
 
 cudaError_t launch_pack(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
 {
-    if (fmt == 0) return dt ? linear_by_sub<0, 1, kPack>(sub, p, st) : linear_by_sub<0, 0, kPack>(sub, p, st);
-    return dt ? linear_by_sub<1, 1, kPack>(sub, p, st) : linear_by_sub<1, 0, kPack>(sub, p, st);
+    if (fmt == 0) return linear_by_dt<0, kPack>(dt, sub, p, st);
+    return linear_by_dt<1, kPack>(dt, sub, p, st);
 }
 
 cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_t st)
 {
     const uint32_t grid = alpha_grid(p.n_chunks);
     if (p.n_chunks > 0) {
-        if (dt) alpha_partial_kernel<1><<<grid, kThreads, 0, st>>>(p);
+        if (dt == 1) alpha_partial_kernel<1><<<grid, kThreads, 0, st>>>(p);
+        else if (dt == 2) alpha_partial_kernel<2><<<grid, kThreads, 0, st>>>(p);
         else alpha_partial_kernel<0><<<grid, kThreads, 0, st>>>(p);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;

@@ -78,7 +78,7 @@ template <int FMT, int DT, int SUB>
 struct Geo {
     static constexpr int B = FMT == 0 ? 32 : 16;   // hardware block (Sec. 3.1)
     static constexpr int K = B / SUB;              // sub-blocks per block (Sec. 3.4)
-    static constexpr int W = DT == 1 ? B / 2 : B;  // 32-bit words of a block of x
+    static constexpr int W = DT != 0 ? B / 2 : B;  // 32-bit words of a block of x
     static_assert(SUB >= 2 && SUB <= B && B % SUB == 0, "sub-block must divide the block");
 };
 
@@ -116,16 +116,19 @@ template <int DT>
 __device__ __forceinline__ float2 elem_pair(const uint32_t* w, int i)
 {
     if (DT == 1) return make_float2(bf16_lo(w[i]), bf16_hi(w[i]));
+    if (DT == 2) return f16x2_to_float2(w[i]);
     return make_float2(__uint_as_float(w[2 * i]), __uint_as_float(w[2 * i + 1]));
 }
 
-// Store a pair of results in the block's output words (bf16 round to
-// nearest even, or binary32 as is).
+// Store a pair of results in the block's output words (bf16 / fp16 round
+// to nearest even, or binary32 as is).
 template <int DT>
 __device__ __forceinline__ void put_pair(uint32_t* w, int i, float2 v)
 {
     if (DT == 1) {
         w[i] = pack_bf16x2(v.x, v.y);
+    } else if (DT == 2) {
+        w[i] = pack_f16x2(v.x, v.y);
     } else {
         w[2 * i] = __float_as_uint(v.x);
         w[2 * i + 1] = __float_as_uint(v.y);
@@ -133,18 +136,21 @@ __device__ __forceinline__ void put_pair(uint32_t* w, int i, float2 v)
 }
 
 // max |x| over a block, read off the stored bits (non-negative floats order
-// like their encodings): packed u16x2 maxima for bf16, u32 for binary32.
+// like their encodings): packed u16x2 maxima for bf16 and fp16, u32 for
+// binary32.
 template <int DT, int W>
 __device__ __forceinline__ float block_absmax(const uint32_t (&w)[W])
 {
-    if (DT == 1) {
+    if (DT != 0) {
         uint32_t m = w[0] & 0x7fff7fffu;
 #pragma unroll
         for (int i = 1; i < W; ++i) {
             const uint32_t a = w[i] & 0x7fff7fffu;
             asm("max.u16x2 %0, %0, %1;" : "+r"(m) : "r"(a));
         }
-        return __uint_as_float(max(m << 16, m & 0xffff0000u));
+        if (DT == 1) return __uint_as_float(max(m << 16, m & 0xffff0000u));
+        const uint32_t top = max(m & 0xffffu, m >> 16);
+        return __half2float(__ushort_as_half(static_cast<unsigned short>(top)));
     }
     uint32_t m = w[0] & 0x7fffffffu;
 #pragma unroll
@@ -427,7 +433,7 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
                                           df (&T)[K], df& gS)
 {
     constexpr int SUB = B / K;
-    constexpr int EPG = DT == 1 ? 16 : 8;  // elements per 256-bit group
+    constexpr int EPG = DT != 0 ? 16 : 8;  // elements per 256-bit group
     const uint32_t live = (ste == 1) ? block_clip_mask<DT, B, K>(xw, sq, dead) : 0xffffffffu;
     const float rc = rcp_approx(c);
     df Q = {0.0f, 0.0f};
@@ -591,7 +597,7 @@ template <int FMT, int DT, int MODE>
 struct Unroll {
     // blocks per thread per step: 64 bytes of x in flight for the streaming
     // passes, one block (x and g) for the backward
-    static constexpr int U = (MODE >= kBwd) ? 1 : ((FMT == 1 && DT == 1) ? 2 : 1);
+    static constexpr int U = (MODE >= kBwd) ? 1 : ((FMT == 1 && DT != 0) ? 2 : 1);
 };
 
 // Resident CTAs per SM the register allocation must allow: enough 256-thread
@@ -610,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
     using G = Geo<FMT, DT, SUB>;
     constexpr int B = G::B, K = G::K, W = G::W;
     constexpr int U = Unroll<FMT, DT, MODE>::U;
-    constexpr int ESZ = DT == 1 ? 2 : 4;
+    constexpr int ESZ = DT != 0 ? 2 : 4;
     constexpr bool BWD = MODE >= kBwd;
     constexpr bool SFPG = MODE == kBwdS || MODE == kBwdSA;
     constexpr bool ADAM = MODE >= kBwdA;
@@ -693,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
                 uint32_t codes[B / 8];
                 block_codes<DT, B, K>(xr[j], sq, dead, codes);
                 if constexpr (MODE == kFwd) {
-                    constexpr int EPG = DT == 1 ? 16 : 8;  // elements per 256-bit group
+                    constexpr int EPG = DT != 0 ? 16 : 8;  // elements per 256-bit group
                     uint32_t grp[8];
 #pragma unroll
                     for (int w = 0; w < B / 8; ++w) {
@@ -787,7 +793,7 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
 {
     using G = Geo<FMT, DT, SUB>;
     constexpr int B = G::B, K = G::K, W = G::W;
-    constexpr int ESZ = DT == 1 ? 2 : 4;
+    constexpr int ESZ = DT != 0 ? 2 : 4;
     __shared__ float2 red[kThreads * K];
     const TensorScale ts = tensor_scale<FMT>(p.alpha);
     const bool want_gx = p.gx != nullptr;
@@ -921,7 +927,7 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams
 template <int DT>
 __global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p)
 {
-    constexpr int U = DT == 1 ? 4 : 2;
+    constexpr int U = DT != 0 ? 4 : 2;
     __shared__ float red[kThreads / 32];
     float m = 0.0f;
     const uint32_t span = U * kThreads;

@@ -98,6 +98,18 @@ cudaError_t linear_by_sub(int sub, const KParams& p, cudaStream_t st)
     return cudaErrorInvalidValue;
 }
 
+// Dispatch over the element type (0 binary32, 1 bfloat16, 2 binary16).
+template <int FMT, int MODE>
+cudaError_t linear_by_dt(int dt, int sub, const KParams& p, cudaStream_t st)
+{
+    switch (dt) {
+    case 0: return linear_by_sub<FMT, 0, MODE>(sub, p, st);
+    case 1: return linear_by_sub<FMT, 1, MODE>(sub, p, st);
+    case 2: return linear_by_sub<FMT, 2, MODE>(sub, p, st);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
 // Shared-row backward: the row-group kernel, then (when coefficient
 // gradients or an optimizer step are wanted) the column finalisation.
 template <int FMT, int SUB>
@@ -131,6 +143,17 @@ cudaError_t bwd_shared_by_sub(int sub, const KParams& p, uint32_t ny, cudaStream
     default: break;
     }
     return cudaErrorInvalidValue;
+}
+
+template <int FMT>
+cudaError_t bwd_shared_by_dt(int dt, int sub, const KParams& p, uint32_t ny, cudaStream_t st)
+{
+    switch (dt) {
+    case 0: return bwd_shared_by_sub<FMT, 0>(sub, p, ny, st);
+    case 1: return bwd_shared_by_sub<FMT, 1>(sub, p, ny, st);
+    case 2: return bwd_shared_by_sub<FMT, 2>(sub, p, ny, st);
+    default: return cudaErrorInvalidValue;
+    }
 }
 
 // Defined in the instantiation units.

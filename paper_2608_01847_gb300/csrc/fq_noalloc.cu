@@ -69,9 +69,10 @@ FOCUS_API int focus_nvfp4_alpha_noalloc(const focus_desc_t* desc, const void* x,
     // same shape rules as focus_nvfp4_alpha (only the tensor shape is used)
     if (!desc) return FOCUS_ERR_INVALID_ARG;
     if (desc->rows < 0 || desc->cols < 0 || desc->ld < desc->cols) return FOCUS_ERR_INVALID_ARG;
-    if (desc->dtype != FOCUS_F32 && desc->dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
+    if (desc->dtype != FOCUS_F32 && desc->dtype != FOCUS_BF16 && desc->dtype != FOCUS_F16)
+        return FOCUS_ERR_INVALID_ARG;
     if (desc->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
-    if ((desc->ld * (desc->dtype == FOCUS_BF16 ? 2 : 4)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
+    if ((desc->ld * (desc->dtype == FOCUS_F32 ? 4 : 2)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
     if (desc->rows > 0 && desc->cols > 0 && desc->rows > ((int64_t(1) << 31) - 1) / (desc->cols / 8))
         return FOCUS_ERR_UNSUPPORTED;
     const bool empty = desc->rows == 0 || desc->cols == 0;

@@ -20,7 +20,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_build", "libfocus_fq.so")
 
 FOCUS_MXFP4, FOCUS_NVFP4 = 0, 1
-FOCUS_F32, FOCUS_BF16 = 0, 1
+FOCUS_F32, FOCUS_BF16, FOCUS_F16 = 0, 1, 2
 FOCUS_STE_IDENTITY, FOCUS_STE_CLIPPED = 0, 1
 FOCUS_MX_CEIL, FOCUS_MX_FLOOR = 0, 1
 FOCUS_WS_ALPHA, FOCUS_WS_BWD = 0, 1
@@ -103,7 +103,9 @@ def _dtype_code(t: torch.Tensor) -> int:
         return FOCUS_F32
     if t.dtype == torch.bfloat16:
         return FOCUS_BF16
-    raise TypeError(f"unsupported dtype {t.dtype} (float32 or bfloat16)")
+    if t.dtype == torch.float16:
+        return FOCUS_F16
+    raise TypeError(f"unsupported dtype {t.dtype} (float32, bfloat16 or float16)")
 
 
 def make_desc(x: torch.Tensor, fmt: int = FOCUS_MXFP4, sub_block: int = 8, shared: bool = False,

@@ -59,7 +59,7 @@ class Workload:
     """One configuration: a list of tensors plus how to draw them."""
     name: str
     tensors: Tuple[TensorSpec, ...]
-    dtype: str                  # "f32" or "bf16"
+    dtype: str                  # "f32", "bf16" or "f16"
     fmts: Tuple[str, ...]       # subset of ("mxfp4", "nvfp4")
     kind: str                   # "weight" or "activation"
     nu: Optional[float]         # Student-t degrees of freedom (weights)
@@ -161,13 +161,16 @@ def draw_grad(rows: int, cols: int, seed: int) -> np.ndarray:
 
 def host_tensor(w: Workload, idx: int, rows: Optional[int] = None):
     """(x, g) host arrays for tensor `idx` (optionally only the first `rows`
-    rows), in the workload's dtype: float32, or uint16 bf16 bits."""
+    rows), in the workload's dtype: float32, uint16 bf16 bits, or float16
+    (numpy's round-to-nearest conversion of the float32 draws)."""
     t = w.tensors[idx]
     r = t.rows if rows is None else min(rows, t.rows)
     x = draw_values(w, r, t.cols, tensor_seed(w, idx))
     g = draw_grad(r, t.cols, tensor_seed(w, idx, 1))
     if w.dtype == "bf16":
         return to_bf16_bits(x), to_bf16_bits(g)
+    if w.dtype == "f16":
+        return x.astype(np.float16), g.astype(np.float16)
     return x, g
 
 
@@ -220,6 +223,8 @@ def device_tensor(w: Workload, idx: int, device, torch_mod=None):
         def trunc(a):
             return (a.view(torch.int32) >> 16).to(torch.int16).view(torch.bfloat16)
         return trunc(v), trunc(g)
+    if w.dtype == "f16":
+        return v.half(), g.half()
     return v, g
 
 

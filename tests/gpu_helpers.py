@@ -18,9 +18,11 @@ FLOOR_SHARED = 2.0 ** -30
 
 
 def dev(a: np.ndarray) -> torch.Tensor:
-    """Host array (float32, or uint16 bf16 bits) -> CUDA tensor."""
+    """Host array (float32, float16, or uint16 bf16 bits) -> CUDA tensor."""
     if a.dtype == np.uint16:
         return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
+    if a.dtype == np.float16:
+        return torch.from_numpy(np.ascontiguousarray(a)).cuda()
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).cuda()
 
 
@@ -70,7 +72,7 @@ def assert_grad_close(got: np.ndarray, ref: np.ndarray, ref_abs: np.ndarray, flo
 
 
 def oracle_dtype(a: np.ndarray) -> int:
-    return O.BF16 if a.dtype == np.uint16 else O.F32
+    return {np.dtype(np.uint16): O.BF16, np.dtype(np.float16): O.F16}.get(a.dtype, O.F32)
 
 
 # ---------------------------------------------------------------------------

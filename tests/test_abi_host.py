@@ -75,7 +75,7 @@ def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None
     (dict(block=64), -2), (dict(fmt=1, block=32), -2), (dict(sub=3), -2), (dict(sub=32, fmt=1), -2),
     (dict(sub=64), -2), (dict(cols=48), -1), (dict(ld=60), -1), (dict(ld=68), -3),
     (dict(ld=72), -3), (dict(ld=72, dtype=0, rows=0), 0),
-    (dict(dtype=2), -1), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
+    (dict(dtype=3), -1), (dict(dtype=2, rows=0), 0), (dict(dtype=2, ld=72), -3), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
     (dict(shared=2), -1), (dict(rows=-1), -1), (dict(rows=1 << 40, cols=1 << 20), -2),
 ])
 def test_descriptor_rejections(L, kw, status):

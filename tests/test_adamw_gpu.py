@@ -119,7 +119,7 @@ def run_adamw(x, g, fmt, learn, step, sub=8, shared=False, ste=O.STE_IDENTITY, s
 # per-row coefficients: formats, dtypes, learned subsets, steps, sub-blocks
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 @pytest.mark.parametrize("learn", [("crs", "dgs", "sfp"), ("crs", "dgs"), ("dgs",), ("sfp",),
                                    ("crs", "sfp")])
 @pytest.mark.parametrize("step", [1, 7, 1000])

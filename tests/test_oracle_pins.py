@@ -821,3 +821,58 @@ def test_fp4_gemm_is_the_product_of_fake_quantized_operands(fmt):
     else:
         bound = 2.0 ** -22 * (np.abs(ya) @ np.abs(yb).T)
         assert np.all(np.abs(d - ya @ yb.T) <= bound)
+
+
+# ---------------------------------------------------------------------------
+# binary16 I/O
+# ---------------------------------------------------------------------------
+def test_f16_decode_all_patterns_matches_numpy():
+    h = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    ours = O.f16_decode(h)
+    ref = h.view(np.float16).astype(np.float32)
+    fin = np.isfinite(ref)
+    assert np.array_equal(ours[fin].view(np.uint32), ref[fin].view(np.uint32))
+    assert np.all(np.isnan(ours[np.isnan(ref)])) and np.array_equal(ours[np.isinf(ref)], ref[np.isinf(ref)])
+
+
+def test_f16_rne_matches_numpy():
+    """Every binary16 value, the midpoints between neighbours and one binary32
+    ulp either side of each (ties to even, subnormals, the overflow
+    threshold 65520), plus random patterns."""
+    h = np.arange(0, 0x7C00, dtype=np.uint32).astype(np.uint16)
+    v = h.view(np.float16).astype(np.float64)
+    mids = ((v[:-1] + v[1:]) / 2).astype(np.float32)
+    ulp = lambda a, d: np.nextafter(a, np.float32(d * np.inf)).astype(np.float32)
+    cand = np.concatenate([v.astype(np.float32), mids, ulp(mids, 1), ulp(mids, -1),
+                           np.array([65504, 65519.996, 65520, 65536, 1e9, 2 ** -25, 2 ** -24,
+                                     3 * 2 ** -26, 2 ** -26], np.float32)])
+    rng = np.random.default_rng(111)
+    cand = np.concatenate([cand, rng.integers(0, 1 << 32, 2_000_000, dtype=np.uint64)
+                           .astype(np.uint32).view(np.float32)])
+    cand = cand[np.isfinite(cand)]
+    cand = np.concatenate([cand, -cand])
+    with np.errstate(over="ignore"):
+        ref = cand.astype(np.float16).view(np.uint16)
+    assert np.array_equal(O.f16_rne(cand), ref)
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_f16_io_is_the_f32_path_rounded(fmt):
+    """binary16 I/O: x widened exactly, every quantity computed as for
+    binary32 inputs, y and gx rounded to binary16 at the end."""
+    rng = np.random.default_rng(113)
+    block = 32 if fmt == O.MXFP4 else 16
+    x16 = (rng.standard_normal((12, 4 * block)) * 0.3).astype(np.float16)
+    g16 = rng.standard_normal((12, 4 * block)).astype(np.float16)
+    crs = rng.uniform(0.8, 1.2, (12, 4)).astype(np.float32)
+    x32, g32 = x16.astype(np.float32), g16.astype(np.float32)
+    a = O.alpha(x16) if fmt == O.NVFP4 else 0.0
+    assert a == (O.alpha(x32) if fmt == O.NVFP4 else 0.0)
+    f16 = O.fwd(x16, fmt, crs=crs, alpha=a, want_codes=True)
+    f32 = O.fwd(x32, fmt, crs=crs, alpha=a, want_codes=True)
+    assert np.array_equal(f16["codes"], f32["codes"]) and np.array_equal(f16["scales"], f32["scales"])
+    assert np.array_equal(f16["y"].view(np.uint16), O.f16_rne(f32["y"]))
+    b16 = O.bwd(x16, g16, fmt, crs=crs, alpha=a)
+    b32 = O.bwd(x32, g32, fmt, crs=crs, alpha=a)
+    assert np.array_equal(b16["gx"].view(np.uint16), O.f16_rne(b32["gx"]))
+    assert np.array_equal(b16["gcrs"], b32["gcrs"])

@@ -97,7 +97,7 @@ def test_w256x512_f32_mxfp4(mode):
 # several tiles + ragged tails, strided rows, both dtypes and formats
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 @pytest.mark.parametrize("rows,cols,pad", [(37, 352, 0), (5, 4096, 0), (129, 96, 32), (1, 32, 0),
                                            (3000, 160, 0), (17, 1216, 16)])
 def test_shapes(fmt, dtype, rows, cols, pad):
@@ -110,7 +110,7 @@ def test_shapes(fmt, dtype, rows, cols, pad):
 
 @pytest.mark.parametrize("fmt,sub", [("mx", 2), ("mx", 4), ("mx", 8), ("mx", 16), ("mx", 32),
                                      ("nv", 2), ("nv", 4), ("nv", 8), ("nv", 16)])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 def test_sub_block_sizes(fmt, sub, dtype):
     rows, cols = 77, 640
     w, x, g = seeded(rows, cols, dtype, seed=sub)
@@ -122,7 +122,7 @@ def test_sub_block_sizes(fmt, sub, dtype):
 
 
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 def test_clipped_ste_and_floor_rule(fmt, dtype):
     rows, cols = 64, 512
     w, x, g = seeded(rows, cols, dtype, seed=3, coef=(0.6, 1.0))   # c < 1: saturation happens
@@ -136,7 +136,7 @@ def test_clipped_ste_and_floor_rule(fmt, dtype):
 
 
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 @pytest.mark.parametrize("rows,cols", [(300, 256), (1030, 96), (3, 4096)])
 def test_shared_row_coefficients(fmt, dtype, rows, cols):
     w, x, g = seeded(rows, cols, dtype, seed=rows, scale=1.0, nu=None, coef=(0.9, 1.1))
@@ -284,7 +284,7 @@ def absmax_sfp_host(x, fmt, alpha):
 
 
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 @pytest.mark.parametrize("sub", [8, 4])
 @pytest.mark.parametrize("ste", [O.STE_IDENTITY, O.STE_CLIPPED])
 def test_learnable_scale(fmt, dtype, sub, ste):
@@ -346,7 +346,7 @@ def test_absmax_sfp_matches_absmax_path_on_gpu(fmt):
 # export in the block-scaled MMA scale-factor layout
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
-@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32", "f16"])
 @pytest.mark.parametrize("rows,cols", [(256, 512), (300, 96), (1, 48 * 2), (129, 1216)])
 def test_pack_mma_layout(fmt, dtype, rows, cols):
     f = FMT[fmt]
@@ -369,3 +369,23 @@ def test_pack_mma_layout(fmt, dtype, rows, cols):
     assert_bits_equal(host(codes), ref["codes"], "codes (mma export)")
     assert_bits_equal(host(codes_rm), ref["codes"], "codes (row-major export)")
     assert_bits_equal(host(tiles), O.mma_scale_tiles(ref["scales"]), "scale tiles")
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_f16_overflow_and_subnormals(fmt):
+    """binary16 I/O at the edges: values whose dequantized result or input
+    gradient leaves the binary16 range (-> inf, as the oracle rounds) and
+    subnormal inputs."""
+    f = FMT[fmt]
+    block = 32 if f == O.MXFP4 else 16
+    rows, cols = 8, 4 * block
+    rng = np.random.default_rng(7)
+    x = (rng.standard_normal((rows, cols)) * 0.2).astype(np.float32)
+    x[0] *= 2.0 ** 15                       # near the top of the binary16 range
+    x[1] *= 2.0 ** -16                      # subnormal binary16 inputs
+    x[2, :block] = 60000.0
+    x[2, 1] = -65504.0
+    g = rng.standard_normal((rows, cols)).astype(np.float32)
+    g[3] = np.clip(g[3] * 16000.0, -65000.0, 65000.0)   # finite in binary16; g / c overflows
+    crs = np.full((rows, cols // block), 0.7, np.float32)   # c < 1: y above x
+    run_case(x.astype(np.float16), g.astype(np.float16), f, crs, None)
