@@ -282,6 +282,69 @@ class Tensor:
         return 2 if phase == "alpha" else (2 if (phase == "bwd" and self.case.shared) else 1)
 
 
+class GroupRunner:
+    """Every phase as one group launch over all tensors of the layer (the
+    group entry points); outputs are the Tensor objects' own buffers."""
+
+    def __init__(self, ts, case, device):
+        import torch
+        from paper_2608_01847_gb300 import focus as F
+        self.ts, self.case = ts, case
+        self.fmt = ts[0].fmt
+        nv = case.fmt == "nvfp4"
+        if nv:
+            # one alpha array for the layer; each tensor reads its own entry
+            self.alphas = torch.zeros(len(ts), dtype=torch.float32, device=device)
+            for i, t in enumerate(ts):
+                self.alphas[i:i + 1].copy_(t.alpha)
+                t.alpha = self.alphas[i:i + 1]
+            self.ws = torch.empty(max(16, F.focus_group_workspace_bytes([t.x for t in ts])),
+                                  dtype=torch.uint8, device=device)
+        common = lambda t: {"x": t.x, "crs": t.crs, "dgs": t.dgs, "alpha": t.alpha if nv else None,
+                            "sfp": t.sfp}
+        self.fwd = [dict(common(t), y=t.y) for t in ts]
+        self.pack = [dict(common(t), codes=t.codes, scale_bytes=t.scales) for t in ts]
+        self.bwd = []
+        for t in ts:
+            d = dict(common(t), g=t.g, gx=t.gx, gcrs=t.gcrs, gdgs=t.gdgs)
+            if t.gsfp is not None:
+                d["gsfp"] = t.gsfp
+            self.bwd.append(d)
+
+    def run(self, phase):
+        from paper_2608_01847_gb300 import focus as F
+        sub = self.case.sub
+        if phase == "alpha":
+            F.focus_nvfp4_alpha_group([t.x for t in self.ts], alpha_out=self.alphas, ws=self.ws)
+        elif phase == "fwd":
+            F.focus_fq_fwd_group(self.fwd, self.fmt, sub_block=sub)
+        elif phase == "bwd":
+            F.focus_fq_bwd_group(self.bwd, self.fmt, sub_block=sub)
+        else:
+            F.focus_pack_group(self.pack, self.fmt, sub_block=sub)
+
+    @staticmethod
+    def launches(phase):
+        return 2 if phase == "alpha" else 1
+
+
+class SeqGraph:
+    """A CUDA graph of `body(stage)` for each stage, in order, on one stream."""
+
+    def __init__(self, body, device, stages):
+        import torch
+        self.graph = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream(device)
+        cap.wait_stream(torch.cuda.current_stream(device))
+        with torch.cuda.graph(self.graph, stream=cap):
+            for stage in stages:
+                body(stage)
+        torch.cuda.current_stream(device).wait_stream(cap)
+
+    def replay(self):
+        self.graph.replay()
+
+
 class BranchGraph:
     """A CUDA graph of one or more stages run in order; in each stage the
     branches (one stream each) run `body(i, stage)` for every tensor i
@@ -378,20 +441,32 @@ def gpu_arm(case, args, rank, world, device):
         if step_t is not None and stage == "bwd":
             step_t.add_(1)
 
+    # per-tensor launches on parallel graph branches (measured fastest on
+    # GB300), or with --group the whole layer per phase in one group launch
+    grouped = args.group and not (case.shared or case.adam) and len(ts) <= 16
+    runner = GroupRunner(ts, case, device) if grouped else None
+
     # eager warm-up (resolves launch configurations), then capture each phase
     for ph in phases:
         before(ph)
-        for t in ts:
-            t.run(ph)
+        if grouped:
+            runner.run(ph)
+        else:
+            for t in ts:
+                t.run(ph)
     torch.cuda.synchronize(device)
     # one graph per phase (for the phase split) and one for the whole step;
     # with the optimizer, one of each per batch parity (alternating batches)
     parities = (0, 1) if case.adam else (0,)
-    graphs = {ph: [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
-                               stages=(ph,), before=before) for par in parities]
-              for ph in phases}
-    step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
-                               stages=phases, before=before) for par in parities]
+    if grouped:
+        graphs = {ph: [SeqGraph(runner.run, device, (ph,))] for ph in phases}
+        step_graphs = [SeqGraph(runner.run, device, phases)]
+    else:
+        graphs = {ph: [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
+                                   stages=(ph,), before=before) for par in parities]
+                  for ph in phases}
+        step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
+                                   stages=phases, before=before) for par in parities]
     n_replay = [0]
 
     def step():
@@ -431,7 +506,9 @@ def gpu_arm(case, args, rank, world, device):
     total_ms = max_over_ranks(total_ms, world, device)
 
     res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, clocks=clk.summary(),
-               ntensors=len(ts), launches_per_step=sum(t.launches(ph) for t in ts for ph in phases))
+               ntensors=len(ts), grouped=grouped,
+               launches_per_step=(sum(GroupRunner.launches(ph) for ph in phases) if grouped else
+                                  sum(t.launches(ph) for t in ts for ph in phases)))
     if args.no_e2e:
         return res
 
@@ -681,6 +758,8 @@ def main():
                     help="backward fused with the AdamW step on the learned arrays")
     ap.add_argument("--io", default="", choices=["", "bf16", "f16", "f32"],
                     help="element type of x, y, g, gx (default: the workload's)")
+    ap.add_argument("--group", action="store_true",
+                    help="one group launch per phase for all tensors instead of per-tensor launches")
     ap.add_argument("--gemm", action="store_true",
                     help="time the W4A4 FP4 GEMMs of the workload's projections on their exports")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -747,6 +826,8 @@ def main():
                    "coefficients": ("shared by all rows" if case.shared else
                                     "per-block CRS + per-sub-block DGS"),
                    "scales": "learnable S^fp (+ dL/dS^fp)" if case.sfp else "absmax",
+                   "launch": "one group launch per phase" if r["grouped"] else
+                             "one launch per tensor and phase, tensors on parallel graph branches",
                    "step": "+".join(case.phases()) + " over all tensors " +
                            ("(bwd: gx + AdamW on the learned arrays)" if case.adam else
                             "(bwd: gx + gcrs + gdgs)"),

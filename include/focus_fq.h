@@ -288,6 +288,57 @@ int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* 
                    const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,
                    int64_t ldd, int32_t* timeout_flag, focus_stream_t stream);
 
+/* ---- Group entry points --------------------------------------------------
+ * One launch for several tensors, e.g. all projections of a transformer
+ * layer: the kernel walks the blocks of all tensors as one range, so no
+ * tensor's tail runs alone on a mostly idle GPU and per-tensor launches are
+ * saved.  Every result is exactly the per-tensor entry point's, bit for bit
+ * (each block is computed by the same code from the same inputs).
+ *
+ * Each tensor is described by one focus_tensor_t (host memory, read during
+ * the call); the fields a call does not use are ignored.  Rules, checked on
+ * the host before anything is launched:
+ * - 0 <= n <= FOCUS_MAX_GROUP (FOCUS_ERR_UNSUPPORTED above);
+ * - all descriptors share fmt, dtype, block, sub_block, ste and mx_rule
+ *   (FOCUS_ERR_INVALID_ARG otherwise); coef_shared_rows must be 0 (shared
+ *   coefficients: use the per-tensor entry points);
+ * - each tensor obeys the per-tensor entry point's rules (pointers,
+ *   alignment, required outputs); empty tensors are skipped;
+ * - at most 2^31 - 1 blocks in total. */
+#define FOCUS_MAX_GROUP 16
+
+typedef struct {
+    focus_desc_t desc;
+    const void* x;          /* input                                  (all)  */
+    const void* g;          /* upstream gradient dL/dy                (bwd)  */
+    void* y;                /* fake-quantized output                  (fwd)  */
+    void* gx;               /* optional dL/dx                         (bwd)  */
+    const float* crs;       /* optional c_i                                  */
+    const float* dgs;       /* optional c_i^k                                */
+    const float* alpha;     /* NVFP4 per-tensor scale (device; fwd, bwd, pack) */
+    const float* sfp;       /* optional learnable S^fp                       */
+    float* gcrs;            /* optional dL/dc_i                       (bwd)  */
+    float* gdgs;            /* optional dL/dc_i^k                     (bwd)  */
+    float* gsfp;            /* optional dL/dS^fp                      (bwd)  */
+    uint8_t* codes;         /* export codes                           (pack) */
+    uint8_t* scale_bytes;   /* scale bytes: optional (fwd), required (pack) */
+} focus_tensor_t;
+
+/* focus_nvfp4_alpha for each tensor (Eq. 2); alpha_out: n device floats.
+ * ws: focus_group_workspace_bytes(t, n) bytes of device scratch, 16-byte
+ * aligned.  desc->fmt / sub_block are not used. */
+int focus_nvfp4_alpha_group(const focus_tensor_t* t, int n, float* alpha_out, void* ws,
+                            size_t ws_bytes, focus_stream_t stream);
+/* Scratch that focus_nvfp4_alpha_group needs for these tensors (0 if the
+ * group is invalid). */
+size_t focus_group_workspace_bytes(const focus_tensor_t* t, int n);
+/* focus_fq_fwd for each tensor (Eq. 1-8). */
+int focus_fq_fwd_group(const focus_tensor_t* t, int n, focus_stream_t stream);
+/* focus_fq_bwd for each tensor (Sec. 3.2), per-row coefficients only. */
+int focus_fq_bwd_group(const focus_tensor_t* t, int n, focus_stream_t stream);
+/* focus_pack for each tensor (Fig. 3(d)), row-major scale bytes. */
+int focus_pack_group(const focus_tensor_t* t, int n, focus_stream_t stream);
+
 /* Device scratch (bytes) that focus_nvfp4_alpha (which = FOCUS_WS_ALPHA) or
  * focus_fq_bwd (which = FOCUS_WS_BWD) needs for this descriptor on the
  * current device; 0 for an invalid descriptor. */

@@ -1,6 +1,7 @@
 // fq_abi.cu -- the extern "C" entry points declared in include/focus_fq.h:
 // argument validation, launch parameters, scratch sizing, error mapping.
 // No allocation, no host synchronisation, no exception crosses the ABI.
+#include <algorithm>
 #include <cstdint>
 #include <cstring>
 
@@ -405,4 +406,181 @@ FOCUS_API int focus_fq_bwd_adamw(const focus_desc_t* desc, const void* x, float*
     const OptArgs opt = {crs, dgs, sfp, hp, state, step};
     return run_bwd(desc, x, crs, dgs, alpha, sfp, g, gx, gcrs, gdgs, gsfp, ws, ws_bytes,
                    reinterpret_cast<cudaStream_t>(stream), &opt);
+}
+
+// ---------------------------------------------------------------------------
+// Group entry points
+// ---------------------------------------------------------------------------
+namespace focus {
+namespace {
+
+enum GroupMode { kGroupAlpha, kGroupFwd, kGroupPack, kGroupBwd };
+
+// Validate a group and fill g (non-empty tensors only); fmt / dt / sub /
+// sfpg describe the kernel to run.
+int build_group(const focus_tensor_t* t, int n, GroupMode mode, KGroup& g, int& dt, int& fmt, int& sub,
+                bool& sfpg)
+{
+    if (n < 0) return FOCUS_ERR_INVALID_ARG;
+    if (n > kMaxGroup) return FOCUS_ERR_UNSUPPORTED;
+    if (n > 0 && !t) return FOCUS_ERR_INVALID_ARG;
+    std::memset(&g, 0, sizeof(g));
+    bool any_dgs = false;
+    sfpg = false;
+    uint64_t total = 0;
+    for (int i = 0; i < n; ++i) {
+        const focus_desc_t& d = t[i].desc;
+        const focus_tensor_t& a = t[i];
+        int rc = check_desc(&d, mode != kGroupAlpha);
+        if (rc) return rc;
+        const focus_desc_t& d0 = t[0].desc;
+        if (d.dtype != d0.dtype) return FOCUS_ERR_INVALID_ARG;
+        if (mode != kGroupAlpha) {
+            if (d.fmt != d0.fmt || d.block != d0.block || d.sub_block != d0.sub_block || d.ste != d0.ste ||
+                d.mx_rule != d0.mx_rule)
+                return FOCUS_ERR_INVALID_ARG;
+            if (d.coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
+            if ((rc = check_coef_ptrs(a.crs, a.dgs, a.gcrs, a.gdgs))) return rc;
+            if (misaligned(a.alpha, 4) || misaligned(a.sfp, 4) || misaligned(a.gsfp, 4))
+                return FOCUS_ERR_MISALIGNED;
+        }
+        const bool empty = d.rows == 0 || d.cols == 0;
+        if (empty && mode != kGroupAlpha) continue;   // (an empty tensor's alpha is 0)
+        if (!empty && !a.x) return FOCUS_ERR_INVALID_ARG;
+        if (mode != kGroupAlpha && d.fmt == FOCUS_NVFP4 && !a.alpha) return FOCUS_ERR_INVALID_ARG;
+        switch (mode) {
+        case kGroupAlpha:
+            if (misaligned(a.x, 16)) return FOCUS_ERR_MISALIGNED;
+            break;
+        case kGroupFwd:
+            if (!a.y) return FOCUS_ERR_INVALID_ARG;
+            if (misaligned(a.x, 32) || misaligned(a.y, 32)) return FOCUS_ERR_MISALIGNED;
+            break;
+        case kGroupPack:
+            if (!a.codes || !a.scale_bytes) return FOCUS_ERR_INVALID_ARG;
+            if (misaligned(a.x, 32) || misaligned(a.codes, 16)) return FOCUS_ERR_MISALIGNED;
+            break;
+        case kGroupBwd:
+            if (!a.g) return FOCUS_ERR_INVALID_ARG;
+            if (misaligned(a.x, 32) || misaligned(a.g, 32) || misaligned(a.gx, 32)) return FOCUS_ERR_MISALIGNED;
+            if (!a.gx && !a.gcrs && !a.gdgs && !a.gsfp) continue;   // nothing asked of this tensor
+            break;
+        }
+        KParams& p = g.p[g.n];
+        p = make_params(&d);
+        p.x = a.x;
+        if (mode != kGroupAlpha) {
+            p.crs = a.crs;
+            p.dgs = a.dgs;
+            p.alpha = a.alpha;
+            p.sfp = a.sfp;
+        }
+        if (mode == kGroupFwd) {
+            p.y = a.y;
+            p.scales = a.scale_bytes;
+        } else if (mode == kGroupPack) {
+            p.codes = a.codes;
+            p.scales = a.scale_bytes;
+        } else if (mode == kGroupBwd) {
+            p.g = a.g;
+            p.gx = a.gx;
+            p.gcrs = a.gcrs;
+            p.gdgs = a.gdgs;
+            p.gsfp = a.gsfp;
+            any_dgs |= a.gdgs != nullptr;
+            sfpg |= a.sfp != nullptr || a.gsfp != nullptr;
+        }
+        any_dgs |= a.dgs != nullptr;
+        total += mode == kGroupAlpha ? p.n_chunks : p.n_blocks;
+        g.n += 1;
+    }
+    if (total > static_cast<uint64_t>(INT32_MAX)) return FOCUS_ERR_UNSUPPORTED;
+    dt = n > 0 ? t[0].desc.dtype : 0;
+    fmt = n > 0 ? t[0].desc.fmt : 0;
+    sub = (n > 0 && any_dgs) ? t[0].desc.sub_block : (n > 0 ? t[0].desc.block : 16);
+    uint32_t at = 0;
+    for (int i = 0; i < g.n; ++i) {
+        g.start[i] = at;
+        at += g.p[i].n_blocks;
+    }
+    g.start[g.n] = at;
+    return FOCUS_OK;
+}
+
+// CTAs of the grouped alpha pass: the per-tensor pass's grid for the whole
+// group, shared in proportion to the tensors' sizes (at least one each).
+void alpha_group_ctas(KGroup& g)
+{
+    uint64_t total = 0;
+    for (int i = 0; i < g.n; ++i) total += g.p[i].n_chunks;
+    const uint64_t G = alpha_grid(static_cast<uint32_t>(total));
+    uint32_t at = 0;
+    for (int i = 0; i < g.n; ++i) {
+        g.start[i] = at;
+        if (g.p[i].n_chunks > 0)
+            at += static_cast<uint32_t>(std::max<uint64_t>(1, G * g.p[i].n_chunks / total));
+    }
+    g.start[g.n] = at;
+}
+
+}  // namespace
+}  // namespace focus
+
+FOCUS_API size_t focus_group_workspace_bytes(const focus_tensor_t* t, int n)
+{
+    KGroup g;
+    int dt, fmt, sub;
+    bool sfpg;
+    if (build_group(t, n, kGroupAlpha, g, dt, fmt, sub, sfpg) != FOCUS_OK) return 0;
+    alpha_group_ctas(g);
+    return static_cast<size_t>(g.start[g.n]) * sizeof(float);
+}
+
+FOCUS_API int focus_nvfp4_alpha_group(const focus_tensor_t* t, int n, float* alpha_out, void* ws,
+                                      size_t ws_bytes, focus_stream_t stream)
+{
+    KGroup g;
+    int dt, fmt, sub;
+    bool sfpg;
+    int rc = build_group(t, n, kGroupAlpha, g, dt, fmt, sub, sfpg);
+    if (rc) return rc;
+    if (n == 0) return FOCUS_OK;
+    if (!alpha_out) return FOCUS_ERR_INVALID_ARG;
+    if (misaligned(alpha_out, 4) || misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
+    alpha_group_ctas(g);
+    const size_t need = static_cast<size_t>(g.start[g.n]) * sizeof(float);
+    if (need > 0 && (!ws || ws_bytes < need)) return FOCUS_ERR_WORKSPACE;
+    g.p[0].ws = static_cast<float*>(ws);
+    return map_cuda(launch_alpha_group(dt, g, alpha_out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_fq_fwd_group(const focus_tensor_t* t, int n, focus_stream_t stream)
+{
+    KGroup g;
+    int dt, fmt, sub;
+    bool sfpg;
+    int rc = build_group(t, n, kGroupFwd, g, dt, fmt, sub, sfpg);
+    if (rc || g.n == 0) return rc;
+    return map_cuda(launch_group_fwd(fmt, dt, sub, g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_pack_group(const focus_tensor_t* t, int n, focus_stream_t stream)
+{
+    KGroup g;
+    int dt, fmt, sub;
+    bool sfpg;
+    int rc = build_group(t, n, kGroupPack, g, dt, fmt, sub, sfpg);
+    if (rc || g.n == 0) return rc;
+    return map_cuda(launch_group_pack(fmt, dt, sub, g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+FOCUS_API int focus_fq_bwd_group(const focus_tensor_t* t, int n, focus_stream_t stream)
+{
+    KGroup g;
+    int dt, fmt, sub;
+    bool sfpg;
+    int rc = build_group(t, n, kGroupBwd, g, dt, fmt, sub, sfpg);
+    if (rc || g.n == 0) return rc;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    return map_cuda(fmt == 0 ? launch_group_bwd_mx(dt, sub, sfpg, g, st) : launch_group_bwd_nv(dt, sub, sfpg, g, st));
 }

@@ -4,8 +4,7 @@
 namespace focus {
 
 // One CTA: max of the per-CTA partial maxima, alpha = fl(amax / 2688) (Eq. 2).
-__global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* partials, uint32_t n,
-                                                               float* alpha_out)
+__device__ __forceinline__ void alpha_final_kernel_body(const float* partials, uint32_t n, float* alpha_out)
 {
     __shared__ float red[kThreads / 32];
     float m = 0.0f;
@@ -22,10 +21,38 @@ __global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* part
     }
 }
 
+__global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* partials, uint32_t n,
+                                                               float* alpha_out)
+{
+    alpha_final_kernel_body(partials, n, alpha_out);
+}
+
 cudaError_t launch_pack(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
 {
     if (fmt == 0) return linear_by_dt<0, kPack>(dt, sub, p, st);
     return linear_by_dt<1, kPack>(dt, sub, p, st);
+}
+
+// Group form: CTA t reduces the partials of tensor t to alpha_out[t].
+__global__ void __launch_bounds__(kThreads) alpha_group_final_kernel(const __grid_constant__ KGroup g,
+                                                                     float* alpha_out)
+{
+    const uint32_t t = blockIdx.x;
+    alpha_final_kernel_body(g.p[0].ws + g.start[t], g.start[t + 1] - g.start[t], alpha_out + t);
+}
+
+cudaError_t launch_alpha_group(int dt, const KGroup& g, float* alpha_out, cudaStream_t st)
+{
+    const uint32_t grid = g.start[g.n];
+    if (grid > 0) {
+        if (dt == 1) alpha_group_partial_kernel<1><<<grid, kThreads, 0, st>>>(g);
+        else if (dt == 2) alpha_group_partial_kernel<2><<<grid, kThreads, 0, st>>>(g);
+        else alpha_group_partial_kernel<0><<<grid, kThreads, 0, st>>>(g);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    alpha_group_final_kernel<<<g.n, kThreads, 0, st>>>(g, alpha_out);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_t st)

@@ -609,9 +609,52 @@ struct MinCtas {
         ((MODE >= kBwd) ? (FMT == 1 ? 3 : 2) : 4) - (SUB == 2 ? 1 : 0);
 };
 
-template <int FMT, int DT, int SUB, int MODE>
-__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
-    fq_block_kernel(const KParams p)
+// Where a block's tensor comes from: one tensor (the per-tensor entry
+// points), or a group of tensors walked as one concatenated block range (the
+// group entry points: one launch for all projections of a layer, so no
+// tensor's tail waits alone and launches are saved).
+template <int FMT>
+struct OneTensor {
+    const KParams& p;
+    TensorScale scale;
+    __device__ __forceinline__ explicit OneTensor(const KParams& q) : p(q), scale(tensor_scale<FMT>(q.alpha)) {}
+    // tiles of `span` blocks; tile i is blocks [i * span, (i + 1) * span)
+    __device__ __forceinline__ uint32_t tiles(uint32_t span) const { return (p.n_blocks + span - 1) / span; }
+    __device__ __forceinline__ int tensor(uint32_t) const { return 0; }
+    __device__ __forceinline__ uint32_t base(uint32_t tile, int, uint32_t span) const { return tile * span; }
+    __device__ __forceinline__ const KParams& at(int) const { return p; }
+    __device__ __forceinline__ const TensorScale& ts(int) const { return scale; }
+};
+
+constexpr int kMaxGroup = 16;
+struct KGroup {
+    KParams p[kMaxGroup];
+    uint32_t start[kMaxGroup + 1];  // first tile of tensor t; a tile is one CTA step of blocks
+    int n;
+};
+
+template <int FMT>
+struct TensorGroup {
+    const KGroup& g;
+    const TensorScale* scale;       // per tensor, in shared memory
+    // tensors start on tile boundaries, so a CTA step never mixes tensors
+    __device__ __forceinline__ uint32_t tiles(uint32_t) const { return g.start[g.n]; }
+    __device__ __forceinline__ int tensor(uint32_t tile) const
+    {
+        int t = 0;
+        while (t + 1 < g.n && tile >= g.start[t + 1]) ++t;
+        return t;
+    }
+    __device__ __forceinline__ uint32_t base(uint32_t tile, int t, uint32_t span) const
+    {
+        return (tile - g.start[t]) * span;
+    }
+    __device__ __forceinline__ const KParams& at(int t) const { return g.p[t]; }
+    __device__ __forceinline__ const TensorScale& ts(int t) const { return scale[t]; }
+};
+
+template <int FMT, int DT, int SUB, int MODE, class Src>
+__device__ __forceinline__ void block_loop(const Src& src)
 {
     using G = Geo<FMT, DT, SUB>;
     constexpr int B = G::B, K = G::K, W = G::W;
@@ -620,15 +663,20 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
     constexpr bool BWD = MODE >= kBwd;
     constexpr bool SFPG = MODE == kBwdS || MODE == kBwdSA;
     constexpr bool ADAM = MODE >= kBwdA;
-    const TensorScale ts = tensor_scale<FMT>(p.alpha);
-    const bool want_gx = BWD && p.gx != nullptr;
-    const bool want_T = SFPG || (BWD && (p.gcrs != nullptr || p.gdgs != nullptr)) ||
-                        (ADAM && (p.new_crs != nullptr || p.new_dgs != nullptr));
     AdamW aw;
-    if constexpr (ADAM) aw = adamw_setup(p);
+    if constexpr (ADAM) aw = adamw_setup(src.at(0));   // one optimizer step for all tensors
     const uint32_t span = U * kThreads;
+    const uint32_t n_tiles = src.tiles(span);
 
-    for (uint32_t base = blockIdx.x * span; base < p.n_blocks; base += gridDim.x * span) {
+    for (uint32_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        // one tensor per CTA step: its parameters are uniform across the CTA
+        const int tt = src.tensor(tile);
+        const KParams& p = src.at(tt);
+        const TensorScale& ts = src.ts(tt);
+        const uint32_t base = src.base(tile, tt, span);
+        const bool want_gx = BWD && p.gx != nullptr;
+        const bool want_T = SFPG || (BWD && (p.gcrs != nullptr || p.gdgs != nullptr)) ||
+                            (ADAM && (p.new_crs != nullptr || p.new_dgs != nullptr));
         uint32_t xr[U][W];
         uint32_t gr[BWD ? U : 1][BWD ? W : 1];
         uint64_t off[U];
@@ -779,6 +827,25 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
     }
 }
 
+
+template <int FMT, int DT, int SUB, int MODE>
+__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
+    fq_block_kernel(const KParams p)
+{
+    block_loop<FMT, DT, SUB, MODE>(OneTensor<FMT>(p));
+}
+
+template <int FMT, int DT, int SUB, int MODE>
+__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
+    fq_group_kernel(const __grid_constant__ KGroup g)
+{
+    static_assert(MODE < kBwdA, "the fused optimizer is per tensor");
+    __shared__ TensorScale scale[kMaxGroup];
+    if (threadIdx.x < g.n) scale[threadIdx.x] = tensor_scale<FMT>(g.p[threadIdx.x].alpha);
+    __syncthreads();
+    block_loop<FMT, DT, SUB, MODE>(TensorGroup<FMT>{g, scale});
+}
+
 // ---------------------------------------------------------------------------
 // Backward with coefficients shared by all rows.  A CTA is p.tx columns of
 // blocks x (kThreads / p.tx) row slots; thread (tx, ty) owns column block
@@ -924,14 +991,15 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_finalize(const KParams
 // NVFP4 per-tensor alpha (Eq. 2): per-CTA max|x| into scratch, then one CTA
 // takes the max of the partials and writes fl(amax / 2688).
 // ---------------------------------------------------------------------------
+// max|x| over the chunks of one tensor that CTA `cta` of `n_ctas` covers
+// (grid-stride), reduced over the CTA; thread 0 holds the result.
 template <int DT>
-__global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p)
+__device__ __forceinline__ float alpha_cta_max(const KParams& p, uint32_t cta, uint32_t n_ctas, float* red)
 {
     constexpr int U = DT != 0 ? 4 : 2;
-    __shared__ float red[kThreads / 32];
     float m = 0.0f;
     const uint32_t span = U * kThreads;
-    for (uint32_t base = blockIdx.x * span; base < p.n_chunks; base += gridDim.x * span) {
+    for (uint32_t base = cta * span; base < p.n_chunks; base += n_ctas * span) {
         ChunkRaw<DT> xr[U];
 #pragma unroll
         for (int j = 0; j < U; ++j) {
@@ -965,8 +1033,29 @@ __global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p
         m = (threadIdx.x < kThreads / 32) ? red[threadIdx.x] : 0.0f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, o));
-        if (threadIdx.x == 0) p.ws[blockIdx.x] = m;
     }
+    return m;
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p)
+{
+    __shared__ float red[kThreads / 32];
+    const float m = alpha_cta_max<DT>(p, blockIdx.x, gridDim.x, red);
+    if (threadIdx.x == 0) p.ws[blockIdx.x] = m;
+}
+
+// Group form: g.start[t] .. g.start[t + 1] are the CTAs given to tensor t
+// (in proportion to its size, at least one); each writes its partial to
+// g.p[0].ws[blockIdx.x].
+template <int DT>
+__global__ void __launch_bounds__(kThreads) alpha_group_partial_kernel(const __grid_constant__ KGroup g)
+{
+    __shared__ float red[kThreads / 32];
+    int t = 0;
+    while (t + 1 < g.n && blockIdx.x >= g.start[t + 1]) ++t;
+    const float m = alpha_cta_max<DT>(g.p[t], blockIdx.x - g.start[t], g.start[t + 1] - g.start[t], red);
+    if (threadIdx.x == 0) g.p[0].ws[blockIdx.x] = m;
 }
 
 }  // namespace focus

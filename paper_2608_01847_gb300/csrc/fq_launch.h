@@ -110,6 +110,60 @@ cudaError_t linear_by_dt(int dt, int sub, const KParams& p, cudaStream_t st)
     }
 }
 
+// Group launches: one kernel over the concatenated blocks of up to
+// kMaxGroup tensors that share format, element type and sub-block size.
+template <int FMT, int DT, int SUB, int MODE>
+cudaError_t run_group(const KGroup& g_blocks, cudaStream_t st)
+{
+    static int occ = 0;
+    auto kern = fq_group_kernel<FMT, DT, SUB, MODE>;
+    // every tensor starts on a tile (one CTA step of U * kThreads blocks)
+    constexpr uint32_t span = Unroll<FMT, DT, MODE>::U * kThreads;
+    KGroup g = g_blocks;
+    uint32_t at = 0;
+    for (int i = 0; i < g.n; ++i) {
+        g.start[i] = at;
+        at += (g.p[i].n_blocks + span - 1) / span;
+    }
+    g.start[g.n] = at;
+    const uint32_t grid = stream_grid(kern, occ, at, 1);
+    kern<<<grid, kThreads, 0, st>>>(g);
+    return cudaGetLastError();
+}
+
+template <int FMT, int DT, int MODE>
+cudaError_t group_by_sub(int sub, const KGroup& g, cudaStream_t st)
+{
+    switch (sub) {
+    case 2: return run_group<FMT, DT, 2, MODE>(g, st);
+    case 4: return run_group<FMT, DT, 4, MODE>(g, st);
+    case 8: return run_group<FMT, DT, 8, MODE>(g, st);
+    case 16: return run_group<FMT, DT, 16, MODE>(g, st);
+    case 32:
+        if constexpr (FMT == 0) return run_group<FMT, DT, 32, MODE>(g, st);
+        break;
+    default: break;
+    }
+    return cudaErrorInvalidValue;
+}
+
+template <int FMT, int MODE>
+cudaError_t group_by_dt(int dt, int sub, const KGroup& g, cudaStream_t st)
+{
+    switch (dt) {
+    case 0: return group_by_sub<FMT, 0, MODE>(sub, g, st);
+    case 1: return group_by_sub<FMT, 1, MODE>(sub, g, st);
+    case 2: return group_by_sub<FMT, 2, MODE>(sub, g, st);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+// Defined in the group instantiation units.
+cudaError_t launch_group_fwd(int fmt, int dt, int sub, const KGroup& g, cudaStream_t st);
+cudaError_t launch_group_pack(int fmt, int dt, int sub, const KGroup& g, cudaStream_t st);
+cudaError_t launch_group_bwd_mx(int dt, int sub, bool sfpg, const KGroup& g, cudaStream_t st);
+cudaError_t launch_group_bwd_nv(int dt, int sub, bool sfpg, const KGroup& g, cudaStream_t st);
+
 // Shared-row backward: the row-group kernel, then (when coefficient
 // gradients or an optimizer step are wanted) the column finalisation.
 template <int FMT, int SUB>
@@ -165,5 +219,6 @@ cudaError_t launch_bwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t 
 cudaError_t launch_bwd_shared(int fmt, int dt, int sub, const KParams& p, uint32_t ny,
                               cudaStream_t st);
 cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_t st);
+cudaError_t launch_alpha_group(int dt, const KGroup& g, float* alpha_out, cudaStream_t st);
 
 }  // namespace focus

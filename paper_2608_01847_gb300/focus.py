@@ -30,7 +30,8 @@ STATUS = {0: "FOCUS_OK", -1: "FOCUS_ERR_INVALID_ARG", -2: "FOCUS_ERR_UNSUPPORTED
 
 ENTRY_POINTS = ("focus_nvfp4_alpha", "focus_nvfp4_alpha_noalloc", "focus_fq_fwd", "focus_fq_bwd",
                 "focus_fq_bwd_adamw", "focus_pack", "focus_pack_mma", "focus_mma_scale_bytes",
-                "focus_fp4_gemm",
+                "focus_fp4_gemm", "focus_nvfp4_alpha_group", "focus_group_workspace_bytes",
+                "focus_fq_fwd_group", "focus_fq_bwd_group", "focus_pack_group",
                 "focus_workspace_bytes", "focus_status_string", "focus_version")
 
 
@@ -46,6 +47,14 @@ class focus_desc_t(ctypes.Structure):
                 ("dtype", ctypes.c_int32), ("fmt", ctypes.c_int32), ("block", ctypes.c_int32),
                 ("sub_block", ctypes.c_int32), ("coef_shared_rows", ctypes.c_int32),
                 ("ste", ctypes.c_int32), ("mx_rule", ctypes.c_int32)]
+
+
+class focus_tensor_t(ctypes.Structure):
+    _fields_ = [("desc", focus_desc_t)] + [(n, ctypes.c_void_p) for n in (
+        "x", "g", "y", "gx", "crs", "dgs", "alpha", "sfp", "gcrs", "gdgs", "gsfp", "codes", "scale_bytes")]
+
+
+FOCUS_MAX_GROUP = 16
 
 
 class focus_adamw_t(ctypes.Structure):
@@ -82,6 +91,14 @@ def lib() -> ctypes.CDLL:
         L.focus_mma_scale_bytes.restype = SZ
         I32, I64 = ctypes.c_int32, ctypes.c_int64
         L.focus_fp4_gemm.argtypes = [I32, I64, I64, I64, P, P, P, P, P, P, P, I32, I64, P, P]
+        T = ctypes.POINTER(focus_tensor_t)
+        L.focus_nvfp4_alpha_group.argtypes = [T, ctypes.c_int, P, P, SZ, P]
+        L.focus_group_workspace_bytes.argtypes = [T, ctypes.c_int]
+        L.focus_group_workspace_bytes.restype = SZ
+        for n in ("focus_fq_fwd_group", "focus_fq_bwd_group", "focus_pack_group"):
+            getattr(L, n).argtypes = [T, ctypes.c_int, P]
+            getattr(L, n).restype = ctypes.c_int
+        L.focus_nvfp4_alpha_group.restype = ctypes.c_int
         L.focus_workspace_bytes.argtypes = [D, ctypes.c_int]
         L.focus_workspace_bytes.restype = SZ
         L.focus_status_string.argtypes = [ctypes.c_int]
@@ -372,3 +389,106 @@ def focus_fp4_gemm(fmt, a_codes, a_tiles, b_codes, b_tiles, alpha_a=None, alpha_
 
 def focus_version() -> int:
     return int(lib().focus_version())
+
+
+# ---------------------------------------------------------------------------
+# group entry points: one launch for several tensors
+# ---------------------------------------------------------------------------
+_GROUP_FIELDS = ("x", "g", "y", "gx", "crs", "dgs", "alpha", "sfp", "gcrs", "gdgs", "gsfp", "codes",
+                 "scale_bytes")
+
+
+def _group_array(items, fmt, sub_block, ste=FOCUS_STE_IDENTITY, mx_rule=FOCUS_MX_CEIL):
+    """ctypes array of focus_tensor_t from dicts of tensors (keys as the
+    struct's fields).  The dicts are kept alive by the caller."""
+    if len(items) > FOCUS_MAX_GROUP:
+        raise ValueError(f"at most {FOCUS_MAX_GROUP} tensors per group")
+    arr = (focus_tensor_t * max(1, len(items)))()
+    for i, it in enumerate(items):
+        x = it["x"]
+        arr[i].desc = make_desc(x, fmt, sub_block, False, ste, mx_rule)
+        for k in _GROUP_FIELDS:
+            t = it.get(k)
+            if t is not None:
+                setattr(arr[i], k, t.data_ptr())
+    return arr
+
+
+def focus_nvfp4_alpha_group(xs, alpha_out=None, ws=None):
+    """Per-tensor NVFP4 alpha (Eq. 2) of every tensor in xs, one launch pair;
+    returns a [n] fp32 tensor."""
+    items = [{"x": x} for x in xs]
+    arr = _group_array(items, FOCUS_NVFP4, 16)
+    dev_ = xs[0].device
+    if alpha_out is None:
+        alpha_out = torch.empty(len(xs), dtype=torch.float32, device=dev_)
+    n = int(lib().focus_group_workspace_bytes(arr, len(xs)))
+    if ws is None:
+        ws = torch.empty(max(16, n), dtype=torch.uint8, device=dev_)
+    _check(lib().focus_nvfp4_alpha_group(arr, len(xs), _p(alpha_out), _p(ws), ws.numel(), _stream(dev_)),
+           "focus_nvfp4_alpha_group")
+    return alpha_out
+
+
+def focus_group_workspace_bytes(xs) -> int:
+    arr = _group_array([{"x": x} for x in xs], FOCUS_NVFP4, 16)
+    return int(lib().focus_group_workspace_bytes(arr, len(xs)))
+
+
+def focus_fq_fwd_group(items, fmt, *, sub_block=8, mx_rule=FOCUS_MX_CEIL):
+    """focus_fq_fwd for each dict of `items` (keys x, crs, dgs, alpha, sfp and
+    optionally y, scale_bytes); allocates a missing y; returns the list of y."""
+    for it in items:
+        if it.get("y") is None:
+            it["y"] = _like_x(it["x"])
+        _same_layout(it["x"], it["y"], "y")
+        _check_coefs(it["x"], fmt, sub_block, False, it.get("crs"), it.get("dgs"))
+        _check_sfp(it["x"], fmt, it.get("sfp"), "sfp")
+    arr = _group_array(items, fmt, sub_block, FOCUS_STE_IDENTITY, mx_rule)
+    _check(lib().focus_fq_fwd_group(arr, len(items), _stream(items[0]["x"].device)), "focus_fq_fwd_group")
+    return [it["y"] for it in items]
+
+
+def focus_pack_group(items, fmt, *, sub_block=8, mx_rule=FOCUS_MX_CEIL):
+    """focus_pack for each dict of `items`; allocates missing codes /
+    scale_bytes; returns the list of (codes, scale_bytes)."""
+    for it in items:
+        x = it["x"]
+        rows, cols = x.shape
+        if it.get("codes") is None:
+            it["codes"] = torch.empty((rows, cols // 2), dtype=torch.uint8, device=x.device)
+        if it.get("scale_bytes") is None:
+            it["scale_bytes"] = torch.empty((rows, cols // block_of(fmt)), dtype=torch.uint8, device=x.device)
+        _dense(it["codes"], rows * cols // 2, torch.uint8, "codes")
+        _dense(it["scale_bytes"], rows * cols // block_of(fmt), torch.uint8, "scale_bytes")
+        _check_coefs(x, fmt, sub_block, False, it.get("crs"), it.get("dgs"))
+        _check_sfp(x, fmt, it.get("sfp"), "sfp")
+    arr = _group_array(items, fmt, sub_block, FOCUS_STE_IDENTITY, mx_rule)
+    _check(lib().focus_pack_group(arr, len(items), _stream(items[0]["x"].device)), "focus_pack_group")
+    return [(it["codes"], it["scale_bytes"]) for it in items]
+
+
+def focus_fq_bwd_group(items, fmt, *, sub_block=8, ste=FOCUS_STE_IDENTITY, mx_rule=FOCUS_MX_CEIL):
+    """focus_fq_bwd for each dict of `items` (keys x, g, crs, dgs, alpha, sfp
+    and the outputs gx, gcrs, gdgs, gsfp, each allocated when the dict has
+    the key with value None); returns the list of dicts."""
+    for it in items:
+        x = it["x"]
+        rows, cols = x.shape
+        _same_layout(x, it["g"], "g")
+        if "gx" in it and it["gx"] is None:
+            it["gx"] = _like_x(x)
+        if "gcrs" in it and it["gcrs"] is None:
+            it["gcrs"] = torch.empty((rows, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
+        if "gdgs" in it and it["gdgs"] is None:
+            it["gdgs"] = torch.empty((rows, cols // sub_block), dtype=torch.float32, device=x.device)
+        if "gsfp" in it and it["gsfp"] is None:
+            it["gsfp"] = torch.empty((rows, cols // block_of(fmt)), dtype=torch.float32, device=x.device)
+        _same_layout(x, it.get("gx"), "gx")
+        _check_coefs(x, fmt, sub_block, False, it.get("crs"), it.get("dgs"))
+        _check_coefs(x, fmt, sub_block, False, it.get("gcrs"), it.get("gdgs"))
+        _check_sfp(x, fmt, it.get("sfp"), "sfp")
+        _check_sfp(x, fmt, it.get("gsfp"), "gsfp")
+    arr = _group_array(items, fmt, sub_block, ste, mx_rule)
+    _check(lib().focus_fq_bwd_group(arr, len(items), _stream(items[0]["x"].device)), "focus_fq_bwd_group")
+    return items

@@ -137,7 +137,7 @@ def draw_values(w: Workload, rows: int, cols: int, seed: int) -> np.ndarray:
         v = rng.standard_t(w.nu, size=(rows, cols)) * w.scale
     else:
         v = rng.standard_normal(size=(rows, cols)) * w.scale
-    if w.outlier == "entries" and w.outlier_count > 0:
+    if w.outlier == "entries" and w.outlier_count > 0 and rows * cols > 0:
         k = max(1, int(round(w.outlier_count * rows * cols)))
         idx = rng.choice(rows * cols, size=k, replace=False)
         v.reshape(-1)[idx] *= w.outlier_mult
@@ -208,7 +208,7 @@ def device_tensor(w: Workload, idx: int, device, torch_mod=None):
         v.mul_(w.scale)
     else:
         v = torch.randn(shape, generator=gen, device=device).mul_(w.scale)
-    if w.outlier == "entries" and w.outlier_count > 0:
+    if w.outlier == "entries" and w.outlier_count > 0 and t.rows * t.cols > 0:
         k = max(1, int(round(w.outlier_count * t.rows * t.cols)))
         idx_ = torch.randint(0, t.rows * t.cols, (k,), generator=gen, device=device)
         v.view(-1)[idx_] *= w.outlier_mult

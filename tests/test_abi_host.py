@@ -198,3 +198,34 @@ def test_adamw_argument_rejections(L):
     assert adamw(L, _desc(fmt=1, block=32), _hp(), _st()) == -2
     d = _desc(rows=64, cols=256, shared=1)
     assert adamw(L, d, _hp(), _st()) == -4                         # shared rows need scratch
+
+
+def _targ(rows=4, cols=64, dtype=1, fmt=1, shared=0, sub=8, x=ALIGNED, y=ALIGNED2, alpha=ALIGNED2):
+    t = F.focus_tensor_t()
+    t.desc = _desc(rows=rows, cols=cols, dtype=dtype, fmt=fmt, shared=shared, sub=sub)
+    t.x, t.y, t.alpha = x.value, y.value, alpha.value
+    t.g, t.codes, t.scale_bytes = ALIGNED2.value, ALIGNED2.value, ALIGNED2.value
+    return t
+
+
+def test_group_rejections(L):
+    def fwd_group(*ts):
+        arr = (F.focus_tensor_t * max(1, len(ts)))(*ts)
+        return L.focus_fq_fwd_group(arr, len(ts), None)
+    assert fwd_group() == 0                                             # nothing to do
+    assert L.focus_fq_fwd_group(None, 1, None) == -1
+    assert L.focus_fq_fwd_group(None, -1, None) == -1
+    arr = (F.focus_tensor_t * 17)(*[_targ(rows=0) for _ in range(17)])
+    assert L.focus_fq_fwd_group(arr, 17, None) == -2                   # more than FOCUS_MAX_GROUP
+    assert fwd_group(_targ(rows=0), _targ(rows=0, dtype=0)) == -1      # element types differ
+    assert fwd_group(_targ(rows=0), _targ(rows=0, sub=4)) == -1        # sub-block sizes differ
+    assert fwd_group(_targ(rows=0), _targ(rows=0, fmt=0, sub=8)) == -1  # formats differ
+    assert fwd_group(_targ(rows=0, shared=1)) == -1                    # shared coefficients
+    assert fwd_group(_targ(x=ODD)) == -3
+    assert fwd_group(_targ(alpha=P(0))) == -1                          # NVFP4 needs alpha
+    assert fwd_group(_targ(y=P(0))) == -1
+    assert fwd_group(_targ(rows=0), _targ(rows=0)) == 0                 # empty tensors are skipped
+    arr = (F.focus_tensor_t * 2)(_targ(rows=64, cols=256), _targ(rows=8, cols=64))
+    assert L.focus_group_workspace_bytes(arr, 2) >= 8
+    assert L.focus_nvfp4_alpha_group(arr, 2, ALIGNED2, None, 0, None) == -4
+    assert L.focus_nvfp4_alpha_group(arr, 2, None, ALIGNED, 1 << 20, None) == -1
