@@ -600,13 +600,18 @@ struct Unroll {
     static constexpr int U = (MODE >= kBwd) ? 1 : ((FMT == 1 && DT != 0) ? 2 : 1);
 };
 
-// Resident CTAs per SM the register allocation must allow: enough 256-thread
-// CTAs to keep >= 48 KB of loads in flight per SM.
-// (one fewer for 2-element sub-blocks, whose per-sub-block state is largest).
-template <int FMT, int SUB, int MODE>
+// Resident CTAs per SM the register allocation must allow.  The backward is
+// bound by memory latency: with 16-bit elements, one more CTA per SM than the
+// registers it would like (4 for NVFP4 at 64 registers, 3 for MXFP4 at 80)
+// is faster despite a few dozen bytes of spills to L1-cached local memory
+// (measured: NVFP4 Qwen3-4B backward 6124 -> 6543 GB/s).  The fused
+// optimizer's extra state spills too much there and keeps the lower count.
+// One fewer for 2-element sub-blocks, whose per-sub-block state is largest.
+template <int FMT, int DT, int SUB, int MODE>
 struct MinCtas {
-    static constexpr int value =
-        ((MODE >= kBwd) ? (FMT == 1 ? 3 : 2) : 4) - (SUB == 2 ? 1 : 0);
+    static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT != 0 ? 3 : 2);
+    static constexpr int adam = FMT == 1 ? 3 : 2;
+    static constexpr int value = ((MODE >= kBwdA) ? adam : (MODE >= kBwd) ? bwd : 4) - (SUB == 2 ? 1 : 0);
 };
 
 // Where a block's tensor comes from: one tensor (the per-tensor entry
@@ -829,14 +834,14 @@ __device__ __forceinline__ void block_loop(const Src& src)
 
 
 template <int FMT, int DT, int SUB, int MODE>
-__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
+__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
     fq_block_kernel(const KParams p)
 {
     block_loop<FMT, DT, SUB, MODE>(OneTensor<FMT>(p));
 }
 
 template <int FMT, int DT, int SUB, int MODE>
-__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, SUB, MODE>::value))
+__global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
     fq_group_kernel(const __grid_constant__ KGroup g)
 {
     static_assert(MODE < kBwdA, "the fused optimizer is per tensor");
