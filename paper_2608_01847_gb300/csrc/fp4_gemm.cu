@@ -10,11 +10,16 @@
 //   warp 0     TMA producer: per K chunk of 256 elements (128 bytes of codes
 //              per row) the A and B code tiles (2D TMA, 128-byte swizzle)
 //              and their scale tiles (1D bulk copies) into a ring of stages;
-//   warp 1     MMA issuer: scale tiles shared -> tensor memory (tcgen05.cp),
-//              four K = 64 block-scaled MMAs per chunk into an accumulator
-//              in tensor memory, commit to free the stage;
+//   warp 1     MMA issuer: four K = 64 block-scaled MMAs per chunk into an
+//              accumulator in tensor memory, commit to free the stage;
 //   warps 2-5  epilogue: accumulator -> registers (one lane quarter each),
-//              alpha scaling, fp32 or bf16 stores.
+//              alpha scaling, fp32 or bf16 stores;
+//   warps 6-9  scale warps: the chunk's scale tiles shared -> tensor memory
+//              (tcgen05.st, one lane quarter each), alternating between two
+//              sets of scale regions, handed to the MMA thread by mbarrier.
+// Writing the scales with tcgen05.st from these warps keeps them off the
+// tensor pipe: copied there with tcgen05.cp they serialised with the MMAs
+// and cost about 40 % of the run time.
 // Two accumulators in tensor memory let the epilogue of one tile overlap
 // the main loop of the next.
 //
@@ -24,7 +29,7 @@
 // n / 32.  Lane l of every quarter must therefore hold, in the four
 // columns, the scale words of rows l, l + 32, l + 64, l + 96: exactly line l
 // of a 128 x 4 export tile, which tcgen05.cp .32x128b.warpx4 broadcasts to
-// all four quarters.  A word holds consecutive K blocks in byte order: one
+// all four quarters (the scale warps write exactly that).  A word holds consecutive K blocks in byte order: one
 // NVFP4 step uses all four bytes, an MXFP4 tile feeds two steps (bytes 0-1,
 // then bytes 2-3 through the scale data id).
 #include <cstdint>
@@ -49,13 +54,20 @@ constexpr int kTileBytes = kTile * kChunk;          // 16 KB of codes per operan
 constexpr int kSfBytes = 4 * 512;                   // up to four scale tiles per operand
 constexpr int kStageBytes = 2 * kTileBytes + 2 * kSfBytes;
 constexpr int kSmemBytes = kStages * kStageBytes + 1024;   // + alignment slack
-constexpr int kThreads = 192;         // producer, MMA, four epilogue warps
-// tensor memory: accumulators in columns 0-127 and 128-255; scale regions
-// for the four steps of a chunk at 256 + 16 j (A) and 320 + 16 j (B), each
-// 4 columns (every region on a 16-column boundary).
+constexpr int kThreads = 320;         // producer, MMA, four epilogue warps, four scale warps
+// tensor memory: the accumulator, then sets of scale regions used by chunks
+// in turn (set k % kSfSets); inside a set, the four steps of a chunk at
+// + 16 j (A) and + 64 + 16 j (B), each 4 columns (every region on a
+// 16-column boundary).  Two accumulators let the epilogue of one tile
+// overlap the main loop of the next (measured: worth more than a third
+// scale set, for which one accumulator would have to go).
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kSfa = 256, kSfb = 320, kSfStep = 16;
-constexpr uint32_t kWaitLimit = 1u << 22;
+constexpr uint32_t kAccBufs = 2;      // accumulators, 128 columns each, from column 0
+constexpr uint32_t kSfSets = 2;       // scale sets, 128 columns each, after the accumulators
+constexpr uint32_t kSfBase = 128 * kAccBufs;
+constexpr uint32_t kSfa = 0, kSfb = 64, kSfStep = 16, kSfSet = 128;   // inside a set
+static_assert(kSfBase + kSfSets * kSfSet <= kTmemCols, "tensor memory");
+constexpr uint32_t kWaitLimit = 1u << 24;   // polls; each try_wait may suspend for a while
 
 struct GemmParams {
     const uint8_t* sfa;    // scale tiles of A
@@ -83,7 +95,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const GemmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2];
+    __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], sf_full[kSfSets];
     __shared__ uint32_t tbase;
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     auto stage_a = [&](uint32_t s) { return smem + s * kStageBytes; };
@@ -101,6 +113,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_init(&acc_full[b], 1);
             tc::mbar_init(&acc_empty[b], 128);
         }
+        for (uint32_t b = 0; b < kSfSets; ++b) tc::mbar_init(&sf_full[b], 128);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 0) {
@@ -124,7 +137,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
                 const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
                 for (uint32_t c = 0; c < n_chunks; ++c) {
-                    if (!tc::mbar_wait(&empty[s], ph ^ 1, kWaitLimit)) {
+                    if (!tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit)) {
                         ok = false;
                         give_up(p);
                         break;
@@ -151,35 +164,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
         if (lane == 0) {
-            uint32_t s = 0, ph = 0, acc = 0, acc_ph = 0;
+            uint32_t s = 0, ph = 0, acc = 0, acc_ph = 0, k = 0;
             bool ok = true;
             for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-                if (!tc::mbar_wait(&acc_empty[acc], acc_ph ^ 1, kWaitLimit)) {
+                if (!tc::mbar_wait_hot(&acc_empty[acc], acc_ph ^ 1, kWaitLimit)) {
                     give_up(p);
                     break;
                 }
                 tc::tc_fence_after();
                 const uint32_t d_tmem = tb + acc * kTile;
                 for (uint32_t c = 0; c < n_chunks; ++c) {
-                    if (!tc::mbar_wait(&full[s], ph, kWaitLimit)) {
+                    // codes in shared memory, then this chunk's scales in tensor memory
+                    const uint32_t set = k % kSfSets;
+                    if (!tc::mbar_wait_hot(&full[s], ph, kWaitLimit) ||
+                        !tc::mbar_wait_hot(&sf_full[set], (k / kSfSets) & 1u, kWaitLimit)) {
                         ok = false;
                         give_up(p);
                         break;
                     }
+                    ++k;
                     tc::tc_fence_after();
                     const uint32_t steps = min(4u, p.n_steps - 4 * c);
-                    const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
-                    const uint32_t sa = tc::smem_u32(stage_sfa(s)), sb = tc::smem_u32(stage_sfb(s));
-                    for (uint32_t j = 0; j < sf_tiles; ++j) {
-                        tc::tmem_cp_32x128b_x4(tb + kSfa + kSfStep * j, sa + 512 * j);
-                        tc::tmem_cp_32x128b_x4(tb + kSfb + kSfStep * j, sb + 512 * j);
-                    }
+                    const uint32_t sfbase = tb + kSfBase + kSfSet * set;
                     const uint32_t a0 = tc::smem_u32(stage_a(s)), b0 = tc::smem_u32(stage_b(s));
                     for (uint32_t kk = 0; kk < steps; ++kk) {
                         const uint64_t ad = tc::smem_desc_sw128(a0 + 32 * kk);
                         const uint64_t bd = tc::smem_desc_sw128(b0 + 32 * kk);
                         const uint32_t j = kk / steps_per_tile;
-                        const uint32_t sfa = tb + kSfa + kSfStep * j, sfb = tb + kSfb + kSfStep * j;
+                        const uint32_t sfa = sfbase + kSfa + kSfStep * j, sfb = sfbase + kSfb + kSfStep * j;
                         const uint32_t accumulate = (c > 0 || kk > 0) ? 1u : 0u;
                         if (FMT == 0)
                             tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTile, true, 2 * (kk % 2)), sfa, sfb,
@@ -196,9 +208,50 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!ok) break;
                 tc::mma_commit(&acc_full[acc]);
-                if (++acc == 2) {
+                if (++acc == kAccBufs) {
                     acc = 0;
                     acc_ph ^= 1;
+                }
+            }
+        }
+    } else if (warp >= 6) {
+        // ---------------- scale warps (warps 6-9: lane quarters 2, 3, 0, 1) ----------------
+        // Chunk k (counted over all tiles of this CTA) uses stage k % kStages
+        // and scale set k % 2.  Before a set is rewritten, the MMAs of chunk
+        // k - 2, which read it, must be complete: their commit completed the
+        // empty barrier of that chunk's stage.
+        const uint32_t q = warp % 4;
+        const uint32_t lane_addr = tb + ((q * 32) << 16);
+        uint32_t s = 0, ph = 0, k = 0;
+        bool ok = true;
+        for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+            for (uint32_t c = 0; c < n_chunks; ++c, ++k) {
+                bool got = tc::mbar_wait_hot(&full[s], ph, kWaitLimit);
+                if (k >= kSfSets) {
+                    const uint32_t k2 = k - kSfSets;
+                    got = got && tc::mbar_wait_hot(&empty[k2 % kStages], (k2 / kStages) & 1u, kWaitLimit);
+                }
+                if (!__all_sync(0xffffffffu, got)) {
+                    if (lane == 0) give_up(p);
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                const uint32_t steps = min(4u, p.n_steps - 4 * c);
+                const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
+                const uint32_t sfbase = lane_addr + kSfBase + kSfSet * (k % kSfSets);
+                for (uint32_t j = 0; j < sf_tiles; ++j) {
+                    const uint4 la = *reinterpret_cast<const uint4*>(stage_sfa(s) + 512 * j + 16 * lane);
+                    const uint4 lb = *reinterpret_cast<const uint4*>(stage_sfb(s) + 512 * j + 16 * lane);
+                    tc::tmem_st_x4(sfbase + kSfa + kSfStep * j, la.x, la.y, la.z, la.w);
+                    tc::tmem_st_x4(sfbase + kSfb + kSfStep * j, lb.x, lb.y, lb.z, lb.w);
+                }
+                tc::tmem_wait_st();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&sf_full[k % kSfSets]);
+                if (++s == kStages) {
+                    s = 0;
+                    ph ^= 1;
                 }
             }
         }
@@ -210,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t acc = 0, acc_ph = 0;
         for (uint32_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
             const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
-            const bool got = __all_sync(0xffffffffu, tc::mbar_wait(&acc_full[acc], acc_ph, kWaitLimit));
+            const bool got = __all_sync(0xffffffffu, tc::mbar_wait_hot(&acc_full[acc], acc_ph, kWaitLimit));
             if (!got) {
                 if (lane == 0) give_up(p);
                 break;
@@ -266,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
-            if (++acc == 2) {
+            if (++acc == kAccBufs) {
                 acc = 0;
                 acc_ph ^= 1;
             }
