@@ -139,3 +139,84 @@ def test_full_size_shared_rows(fmt, tmp_path):
     rb = O.bwd(np.ascontiguousarray(xs), np.ascontiguousarray(gs), fmt, crs=ch, dgs=dh, alpha=a,
                sub=sub, shared=True)
     assert_bits_equal(host(gx.index_select(0, torch.from_numpy(rs).cuda())), rb["gx"], "shared gx")
+
+
+# ---------------------------------------------------------------------------
+# learnable S^fp and the fused AdamW step at full size (sampled rows)
+# ---------------------------------------------------------------------------
+def _sfp_init(x, fmt, a_dev, seed):
+    """S^fp as the benchmark initialises it: the absmax scale moved by U(0.9, 1.1)."""
+    block = 32 if fmt == O.MXFP4 else 16
+    rows, cols = x.shape
+    m = x.float().abs().view(rows, cols // block, block).amax(-1)
+    den = a_dev * 6.0 if fmt == O.NVFP4 else torch.full((1,), 6.0, device=x.device)
+    gen = torch.Generator(device=x.device)
+    gen.manual_seed(seed)
+    return (m / den * (torch.rand(m.shape, generator=gen, device=x.device) * 0.2 + 0.9)).contiguous()
+
+
+@pytest.mark.parametrize("name,fmt,idx", [("qwen3_4b_layer", O.NVFP4, 4), ("llama_70b_layer", O.MXFP4, 6)])
+def test_full_size_learnable_scale(name, fmt, idx):
+    w = W.WORKLOADS[name]
+    block = 32 if fmt == O.MXFP4 else 16
+    x, g = W.device_tensor(w, idx, "cuda")
+    crs, dgs = W.device_coefs(w, idx, block, 8, "cuda")
+    a_dev = F.focus_nvfp4_alpha(x) if fmt == O.NVFP4 else torch.zeros(1, device="cuda")
+    sfp = _sfp_init(x, fmt, a_dev, 11)
+    y, sb = F.focus_fq_fwd(x, fmt, crs, dgs, a_dev, want_scales=True, sfp=sfp)
+    codes, _ = F.focus_pack(x, fmt, crs, dgs, a_dev, sfp=sfp)
+    gx, gc, gd, gs = F.focus_fq_bwd(x, g, fmt, crs, dgs, a_dev, sfp=sfp)
+    torch.cuda.synchronize()
+    rows = x.shape[0]
+    a = float(host(a_dev)[0]) if fmt == O.NVFP4 else 0.0
+    rng = np.random.default_rng(idx + 100)
+    rs = np.unique(np.concatenate([[0, rows - 1], rng.choice(rows, 24, replace=False)]))
+    ri = torch.from_numpy(rs).cuda()
+    sel = lambda t: host(t.index_select(0, ri))
+    xs, gsel, cs, ds, ss = sel(x), sel(g), sel(crs), sel(dgs), sel(sfp)
+    ref = O.fwd(xs, fmt, crs=cs, dgs=ds, alpha=a, sfp=ss, want_codes=True)
+    rb = O.bwd(xs, gsel, fmt, crs=cs, dgs=ds, alpha=a, sfp=ss, want_abs=True, want_gsfp=True)
+    assert_bits_equal(sel(y), ref["y"], f"{name} y")
+    assert_bits_equal(sel(sb), ref["scales"], f"{name} scale bytes")
+    assert_bits_equal(sel(codes), ref["codes"], f"{name} codes")
+    assert_bits_equal(sel(gx), rb["gx"], f"{name} gx")
+    assert_grad_close(sel(gc), rb["gcrs"], rb["gcrs_abs"], FLOOR_ROW, f"{name} dL/dc")
+    assert_grad_close(sel(gd), rb["gdgs"], rb["gdgs_abs"], FLOOR_ROW, f"{name} dL/dc^k")
+    assert_grad_close(sel(gs), rb["gsfp"], rb["gsfp_abs"], FLOOR_ROW, f"{name} dL/dS^fp")
+
+
+@pytest.mark.parametrize("name,fmt,idx", [("qwen3_4b_layer", O.NVFP4, 4), ("llama_70b_layer", O.MXFP4, 6)])
+def test_full_size_fused_adamw(name, fmt, idx):
+    from gpu_helpers import assert_adamw_close
+    hp = dict(lr_coef=5e-2 if fmt == O.MXFP4 else 1e-3, lr_scale=2e-2 * 2.0 ** -7 if fmt == O.MXFP4 else 5e-3,
+              beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+    w = W.WORKLOADS[name]
+    block = 32 if fmt == O.MXFP4 else 16
+    x, g = W.device_tensor(w, idx, "cuda")
+    crs, dgs = W.device_coefs(w, idx, block, 8, "cuda")
+    a_dev = F.focus_nvfp4_alpha(x) if fmt == O.NVFP4 else torch.zeros(1, device="cuda")
+    sfp = _sfp_init(x, fmt, a_dev, 12)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(idx)
+    params = {"crs": crs, "dgs": dgs, "sfp": sfp}
+    before = {k: v.clone() for k, v in params.items()}
+    moments = {k: ((torch.rand(v.shape, generator=gen, device="cuda") - 0.5) * 0.1,
+                   torch.rand(v.shape, generator=gen, device="cuda") * 0.01) for k, v in params.items()}
+    mom0 = {k: (m.clone(), v.clone()) for k, (m, v) in moments.items()}
+    step = torch.tensor([7], dtype=torch.int64, device="cuda")
+    gx = F.focus_fq_bwd_adamw(x, g, fmt, step, hp, crs=crs, dgs=dgs, sfp=sfp, moments=moments, alpha=a_dev)
+    torch.cuda.synchronize()
+    rows = x.shape[0]
+    a = float(host(a_dev)[0]) if fmt == O.NVFP4 else 0.0
+    rng = np.random.default_rng(idx + 200)
+    rs = np.unique(np.concatenate([[0, rows - 1], rng.choice(rows, 24, replace=False)]))
+    ri = torch.from_numpy(rs).cuda()
+    sel = lambda t: host(t.index_select(0, ri))
+    p0 = {k: sel(v) for k, v in before.items()}
+    m0 = {k: (sel(m), sel(v)) for k, (m, v) in mom0.items()}
+    ref = O.bwd_adamw(sel(x), sel(g), fmt, p0, m0, hp, 7, alpha=a)
+    assert_bits_equal(sel(gx), ref["gx"], f"{name} gx")
+    for k in params:
+        lr = hp["lr_scale"] if k == "sfp" else hp["lr_coef"]
+        assert_adamw_close((sel(params[k]), sel(moments[k][0]), sel(moments[k][1])), p0[k], m0[k][0], m0[k][1],
+                           ref[k], FLOOR_ROW, lr, hp, 7, f"{name} {k}")
