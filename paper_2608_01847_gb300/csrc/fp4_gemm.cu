@@ -6,37 +6,43 @@
 // the paper's "no inference overhead" refers to (Sec. 1, Sec. 3.1): only the
 // exported codes and hardware scales enter the product.
 //
-// Persistent, warp-specialised kernel, one CTA per SM, 128 x 128 tiles of D:
+// Persistent, warp-specialised kernel, one CTA per SM, 128 x 256 tiles of D
+// (one M = 128, N = 256 MMA per K = 64 step):
 //   warp 0     TMA producer: per K chunk of 256 elements (128 bytes of codes
 //              per row) the A and B code tiles (2D TMA, 128-byte swizzle)
 //              and their scale tiles (1D bulk copies) into a ring of stages;
 //   warp 1     MMA issuer: four K = 64 block-scaled MMAs per chunk into an
 //              accumulator in tensor memory, commit to free the stage;
 //   warps 2-5  epilogue: accumulator -> registers (one lane quarter each),
-//              alpha scaling, fp32 or bf16 stores;
+//              alpha scaling, then 32-row x 128-byte boxes of D staged in
+//              shared memory and written by TMA stores;
 //   warps 6-9  scale warps: the chunk's scale tiles shared -> tensor memory
 //              (tcgen05.st, one lane quarter each), alternating between two
 //              sets of scale regions, handed to the MMA thread by mbarrier.
 // Writing the scales with tcgen05.st from these warps keeps them off the
 // tensor pipe: copied there with tcgen05.cp they serialised with the MMAs
-// and cost about 40 % of the run time.
-// Two accumulators in tensor memory let the epilogue of one tile overlap
-// the main loop of the next.
+// and cost about 40 % of the run time.  Per-lane row stores of D (32 rows
+// per warp instruction) cost a third of the run time; the staged TMA stores
+// write whole lines.  The 256-column accumulator fills half of tensor
+// memory, the scale sets the other half, so there is one accumulator: the
+// bf16 epilogue holds its whole row in registers and releases it before
+// staging.
 //
-// Scale factors in tensor memory (M = N = 128): one MMA step reads a
-// 4-column region; row m of A takes lane m, column m / 32; column n of B is
-// read by each 32-lane quarter from its own quarter, lane n % 32, column
-// n / 32.  Lane l of every quarter must therefore hold, in the four
-// columns, the scale words of rows l, l + 32, l + 64, l + 96: exactly line l
-// of a 128 x 4 export tile, which tcgen05.cp .32x128b.warpx4 broadcasts to
-// all four quarters (the scale warps write exactly that).  A word holds consecutive K blocks in byte order: one
-// NVFP4 step uses all four bytes, an MXFP4 tile feeds two steps (bytes 0-1,
-// then bytes 2-3 through the scale data id).
+// Scale factors in tensor memory: one MMA step reads an A region of 4
+// columns and a B region of 8; row m of A takes lane m, column m / 32;
+// column n of B is read by each 32-lane quarter from its own quarter, lane
+// n % 32, column n / 32.  Lane l of every quarter must therefore hold, in
+// four consecutive columns, the scale words of rows l, l + 32, l + 64,
+// l + 96 of a 128-row group: exactly line l of a 128 x 4 export tile (B
+// rows 128-255 take the next four columns).  A word holds consecutive K
+// blocks in byte order: one NVFP4 step uses all four bytes, an MXFP4 tile
+// feeds two steps (bytes 0-1, then bytes 2-3 through the scale data id).
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <algorithm>
+#include <cstring>
 #include <mutex>
 
 #include "../../include/focus_fq.h"
@@ -47,24 +53,32 @@
 namespace focus {
 namespace {
 
-constexpr int kTile = 128;            // M and N of a CTA tile
+constexpr int kTile = 128;            // M of a CTA tile (rows of A)
+constexpr int kTileN = 256;           // N of a CTA tile (rows of B)
 constexpr int kChunk = 128;           // K bytes (256 FP4) per stage
-constexpr int kStages = 5;
-constexpr int kTileBytes = kTile * kChunk;          // 16 KB of codes per operand
-constexpr int kSfBytes = 4 * 512;                   // up to four scale tiles per operand
-constexpr int kStageBytes = 2 * kTileBytes + 2 * kSfBytes;
-constexpr int kSmemBytes = kStages * kStageBytes + 1024;   // + alignment slack
+constexpr int kStages = 3;
+constexpr int kTileBytes = kTile * kChunk;          // 16 KB of A codes
+constexpr int kTileBytesB = kTileN * kChunk;        // 32 KB of B codes
+constexpr int kSfBytes = 4 * 512;                   // up to four scale tiles of A
+constexpr int kSfBytesB = 2 * kSfBytes;             // the same for both 128-row halves of B
+constexpr int kStageBytes = kTileBytes + kTileBytesB + kSfBytes + kSfBytesB;   // 54 KB, 1024-aligned
+// output staging: per epilogue warp two buffers of 32 rows x 128 bytes of D
+// (128-byte swizzle), written to global memory by TMA stores
+constexpr int kOutBox = 32 * 128;
+constexpr int kOutBufs = 2;
+constexpr int kSmemBytes = kStages * kStageBytes + 4 * kOutBufs * kOutBox + 1024;   // + alignment slack
 constexpr int kThreads = 320;         // producer, MMA, four epilogue warps, four scale warps
-// tensor memory: the accumulator, then sets of scale regions used by chunks
-// in turn (set k % kSfSets); inside a set, the four steps of a chunk at
-// + 16 j (A) and + 64 + 16 j (B), each 4 columns (every region on a
-// 16-column boundary).  Two accumulators let the epilogue of one tile
-// overlap the main loop of the next (measured: worth more than a third
-// scale set, for which one accumulator would have to go).
+// tensor memory: the 256-column accumulator, then two sets of scale regions
+// used by chunks in turn (set k % 2); inside a set, the four steps of a chunk
+// at + 16 j (A, 4 columns) and + 64 + 16 j (B, 8 columns: B rows 0-127 in
+// the first four, rows 128-255 in the next four -- column n of an N = 256
+// MMA is read from column n / 32).  Every region starts on a 16-column
+// boundary.  The epilogue releases the accumulator as soon as it has been
+// read into registers, before its stores.
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAccBufs = 2;      // accumulators, 128 columns each, from column 0
+constexpr uint32_t kAccBufs = 1;      // accumulators, kTileN columns each, from column 0
 constexpr uint32_t kSfSets = 2;       // scale sets, 128 columns each, after the accumulators
-constexpr uint32_t kSfBase = 128 * kAccBufs;
+constexpr uint32_t kSfBase = kTileN * kAccBufs;
 constexpr uint32_t kSfa = 0, kSfb = 64, kSfStep = 16, kSfSet = 128;   // inside a set
 static_assert(kSfBase + kSfSets * kSfSet <= kTmemCols, "tensor memory");
 constexpr uint32_t kWaitLimit = 1u << 24;   // polls; each try_wait may suspend for a while
@@ -79,9 +93,10 @@ struct GemmParams {
     int64_t M, N, ldd;
     uint32_t tiles_k;      // scale tiles per 128-row tile row: ceil(K / block / 4)
     uint32_t tiles_m, tiles_n;
+    uint32_t tile_rows_b;  // 128-row scale-tile rows of B: ceil(N / 128)
     uint32_t n_steps;      // K / 64
     int d_bf16;
-    int d_vec;             // rows of D start on 16-byte boundaries (vector stores)
+    int d_vec;             // rows of D start on 16-byte boundaries: TMA stores through tma_d
 };
 
 __device__ __forceinline__ void give_up(const GemmParams& p)
@@ -92,7 +107,7 @@ __device__ __forceinline__ void give_up(const GemmParams& p)
 template <int FMT>
 __global__ void __launch_bounds__(kThreads, 1)
     fp4_gemm_kernel(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b,
-                    const GemmParams p)
+                    const __grid_constant__ CUtensorMap tma_d, const GemmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], sf_full[kSfSets];
@@ -100,8 +115,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     auto stage_a = [&](uint32_t s) { return smem + s * kStageBytes; };
     auto stage_b = [&](uint32_t s) { return smem + s * kStageBytes + kTileBytes; };
-    auto stage_sfa = [&](uint32_t s) { return smem + s * kStageBytes + 2 * kTileBytes; };
-    auto stage_sfb = [&](uint32_t s) { return smem + s * kStageBytes + 2 * kTileBytes + kSfBytes; };
+    auto stage_sfa = [&](uint32_t s) { return smem + s * kStageBytes + kTileBytes + kTileBytesB; };
+    auto stage_sfb = [&](uint32_t s) { return smem + s * kStageBytes + kTileBytes + kTileBytesB + kSfBytes; };
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     if (threadIdx.x == 0) {
@@ -145,15 +160,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t steps = min(4u, p.n_steps - 4 * c);
                     const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
                     const uint32_t tile0 = (4 * c) / steps_per_tile;
-                    tc::mbar_arrive_expect_tx(&full[s], 2 * kTileBytes + 2 * sf_tiles * 512);
+                    const bool hi = 2 * tn + 1 < p.tile_rows_b;   // second 128-row half of B exists
+                    tc::mbar_arrive_expect_tx(&full[s], kTileBytes + kTileBytesB + (hi ? 3 : 2) * sf_tiles * 512);
                     tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
                                     static_cast<int32_t>(tm * kTile), &full[s]);
                     tc::tma_load_2d(stage_b(s), &tma_b, static_cast<int32_t>(c * kChunk),
-                                    static_cast<int32_t>(tn * kTile), &full[s]);
+                                    static_cast<int32_t>(tn * kTileN), &full[s]);
                     tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
                                   sf_tiles * 512, &full[s]);
-                    tc::bulk_load(stage_sfb(s), p.sfb + (static_cast<size_t>(tn) * p.tiles_k + tile0) * 512,
+                    tc::bulk_load(stage_sfb(s), p.sfb + (static_cast<size_t>(2 * tn) * p.tiles_k + tile0) * 512,
                                   sf_tiles * 512, &full[s]);
+                    if (hi)
+                        tc::bulk_load(stage_sfb(s) + kSfBytes,
+                                      p.sfb + (static_cast<size_t>(2 * tn + 1) * p.tiles_k + tile0) * 512,
+                                      sf_tiles * 512, &full[s]);
                     if (++s == kStages) {
                         s = 0;
                         ph ^= 1;
@@ -172,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc::tc_fence_after();
-                const uint32_t d_tmem = tb + acc * kTile;
+                const uint32_t d_tmem = tb + acc * kTileN;
                 for (uint32_t c = 0; c < n_chunks; ++c) {
                     // codes in shared memory, then this chunk's scales in tensor memory
                     const uint32_t set = k % kSfSets;
@@ -194,10 +214,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint32_t sfa = sfbase + kSfa + kSfStep * j, sfb = sfbase + kSfb + kSfStep * j;
                         const uint32_t accumulate = (c > 0 || kk > 0) ? 1u : 0u;
                         if (FMT == 0)
-                            tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTile, true, 2 * (kk % 2)), sfa, sfb,
+                            tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, true, 2 * (kk % 2)), sfa, sfb,
                                          accumulate);
                         else
-                            tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTile, false), sfa, sfb,
+                            tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, false), sfa, sfb,
                                          accumulate);
                     }
                     tc::mma_commit(&empty[s]);
@@ -243,8 +263,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (uint32_t j = 0; j < sf_tiles; ++j) {
                     const uint4 la = *reinterpret_cast<const uint4*>(stage_sfa(s) + 512 * j + 16 * lane);
                     const uint4 lb = *reinterpret_cast<const uint4*>(stage_sfb(s) + 512 * j + 16 * lane);
+                    const uint4 lh = *reinterpret_cast<const uint4*>(stage_sfb(s) + kSfBytes + 512 * j + 16 * lane);
                     tc::tmem_st_x4(sfbase + kSfa + kSfStep * j, la.x, la.y, la.z, la.w);
                     tc::tmem_st_x4(sfbase + kSfb + kSfStep * j, lb.x, lb.y, lb.z, lb.w);
+                    // rows 128-255 of B (stale but finite-or-not bytes when B has no such
+                    // rows: they only reach columns of D that are not stored)
+                    tc::tmem_st_x4(sfbase + kSfb + kSfStep * j + 4, lh.x, lh.y, lh.z, lh.w);
                 }
                 tc::tmem_wait_st();
                 tc::tc_fence_before();
@@ -261,6 +285,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lane_addr = tb + ((q * 32) << 16);
         const float scale = FMT == 1 ? __fmul_rn(__ldg(p.alpha_a), __ldg(p.alpha_b)) : 1.0f;
         uint32_t acc = 0, acc_ph = 0;
+        // staging buffers of this warp; lane 0 tracks which committed bulk
+        // group last read each one
+        uint8_t* const obase = smem + kStages * kStageBytes + (warp - 2) * kOutBufs * kOutBox;
+        uint32_t obuf = 0, ngroups = 0;
+        uint32_t last_group[kOutBufs];
+#pragma unroll
+        for (int b = 0; b < kOutBufs; ++b) last_group[b] = 0xffffffffu;
+        // the next buffer, once the store that last read it is done reading
+        auto out_stage = [&](uint32_t ob) {
+            const uint32_t b = ob % kOutBufs;
+            if (lane == 0 && last_group[b] != 0xffffffffu) {
+                if (ngroups - 1 - last_group[b] == 0) tc::bulk_wait_read<0>();
+                else tc::bulk_wait_read<1>();
+            }
+            __syncwarp();
+            return obase + b * kOutBox;
+        };
+        auto out_issue = [&](uint8_t* buf, int32_t x, int32_t y) {
+            tc::fence_async_smem();
+            __syncwarp();
+            if (lane == 0 && x < p.N && y < p.M) {
+                tc::tma_store_2d(&tma_d, buf, x, y);
+                tc::bulk_commit();
+                last_group[obuf % kOutBufs] = ngroups++;
+            }
+            ++obuf;
+        };
         for (uint32_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
             const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
             const bool got = __all_sync(0xffffffffu, tc::mbar_wait_hot(&acc_full[acc], acc_ph, kWaitLimit));
@@ -270,52 +321,89 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc::tc_fence_after();
             const int64_t m = static_cast<int64_t>(tm) * kTile + q * 32 + lane;
-            const int64_t n0 = static_cast<int64_t>(tn) * kTile;
+            const int64_t n0 = static_cast<int64_t>(tn) * kTileN;
+            if (p.d_vec) {
+                // D through shared memory: per 32-row x 128-byte box, each
+                // lane writes its row (16-byte chunk j of row r at chunk
+                // j ^ (r % 8), the TMA 128-byte swizzle), then lane 0 issues
+                // the TMA store.  Rows >= M and columns >= N are clipped by
+                // the tensor map.
+                const int32_t y = static_cast<int32_t>(tm) * kTile + q * 32;
+                if (p.d_bf16) {
+                    // the whole row of the tile in registers first, so that the
+                    // accumulator is released before any staging
+                    uint32_t w[kTileN / 2];
+#pragma unroll
+                    for (int cb = 0; cb < kTileN / 32; ++cb) {
+                        uint32_t r[32];
+                        tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * cb, r);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const __nv_bfloat162 h = __floats2bfloat162_rn(
+                                __fmul_rn(__uint_as_float(r[2 * e]), scale), __fmul_rn(__uint_as_float(r[2 * e + 1]), scale));
+                            w[16 * cb + e] = *reinterpret_cast<const uint32_t*>(&h);
+                        }
+                    }
+                    tc::tc_fence_before();
+                    tc::mbar_arrive(&acc_empty[acc]);
+#pragma unroll
+                    for (int i = 0; i < kTileN / 64; ++i) {
+                        uint8_t* buf = out_stage(obuf);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            *reinterpret_cast<uint4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                make_uint4(w[32 * i + 4 * j], w[32 * i + 4 * j + 1], w[32 * i + 4 * j + 2],
+                                           w[32 * i + 4 * j + 3]);
+                        out_issue(buf, static_cast<int32_t>(n0) + 64 * i, y);
+                    }
+                } else {
 #pragma unroll 1
-            for (int cb = 0; cb < kTile / 32; ++cb) {
+                    for (int cb = 0; cb < kTileN / 32; ++cb) {
+                        uint32_t r[32];
+                        tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * cb, r);
+                        tc::tmem_wait_ld();
+                        if (cb == kTileN / 32 - 1) {
+                            tc::tc_fence_before();
+                            tc::mbar_arrive(&acc_empty[acc]);
+                        }
+                        uint8_t* buf = out_stage(obuf);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                make_float4(__fmul_rn(__uint_as_float(r[4 * j]), scale),
+                                            __fmul_rn(__uint_as_float(r[4 * j + 1]), scale),
+                                            __fmul_rn(__uint_as_float(r[4 * j + 2]), scale),
+                                            __fmul_rn(__uint_as_float(r[4 * j + 3]), scale));
+                        out_issue(buf, static_cast<int32_t>(n0) + 32 * cb, y);
+                    }
+                }
+                if (++acc == kAccBufs) {
+                    acc = 0;
+                    acc_ph ^= 1;
+                }
+                continue;
+            }
+#pragma unroll 1
+            for (int cb = 0; cb < kTileN / 32; ++cb) {
                 uint32_t r[32];
-                tc::tmem_ld_x32(lane_addr + acc * kTile + 32 * cb, r);
+                tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * cb, r);
                 tc::tmem_wait_ld();
-                if (cb == kTile / 32 - 1) {
+                if (cb == kTileN / 32 - 1) {
                     // the accumulator is free once its last columns are in registers
                     tc::tc_fence_before();
                     tc::mbar_arrive(&acc_empty[acc]);
                 }
+                // rows of D off 16-byte boundaries: element stores
                 if (m < p.M) {
                     const int64_t nb = n0 + 32 * cb;
                     if (p.d_bf16) {
                         __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.d) + m * p.ldd + nb;
-                        if (nb + 32 <= p.N && p.d_vec) {
-#pragma unroll
-                            for (int i = 0; i < 32; i += 8) {
-                                uint32_t w[4];
-#pragma unroll
-                                for (int e = 0; e < 4; ++e) {
-                                    const __nv_bfloat162 h = __floats2bfloat162_rn(
-                                        __fmul_rn(__uint_as_float(r[i + 2 * e]), scale),
-                                        __fmul_rn(__uint_as_float(r[i + 2 * e + 1]), scale));
-                                    w[e] = *reinterpret_cast<const uint32_t*>(&h);
-                                }
-                                *reinterpret_cast<uint4*>(dst + i) = make_uint4(w[0], w[1], w[2], w[3]);
-                            }
-                        } else {
-                            for (int i = 0; i < 32 && nb + i < p.N; ++i)
-                                dst[i] = __float2bfloat16_rn(__fmul_rn(__uint_as_float(r[i]), scale));
-                        }
+                        for (int i = 0; i < 32 && nb + i < p.N; ++i)
+                            dst[i] = __float2bfloat16_rn(__fmul_rn(__uint_as_float(r[i]), scale));
                     } else {
                         float* dst = static_cast<float*>(p.d) + m * p.ldd + nb;
-                        if (nb + 32 <= p.N && p.d_vec) {
-#pragma unroll
-                            for (int i = 0; i < 32; i += 4)
-                                *reinterpret_cast<float4*>(dst + i) =
-                                    make_float4(__fmul_rn(__uint_as_float(r[i]), scale),
-                                                __fmul_rn(__uint_as_float(r[i + 1]), scale),
-                                                __fmul_rn(__uint_as_float(r[i + 2]), scale),
-                                                __fmul_rn(__uint_as_float(r[i + 3]), scale));
-                        } else {
-                            for (int i = 0; i < 32 && nb + i < p.N; ++i)
-                                dst[i] = __fmul_rn(__uint_as_float(r[i]), scale);
-                        }
+                        for (int i = 0; i < 32 && nb + i < p.N; ++i) dst[i] = __fmul_rn(__uint_as_float(r[i]), scale);
                     }
                 }
             }
@@ -325,6 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     }
+    if (warp >= 2 && warp < 6 && lane == 0) tc::bulk_wait_all();   // output stores complete
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -364,18 +453,20 @@ EncodeTiled encode_fn()
     return fn;
 }
 
-// Tensor map of a [rows, row_bytes] code matrix, boxes of 128 rows x 128
-// bytes, 128-byte swizzle, zero fill outside.
-bool make_map(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t row_bytes)
+// Tensor map of a row-major [rows, cols] matrix with row pitch `pitch`
+// bytes, boxes of box_rows rows x 128 bytes, 128-byte swizzle, zero fill
+// (loads) or clipping (stores) outside.
+bool make_map(CUtensorMap* map, CUtensorMapDataType type, const void* base, int64_t rows, int64_t cols,
+              int64_t pitch, uint32_t elem_bytes, uint32_t box_rows)
 {
     EncodeTiled fn = encode_fn();
     if (!fn) return false;
-    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(row_bytes), static_cast<cuuint64_t>(rows)};
-    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
-    const cuuint32_t box[2] = {kChunk, kTile};
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(pitch)};
+    const cuuint32_t box[2] = {128u / elem_bytes, box_rows};
     const cuuint32_t estr[2] = {1, 1};
-    return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(codes), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    return fn(map, type, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -388,7 +479,8 @@ int device_sm_count()
 }
 
 template <int FMT>
-cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, cudaStream_t st)
+cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md, const GemmParams& p,
+                   cudaStream_t st)
 {
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
@@ -398,7 +490,7 @@ cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParam
     if (attr != cudaSuccess) return attr;
     const uint32_t tiles = p.tiles_m * p.tiles_n;
     const uint32_t grid = std::min<uint32_t>(tiles, static_cast<uint32_t>(device_sm_count()));
-    fp4_gemm_kernel<FMT><<<grid, kThreads, kSmemBytes, st>>>(ma, mb, p);
+    fp4_gemm_kernel<FMT><<<grid, kThreads, kSmemBytes, st>>>(ma, mb, md, p);
     return cudaGetLastError();
 }
 
@@ -433,8 +525,10 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
     if (misaligned(a_codes, 16) || misaligned(b_codes, 16) || misaligned(a_scale_tiles, 16) ||
         misaligned(b_scale_tiles, 16) || misaligned(alpha_a, 4) || misaligned(alpha_b, 4))
         return FOCUS_ERR_MISALIGNED;
-    CUtensorMap ma, mb;
-    if (!make_map(&ma, a_codes, M, K / 2) || !make_map(&mb, b_codes, N, K / 2)) return FOCUS_ERR_CUDA;
+    CUtensorMap ma, mb, md;
+    if (!make_map(&ma, CU_TENSOR_MAP_DATA_TYPE_UINT8, a_codes, M, K / 2, K / 2, 1, kTile) ||
+        !make_map(&mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, b_codes, N, K / 2, K / 2, 1, kTileN))
+        return FOCUS_ERR_CUDA;
     GemmParams p;
     p.sfa = a_scale_tiles;
     p.sfb = b_scale_tiles;
@@ -448,10 +542,15 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
     const int64_t block = fmt == FOCUS_MXFP4 ? 32 : 16;
     p.tiles_k = static_cast<uint32_t>((K / block + 3) / 4);
     p.tiles_m = static_cast<uint32_t>((M + kTile - 1) / kTile);
-    p.tiles_n = static_cast<uint32_t>((N + kTile - 1) / kTile);
+    p.tiles_n = static_cast<uint32_t>((N + kTileN - 1) / kTileN);
+    p.tile_rows_b = static_cast<uint32_t>((N + kTile - 1) / kTile);
     p.n_steps = static_cast<uint32_t>(K / 64);
     p.d_bf16 = bf16;
     p.d_vec = !misaligned(d, 16) && (ldd * (bf16 ? 2 : 4)) % 16 == 0;
-    const cudaError_t e = fmt == FOCUS_MXFP4 ? launch<0>(ma, mb, p, st) : launch<1>(ma, mb, p, st);
+    std::memset(&md, 0, sizeof(md));
+    if (p.d_vec && !make_map(&md, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, d, M, N,
+                             ldd * (bf16 ? 2 : 4), bf16 ? 2 : 4, 32))
+        return FOCUS_ERR_CUDA;
+    const cudaError_t e = fmt == FOCUS_MXFP4 ? launch<0>(ma, mb, md, p, st) : launch<1>(ma, mb, md, p, st);
     return e == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA;
 }
