@@ -7,36 +7,41 @@
 // exported codes and hardware scales enter the product.
 //
 // Persistent, warp-specialised kernel, one CTA per SM, 128 x 256 tiles of D
-// (one M = 128, N = 256 MMA per K = 64 step):
+// (one M = 128, N = 256 MMA per K = 64 step), CTA pairs in clusters:
 //   warp 0     TMA producer: per K chunk of 256 elements (128 bytes of codes
-//              per row) the A and B code tiles (2D TMA, 128-byte swizzle)
-//              and their scale tiles (1D bulk copies) into a ring of stages;
+//              per row) the CTA's A tile and its half of the pair's B tile
+//              (2D TMA, 128-byte swizzle; the B half multicast to both CTAs
+//              of the cluster) and the chunk's scale tiles (1D bulk copies)
+//              into a ring of stages;
 //   warp 1     MMA issuer: four K = 64 block-scaled MMAs per chunk into an
-//              accumulator in tensor memory, commit to free the stage;
+//              accumulator in tensor memory, a commit to free the stage on
+//              both CTAs;
 //   warps 2-5  epilogue: accumulator -> registers (one lane quarter each),
 //              alpha scaling, then 32-row x 128-byte boxes of D staged in
 //              shared memory and written by TMA stores;
 //   warps 6-9  scale warps: the chunk's scale tiles shared -> tensor memory
 //              (tcgen05.st, one lane quarter each), alternating between two
-//              sets of scale regions, handed to the MMA thread by mbarrier.
-// Writing the scales with tcgen05.st from these warps keeps them off the
-// tensor pipe: copied there with tcgen05.cp they serialised with the MMAs
-// and cost about 40 % of the run time.  Per-lane row stores of D (32 rows
-// per warp instruction) cost a third of the run time; the staged TMA stores
-// write whole lines.  The 256-column accumulator fills half of tensor
-// memory, the scale sets the other half, so there is one accumulator: the
-// bf16 epilogue holds its whole row in registers and releases it before
-// staging.
+//              sets of scale regions, handed to the MMA warp by mbarrier.
+// The producer and MMA warps run their loops converged (all lanes wait,
+// lane 0 issues).  Writing the scales with tcgen05.st from their own warps
+// keeps them off the tensor pipe: copied there with tcgen05.cp they
+// serialised with the MMAs and cost about 40 % of the run time.  Per-lane
+// row stores of D (32 rows per warp instruction) cost a third of the run
+// time; the staged TMA stores write whole lines.  The 256-column accumulator
+// fills half of tensor memory, the scale sets the other half, so there is
+// one accumulator: the bf16 epilogue holds its whole row in registers and
+// releases it before staging.
 //
 // Scale factors in tensor memory: one MMA step reads an A region of 4
-// columns and a B region of 8; row m of A takes lane m, column m / 32;
-// column n of B is read by each 32-lane quarter from its own quarter, lane
-// n % 32, column n / 32.  Lane l of every quarter must therefore hold, in
-// four consecutive columns, the scale words of rows l, l + 32, l + 64,
-// l + 96 of a 128-row group: exactly line l of a 128 x 4 export tile (B
-// rows 128-255 take the next four columns).  A word holds consecutive K
-// blocks in byte order: one NVFP4 step uses all four bytes, an MXFP4 tile
-// feeds two steps (bytes 0-1, then bytes 2-3 through the scale data id).
+// columns and a B region of 8; row m of A takes lane m, column m / 32 (so
+// quarter q reads only column q: the scale warps write that one); column n
+// of B is read by each 32-lane quarter from its own quarter, lane n % 32,
+// column n / 32.  Lane l of every quarter must therefore hold, in four
+// consecutive columns, the scale words of rows l, l + 32, l + 64, l + 96 of
+// a 128-row group of B: exactly line l of a 128 x 4 export tile (B rows
+// 128-255 take the next four columns).  A word holds consecutive K blocks in
+// byte order: one NVFP4 step uses all four bytes, an MXFP4 tile feeds two
+// steps (bytes 0-1, then bytes 2-3 through the scale data id).
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -68,18 +73,24 @@ constexpr int kOutBox = 32 * 128;
 constexpr int kOutBufs = 2;
 constexpr int kSmemBytes = kStages * kStageBytes + 4 * kOutBufs * kOutBox + 1024;   // + alignment slack
 constexpr int kThreads = 320;         // producer, MMA, four epilogue warps, four scale warps
+// CTAs of a cluster: consecutive 128-row tiles of A with the same 256-row
+// tile of B; each CTA loads 1 / kCluster of the B tile and multicasts it to
+// all of them, so B is read from L2 once per cluster.
+constexpr int kCluster = 2;
+constexpr int kSliceRows = kTileN / kCluster;
+constexpr int kSliceBytes = kTileBytesB / kCluster;
+constexpr uint16_t kClusterMask = static_cast<uint16_t>((1u << kCluster) - 1);
 // tensor memory: the 256-column accumulator, then two sets of scale regions
 // used by chunks in turn (set k % 2); inside a set, the four steps of a chunk
 // at + 16 j (A, 4 columns) and + 64 + 16 j (B, 8 columns: B rows 0-127 in
 // the first four, rows 128-255 in the next four -- column n of an N = 256
 // MMA is read from column n / 32).  Every region starts on a 16-column
-// boundary.  The epilogue releases the accumulator as soon as it has been
-// read into registers, before its stores.
+// boundary (a scale address at an odd column faulted).
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccBufs = 1;      // accumulators, kTileN columns each, from column 0
-constexpr uint32_t kSfSets = 2;       // scale sets, 128 columns each, after the accumulators
 constexpr uint32_t kSfBase = kTileN * kAccBufs;
-constexpr uint32_t kSfa = 0, kSfb = 64, kSfStep = 16, kSfSet = 128;   // inside a set
+constexpr uint32_t kSfStep = 16;
+constexpr uint32_t kSfSets = 2, kSfSet = 128, kSfb = 64;
 static_assert(kSfBase + kSfSets * kSfSet <= kTmemCols, "tensor memory");
 constexpr uint32_t kWaitLimit = 1u << 24;   // polls; each try_wait may suspend for a while
 
@@ -122,13 +133,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(&full[s], 1);
-            tc::mbar_init(&empty[s], 1);
+            tc::mbar_init(&empty[s], kCluster);   // the MMA commits of every CTA of the cluster
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(&acc_full[b], 1);
             tc::mbar_init(&acc_empty[b], 128);
         }
-        for (uint32_t b = 0; b < kSfSets; ++b) tc::mbar_init(&sf_full[b], 128);
+        for (uint32_t b = 0; b < kSfSets; ++b) tc::mbar_init(&sf_full[b], 128);   // every scale-warp thread
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 0) {
@@ -137,73 +148,103 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::tc_fence_before();
     __syncthreads();
+    tc::cluster_sync();   // every barrier of the cluster initialised before any multicast
     tc::tc_fence_after();
     const uint32_t tb = tbase;
 
-    const uint32_t n_tiles = p.tiles_m * p.tiles_n;
+    // tile groups: kCluster consecutive 128-row tiles of A (one per CTA of
+    // the cluster; the last group may have CTAs past M, which load no A,
+    // store nothing and keep the cluster's pipeline going) x one tile of B
+    const uint32_t rank = tc::cluster_rank();
+    const uint32_t tiles_mg = (p.tiles_m + kCluster - 1) / kCluster;
+    const uint32_t n_groups = tiles_mg * p.tiles_n;
+    const uint32_t group0 = tc::cluster_id(), groups_step = tc::cluster_count();
     const uint32_t n_chunks = (p.n_steps + 3) / 4;
     constexpr uint32_t steps_per_tile = FMT == 0 ? 2 : 1;   // K steps one scale tile covers
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
-        if (lane == 0) {
-            uint32_t s = 0, ph = 0;
-            bool ok = true;
-            for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-                const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
-                for (uint32_t c = 0; c < n_chunks; ++c) {
-                    if (!tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit)) {
-                        ok = false;
-                        give_up(p);
-                        break;
-                    }
+        // The whole warp runs the loop (converged waits); lane 0 issues.
+        uint32_t s = 0, ph = 0;
+        bool ok = true;
+        for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
+            const uint32_t tm = (u % tiles_mg) * kCluster + rank, tn = u / tiles_mg;
+            const bool valid = tm < p.tiles_m;
+            for (uint32_t c = 0; c < n_chunks; ++c) {
+                if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit))) {
+                    ok = false;
+                    if (lane == 0) give_up(p);
+                    break;
+                }
+                if (lane == 0) {
                     const uint32_t steps = min(4u, p.n_steps - 4 * c);
                     const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
                     const uint32_t tile0 = (4 * c) / steps_per_tile;
                     const bool hi = 2 * tn + 1 < p.tile_rows_b;   // second 128-row half of B exists
-                    tc::mbar_arrive_expect_tx(&full[s], kTileBytes + kTileBytesB + (hi ? 3 : 2) * sf_tiles * 512);
-                    tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
-                                    static_cast<int32_t>(tm * kTile), &full[s]);
-                    tc::tma_load_2d(stage_b(s), &tma_b, static_cast<int32_t>(c * kChunk),
-                                    static_cast<int32_t>(tn * kTileN), &full[s]);
-                    tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
-                                  sf_tiles * 512, &full[s]);
+                    // this CTA's A tile and scales, the whole B tile (one slice from
+                    // each CTA of the cluster) and the B scales
+                    tc::mbar_arrive_expect_tx(&full[s], (valid ? kTileBytes + sf_tiles * 512 : 0) + kTileBytesB +
+                                                            (hi ? 2 : 1) * sf_tiles * 512);
+                    tc::tma_load_2d_mc(stage_b(s) + rank * kSliceBytes, &tma_b, static_cast<int32_t>(c * kChunk),
+                                       static_cast<int32_t>(tn * kTileN + rank * kSliceRows), &full[s], kClusterMask);
+                    if (valid) {
+                        tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
+                                        static_cast<int32_t>(tm * kTile), &full[s]);
+                        tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
+                                      sf_tiles * 512, &full[s]);
+                    }
                     tc::bulk_load(stage_sfb(s), p.sfb + (static_cast<size_t>(2 * tn) * p.tiles_k + tile0) * 512,
                                   sf_tiles * 512, &full[s]);
                     if (hi)
                         tc::bulk_load(stage_sfb(s) + kSfBytes,
                                       p.sfb + (static_cast<size_t>(2 * tn + 1) * p.tiles_k + tile0) * 512,
                                       sf_tiles * 512, &full[s]);
-                    if (++s == kStages) {
-                        s = 0;
-                        ph ^= 1;
-                    }
                 }
+                __syncwarp();
+                if (++s == kStages) {
+                    s = 0;
+                    ph ^= 1;
+                }
+            }
+        }
+        // every stage released by every CTA of the cluster: no commit of
+        // another CTA still to arrive on this CTA's barriers
+        for (int i = 0; i < kStages && ok; ++i) {
+            if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit))) {
+                if (lane == 0) give_up(p);
+                break;
+            }
+            if (++s == kStages) {
+                s = 0;
+                ph ^= 1;
             }
         }
     } else if (warp == 1) {
         // ---------------- MMA issuer ----------------
-        if (lane == 0) {
-            uint32_t s = 0, ph = 0, acc = 0, acc_ph = 0, k = 0;
-            bool ok = true;
-            for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-                if (!tc::mbar_wait_hot(&acc_empty[acc], acc_ph ^ 1, kWaitLimit)) {
-                    give_up(p);
+        // The whole warp runs the loop (converged waits); lane 0 issues.
+        uint32_t s = 0, ph = 0, acc = 0, acc_ph = 0, k = 0;
+        bool ok = true;
+        for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
+            if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&acc_empty[acc], acc_ph ^ 1, kWaitLimit))) {
+                if (lane == 0) give_up(p);
+                break;
+            }
+            tc::tc_fence_after();
+            const uint32_t d_tmem = tb + acc * kTileN;
+            for (uint32_t c = 0; c < n_chunks; ++c) {
+                // this chunk's scales in tensor memory; the scale warps arrive on
+                // sf_full only after observing the stage's full barrier, so its
+                // codes are in shared memory too
+                const uint32_t set = k % kSfSets;
+                const bool got = tc::mbar_wait_hot(&sf_full[set], (k / kSfSets) & 1u, kWaitLimit);
+                if (!__all_sync(0xffffffffu, got)) {
+                    ok = false;
+                    if (lane == 0) give_up(p);
                     break;
                 }
+                ++k;
                 tc::tc_fence_after();
-                const uint32_t d_tmem = tb + acc * kTileN;
-                for (uint32_t c = 0; c < n_chunks; ++c) {
-                    // codes in shared memory, then this chunk's scales in tensor memory
-                    const uint32_t set = k % kSfSets;
-                    if (!tc::mbar_wait_hot(&full[s], ph, kWaitLimit) ||
-                        !tc::mbar_wait_hot(&sf_full[set], (k / kSfSets) & 1u, kWaitLimit)) {
-                        ok = false;
-                        give_up(p);
-                        break;
-                    }
-                    ++k;
-                    tc::tc_fence_after();
+                if (lane == 0) {
                     const uint32_t steps = min(4u, p.n_steps - 4 * c);
                     const uint32_t sfbase = tb + kSfBase + kSfSet * set;
                     const uint32_t a0 = tc::smem_u32(stage_a(s)), b0 = tc::smem_u32(stage_b(s));
@@ -211,27 +252,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const uint64_t ad = tc::smem_desc_sw128(a0 + 32 * kk);
                         const uint64_t bd = tc::smem_desc_sw128(b0 + 32 * kk);
                         const uint32_t j = kk / steps_per_tile;
-                        const uint32_t sfa = sfbase + kSfa + kSfStep * j, sfb = sfbase + kSfb + kSfStep * j;
+                        const uint32_t sfa = sfbase + kSfStep * j, sfb = sfbase + kSfb + kSfStep * j;
                         const uint32_t accumulate = (c > 0 || kk > 0) ? 1u : 0u;
                         if (FMT == 0)
-                            tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, true, 2 * (kk % 2)), sfa, sfb,
-                                         accumulate);
+                            tc::mma_mxf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, true, 2 * (kk % 2)), sfa,
+                                         sfb, accumulate);
                         else
-                            tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, false), sfa, sfb,
-                                         accumulate);
+                            tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, false), sfa, sfb, accumulate);
                     }
-                    tc::mma_commit(&empty[s]);
-                    if (++s == kStages) {
-                        s = 0;
-                        ph ^= 1;
-                    }
+                    tc::mma_commit_mc(&empty[s], kClusterMask);
                 }
-                if (!ok) break;
-                tc::mma_commit(&acc_full[acc]);
-                if (++acc == kAccBufs) {
-                    acc = 0;
-                    acc_ph ^= 1;
+                __syncwarp();
+                if (++s == kStages) {
+                    s = 0;
+                    ph ^= 1;
                 }
+            }
+            if (!ok) break;
+            if (lane == 0) tc::mma_commit(&acc_full[acc]);
+            __syncwarp();
+            if (++acc == kAccBufs) {
+                acc = 0;
+                acc_ph ^= 1;
             }
         }
     } else if (warp >= 6) {
@@ -239,12 +281,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Chunk k (counted over all tiles of this CTA) uses stage k % kStages
         // and scale set k % 2.  Before a set is rewritten, the MMAs of chunk
         // k - 2, which read it, must be complete: their commit completed the
-        // empty barrier of that chunk's stage.
+        // empty barrier of that chunk's stage (on every CTA of the cluster).
         const uint32_t q = warp % 4;
         const uint32_t lane_addr = tb + ((q * 32) << 16);
         uint32_t s = 0, ph = 0, k = 0;
         bool ok = true;
-        for (uint32_t t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
             for (uint32_t c = 0; c < n_chunks; ++c, ++k) {
                 bool got = tc::mbar_wait_hot(&full[s], ph, kWaitLimit);
                 if (k >= kSfSets) {
@@ -261,14 +303,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
                 const uint32_t sfbase = lane_addr + kSfBase + kSfSet * (k % kSfSets);
                 for (uint32_t j = 0; j < sf_tiles; ++j) {
-                    const uint4 la = *reinterpret_cast<const uint4*>(stage_sfa(s) + 512 * j + 16 * lane);
+                    // A: quarter q reads only column q of the region (row q * 32 + lane)
+                    const uint32_t la = *reinterpret_cast<const uint32_t*>(stage_sfa(s) + 512 * j + 16 * lane + 4 * q);
                     const uint4 lb = *reinterpret_cast<const uint4*>(stage_sfb(s) + 512 * j + 16 * lane);
                     const uint4 lh = *reinterpret_cast<const uint4*>(stage_sfb(s) + kSfBytes + 512 * j + 16 * lane);
-                    tc::tmem_st_x4(sfbase + kSfa + kSfStep * j, la.x, la.y, la.z, la.w);
-                    tc::tmem_st_x4(sfbase + kSfb + kSfStep * j, lb.x, lb.y, lb.z, lb.w);
+                    tc::tmem_st_x1(sfbase + kSfStep * j + q, la);
                     // rows 128-255 of B (stale but finite-or-not bytes when B has no such
                     // rows: they only reach columns of D that are not stored)
-                    tc::tmem_st_x4(sfbase + kSfb + kSfStep * j + 4, lh.x, lh.y, lh.z, lh.w);
+                    tc::tmem_st_x8(sfbase + kSfb + kSfStep * j, lb.x, lb.y, lb.z, lb.w, lh.x, lh.y, lh.z, lh.w);
                 }
                 tc::tmem_wait_st();
                 tc::tc_fence_before();
@@ -312,8 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             ++obuf;
         };
-        for (uint32_t t = blockIdx.x; t < n_tiles; t += gridDim.x) {
-            const uint32_t tm = t % p.tiles_m, tn = t / p.tiles_m;
+        for (uint32_t u = group0; u < n_groups; u += groups_step) {
+            const uint32_t tm = (u % tiles_mg) * kCluster + rank, tn = u / tiles_mg;
             const bool got = __all_sync(0xffffffffu, tc::mbar_wait_hot(&acc_full[acc], acc_ph, kWaitLimit));
             if (!got) {
                 if (lane == 0) give_up(p);
@@ -416,6 +458,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp >= 2 && warp < 6 && lane == 0) tc::bulk_wait_all();   // output stores complete
     tc::tc_fence_before();
     __syncthreads();
+    tc::cluster_sync();
     tc::tc_fence_after();
     if (warp == 0) tc::tmem_dealloc(tb, kTmemCols);
 }
@@ -488,10 +531,29 @@ cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorM
         attr = cudaFuncSetAttribute(fp4_gemm_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     });
     if (attr != cudaSuccess) return attr;
-    const uint32_t tiles = p.tiles_m * p.tiles_n;
-    const uint32_t grid = std::min<uint32_t>(tiles, static_cast<uint32_t>(device_sm_count()));
-    fp4_gemm_kernel<FMT><<<grid, kThreads, kSmemBytes, st>>>(ma, mb, md, p);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kCluster;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = st;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    // persistent: as many clusters as are resident at once (one CTA per SM)
+    static int resident = 0;
+    if (resident <= 0) {
+        cfg.gridDim = dim3(kCluster * static_cast<uint32_t>(device_sm_count() / kCluster));
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, fp4_gemm_kernel<FMT>, &cfg) != cudaSuccess || n <= 0)
+            n = device_sm_count() / kCluster;
+        resident = std::max(n, 1);
+    }
+    const uint32_t groups = ((p.tiles_m + kCluster - 1) / kCluster) * p.tiles_n;
+    cfg.gridDim = dim3(kCluster * std::min<uint32_t>(groups, static_cast<uint32_t>(resident)));
+    return cudaLaunchKernelEx(&cfg, fp4_gemm_kernel<FMT>, ma, mb, md, p);
 }
 
 }  // namespace
@@ -527,7 +589,7 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
         return FOCUS_ERR_MISALIGNED;
     CUtensorMap ma, mb, md;
     if (!make_map(&ma, CU_TENSOR_MAP_DATA_TYPE_UINT8, a_codes, M, K / 2, K / 2, 1, kTile) ||
-        !make_map(&mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, b_codes, N, K / 2, K / 2, 1, kTileN))
+        !make_map(&mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, b_codes, N, K / 2, K / 2, 1, kSliceRows))
         return FOCUS_ERR_CUDA;
     GemmParams p;
     p.sfa = a_scale_tiles;
