@@ -606,6 +606,9 @@ struct Unroll {
 // is faster despite a few dozen bytes of spills to L1-cached local memory
 // (measured: NVFP4 Qwen3-4B backward 6124 -> 6543 GB/s).  The fused
 // optimizer's extra state spills too much there and keeps the lower count.
+// The MXFP4 backward with binary16 elements is the exception: its
+// conversions spill three times as much at 3 CTAs, and 2 CTAs per SM are
+// faster (Llama-70B layer set, fp16 I/O: backward 5927 -> 6413 GB/s).
 // The NVFP4 export (pack) likewise runs faster at 5 CTAs per SM than at 4
 // (pack phase: Qwen3-4B 5746 -> 5913 GB/s, Llama-70B layer 6715 -> 6796);
 // the MXFP4 export (70B: 6915 -> 6722) and the forward (Qwen3-4B NVFP4: 6409
@@ -613,7 +616,7 @@ struct Unroll {
 // state is largest.
 template <int FMT, int DT, int SUB, int MODE>
 struct MinCtas {
-    static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT != 0 ? 3 : 2);
+    static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT == 1 ? 3 : 2);
     static constexpr int adam = FMT == 1 ? 3 : 2;
     static constexpr int value =
         ((MODE >= kBwdA) ? adam : (MODE >= kBwd) ? bwd : (MODE == kPack && FMT == 1) ? 5 : 4) - (SUB == 2 ? 1 : 0);
