@@ -62,12 +62,12 @@ inline uint32_t shared_row_groups(uint32_t rows, uint32_t bpr)
 // that: with CTAs finishing and starting, the CTAs of an SM fall out of step
 // and their load and compute phases overlap, where resident CTAs that start
 // together walk the tensor in lockstep (one 2 GiB tensor, MXFP4 step: 6219
-// -> 6845 GB/s; Llama-70B layer set 6781 -> 7052).  Smaller tensors keep
-// one round: launched side by side on parallel branches they already
-// overlap, and more CTAs there measured slower (Qwen3-4B backward at 10
-// rounds: 6520 -> 6331 GB/s).
+// -> 6845 GB/s; one 256 MB tensor at 27 rounds 6436 -> 6688; Llama-70B
+// layer set 6781 -> 7036).  Smaller tensors keep one round: launched side
+// by side on parallel branches they already overlap, and more CTAs there
+// measured slower (Qwen3-4B backward at 10 rounds: 6520 -> 6331 GB/s).
 constexpr uint64_t kOversub = 8;
-constexpr uint64_t kOversubRounds = 32;
+constexpr uint64_t kOversubRounds = 16;
 
 template <typename Kern>
 inline uint32_t stream_grid(Kern kern, int& occ_cache, uint32_t n_chunks, uint32_t span)
