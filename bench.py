@@ -701,18 +701,32 @@ class OraclePool:
                 np.ndarray(a.shape, dtype=a.dtype, buffer=shm.buf)[...] = a
                 spec.append((shm.name, a.shape, a.dtype.str))
             specs.append(spec)
-        self.pool = cf.ProcessPoolExecutor(procs, mp_context=mp.get_context("spawn"), initializer=_pool_init,
-                                           initargs=(case, specs))
-        self.step()   # every worker has started and mapped the samples
+        self.pool = None
+        try:
+            self.pool = cf.ProcessPoolExecutor(procs, mp_context=mp.get_context("spawn"), initializer=_pool_init,
+                                               initargs=(case, specs))
+            self.step()   # every worker has started and mapped the samples
+        except BaseException:
+            self.close()
+            raise
 
     def step(self):
         list(self.pool.map(_pool_step, [(k, self.procs) for k in range(self.procs)]))
 
     def close(self):
-        self.pool.shutdown()
+        if self.pool is not None:
+            self.pool.shutdown()
+            self.pool = None
         for shm in self.shm:
             shm.close()
             shm.unlink()
+        self.shm = []
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
 
 
 def pool_fits(samples) -> bool:
@@ -743,14 +757,13 @@ def cpu_baseline(case, target_s=15.0):
     dt1 = time.perf_counter() - t0
     procs = host_cores() if pool_fits(samples) else 1
     if procs > 1:
-        pool = OraclePool(case, samples, procs)
-        del samples
         times = []
-        while len(times) < 3 or sum(times) < 2.0:
-            t0 = time.perf_counter()
-            pool.step()
-            times.append(time.perf_counter() - t0)
-        pool.close()
+        with OraclePool(case, samples, procs) as pool:
+            del samples
+            while len(times) < 3 or sum(times) < 2.0:
+                t0 = time.perf_counter()
+                pool.step()
+                times.append(time.perf_counter() - t0)
         dt = sorted(times)[len(times) // 2]
     else:
         times, dt = [dt1], dt1
@@ -783,13 +796,15 @@ def reference_arm(case, args):
             samples = oracle_samples(case, rows)
             n, nbytes = sample_elems_and_bytes(case, samples)
         run, done = (lambda: oracle_step(case, samples)), (lambda: None)
-    for _ in range(args.warmup):
-        run()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        run()
-    dt = (time.perf_counter() - t0) / max(1, args.steps)
-    done()
+    try:
+        for _ in range(args.warmup):
+            run()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            run()
+        dt = (time.perf_counter() - t0) / max(1, args.steps)
+    finally:
+        done()
     value = nbytes / dt / 1e9
     return {"metric": METRIC, "value": round(value, 6), "unit": "GB/s", "impl": "reference",
             "n_gpus": 0, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3),
