@@ -281,8 +281,9 @@ size_t focus_mma_scale_bytes(const focus_desc_t* desc);
  * fp32 sum before the output rounding.
  * Requirements: K % 64 == 0 (FOCUS_ERR_UNSUPPORTED otherwise); codes and
  * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
- * kernel whose wait for its MMAs gives up sets it to 1 (the output is then
- * not written) instead of waiting for ever.  Enqueued on `stream`. */
+ * kernel whose wait on its pipeline gives up sets it to 1 (the output is
+ * then incomplete) instead of waiting for ever.  Enqueued on `stream`; the
+ * kernel runs as clusters of two CTAs. */
 int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
                    const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
                    const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,
