@@ -21,7 +21,8 @@
 //              shared memory and written by TMA stores;
 //   warps 6-9  scale warps: the chunk's scale tiles shared -> tensor memory
 //              (tcgen05.st, one lane quarter each), alternating between two
-//              sets of scale regions, handed to the MMA warp by mbarrier.
+//              sets of scale regions (an NVFP4 chunk fills a set, an MXFP4
+//              set holds two chunks), handed to the MMA warp by mbarrier.
 // The producer and MMA warps run their loops converged (all lanes wait,
 // lane 0 issues).  Writing the scales with tcgen05.st from their own warps
 // keeps them off the tensor pipe: copied there with tcgen05.cp they
@@ -121,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const __grid_constant__ CUtensorMap tma_d, const GemmParams p)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], sf_full[kSfSets];
+    __shared__ __align__(8) uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], sf_full[2 * kSfSets];
     __shared__ uint32_t tbase;
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     auto stage_a = [&](uint32_t s) { return smem + s * kStageBytes; };
@@ -139,7 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_init(&acc_full[b], 1);
             tc::mbar_init(&acc_empty[b], 128);
         }
-        for (uint32_t b = 0; b < kSfSets; ++b) tc::mbar_init(&sf_full[b], 128);   // every scale-warp thread
+        for (uint32_t b = 0; b < 2 * kSfSets; ++b) tc::mbar_init(&sf_full[b], 128);   // every scale-warp thread
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 0) {
@@ -161,6 +162,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t group0 = tc::cluster_id(), groups_step = tc::cluster_count();
     const uint32_t n_chunks = (p.n_steps + 3) / 4;
     constexpr uint32_t steps_per_tile = FMT == 0 ? 2 : 1;   // K steps one scale tile covers
+    // chunks per scale set: an MXFP4 chunk has two scale tiles, so a set
+    // (four tiles) holds two consecutive chunks, each handed over on its own
+    // barrier (sf_full[set * 2 + half]); an NVFP4 chunk fills a set alone
+    constexpr uint32_t kChunksPerSet = FMT == 0 ? 2 : 1;
+    constexpr uint32_t kTilesPerChunk = 4 / steps_per_tile;
 
     if (warp == 0) {
         // ---------------- TMA producer ----------------
@@ -235,8 +241,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // this chunk's scales in tensor memory; the scale warps arrive on
                 // sf_full only after observing the stage's full barrier, so its
                 // codes are in shared memory too
-                const uint32_t set = k % kSfSets;
-                const bool got = tc::mbar_wait_hot(&sf_full[set], (k / kSfSets) & 1u, kWaitLimit);
+                const uint32_t pair = k / kChunksPerSet, set = pair % kSfSets;
+                const bool got = tc::mbar_wait_hot(&sf_full[set * kChunksPerSet + k % kChunksPerSet],
+                                                   (pair / kSfSets) & 1u, kWaitLimit);
                 if (!__all_sync(0xffffffffu, got)) {
                     ok = false;
                     if (lane == 0) give_up(p);
@@ -246,7 +253,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::tc_fence_after();
                 if (lane == 0) {
                     const uint32_t steps = min(4u, p.n_steps - 4 * c);
-                    const uint32_t sfbase = tb + kSfBase + kSfSet * set;
+                    const uint32_t sfbase =
+                        tb + kSfBase + kSfSet * set + kSfStep * kTilesPerChunk * ((k - 1) % kChunksPerSet);
                     const uint32_t a0 = tc::smem_u32(stage_a(s)), b0 = tc::smem_u32(stage_b(s));
                     for (uint32_t kk = 0; kk < steps; ++kk) {
                         const uint64_t ad = tc::smem_desc_sw128(a0 + 32 * kk);
@@ -279,9 +287,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (warp >= 6) {
         // ---------------- scale warps (warps 6-9: lane quarters 2, 3, 0, 1) ----------------
         // Chunk k (counted over all tiles of this CTA) uses stage k % kStages
-        // and scale set k % 2.  Before a set is rewritten, the MMAs of chunk
-        // k - 2, which read it, must be complete: their commit completed the
-        // empty barrier of that chunk's stage (on every CTA of the cluster).
+        // and scale set (k / kChunksPerSet) % 2.  Before a set is rewritten,
+        // the MMAs of the chunks that last used it must be complete.  NVFP4
+        // (one chunk per set): those of chunk k - 2, whose commit completed
+        // the empty barrier of that chunk's stage (on every CTA of the
+        // cluster).  MXFP4 (pairs of chunks): the last of them is chunk
+        // 2 p - 3 for pair p, and the producer loaded chunk 2 p into the stage
+        // that chunk freed (three stages), so the full barrier of chunk 2 p
+        // already implies it.
+        static_assert(kStages == 3, "the MXFP4 set release relies on three stages");
         const uint32_t q = warp % 4;
         const uint32_t lane_addr = tb + ((q * 32) << 16);
         uint32_t s = 0, ph = 0, k = 0;
@@ -289,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
             for (uint32_t c = 0; c < n_chunks; ++c, ++k) {
                 bool got = tc::mbar_wait_hot(&full[s], ph, kWaitLimit);
-                if (k >= kSfSets) {
+                if (kChunksPerSet == 1 && k >= kSfSets) {
                     const uint32_t k2 = k - kSfSets;
                     got = got && tc::mbar_wait_hot(&empty[k2 % kStages], (k2 / kStages) & 1u, kWaitLimit);
                 }
@@ -301,7 +315,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::tc_fence_after();
                 const uint32_t steps = min(4u, p.n_steps - 4 * c);
                 const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
-                const uint32_t sfbase = lane_addr + kSfBase + kSfSet * (k % kSfSets);
+                const uint32_t set = (k / kChunksPerSet) % kSfSets;
+                const uint32_t sfbase =
+                    lane_addr + kSfBase + kSfSet * set + kSfStep * kTilesPerChunk * (k % kChunksPerSet);
                 for (uint32_t j = 0; j < sf_tiles; ++j) {
                     // A: quarter q reads only column q of the region (row q * 32 + lane)
                     const uint32_t la = *reinterpret_cast<const uint32_t*>(stage_sfa(s) + 512 * j + 16 * lane + 4 * q);
@@ -314,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc::tmem_wait_st();
                 tc::tc_fence_before();
-                tc::mbar_arrive(&sf_full[k % kSfSets]);
+                tc::mbar_arrive(&sf_full[set * kChunksPerSet + k % kChunksPerSet]);
                 if (++s == kStages) {
                     s = 0;
                     ph ^= 1;
