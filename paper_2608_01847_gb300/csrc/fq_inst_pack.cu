@@ -24,6 +24,9 @@ __device__ __forceinline__ void alpha_final_kernel_body(const float* partials, u
 __global__ void __launch_bounds__(kThreads) alpha_final_kernel(const float* partials, uint32_t n,
                                                                float* alpha_out)
 {
+    // launched early behind the partial pass: wait until it has completed
+    // and its partials are visible (a no-op without that dependency)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     alpha_final_kernel_body(partials, n, alpha_out);
 }
 
@@ -65,8 +68,19 @@ cudaError_t launch_alpha(int dt, const KParams& p, float* alpha_out, cudaStream_
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    alpha_final_kernel<<<1, kThreads, 0, st>>>(p.ws, p.n_chunks > 0 ? grid : 0u, alpha_out);
-    return cudaGetLastError();
+    // programmatic dependent launch: the one-CTA reduction is scheduled while
+    // the partial pass still runs, instead of after it
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(kThreads);
+    cfg.stream = st;
+    cfg.attrs = at;
+    cfg.numAttrs = p.n_chunks > 0 ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, alpha_final_kernel, static_cast<const float*>(p.ws),
+                              p.n_chunks > 0 ? grid : 0u, alpha_out);
 }
 
 }  // namespace focus

@@ -1053,6 +1053,9 @@ __device__ __forceinline__ float alpha_cta_max(const KParams& p, uint32_t cta, u
 template <int DT>
 __global__ void __launch_bounds__(kThreads) alpha_partial_kernel(const KParams p)
 {
+    // the final reduction may be launched now: it waits for this grid to
+    // complete (programmatic dependent launch) before reading the partials
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float red[kThreads / 32];
     const float m = alpha_cta_max<DT>(p, blockIdx.x, gridDim.x, red);
     if (threadIdx.x == 0) p.ws[blockIdx.x] = m;
