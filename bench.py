@@ -80,7 +80,7 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
 # dram__bytes_read, dram__bytes_write; --cache-control none), and the sha256
 # prefix of the kernel sources it was taken on.  Reported only for the
 # default case and while the sources are unchanged.
-BWD_TRAFFIC = {"sources": "14e3da1841cd326b", "bytes_per_step": 740.8e6}
+BWD_TRAFFIC = {"sources": "dfa36b6672f90c55", "bytes_per_step": 703.1e6}
 
 # AdamW hyper-parameters of the fused optimizer: the paper's learning rates
 # per format (Sec. 4.1: block scale / relaxation coefficients) and PyTorch's
@@ -465,8 +465,15 @@ def gpu_arm(case, args, rank, world, device):
         graphs = {ph: [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
                                    stages=(ph,), before=before) for par in parities]
                   for ph in phases}
-        step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
-                                   stages=phases, before=before) for par in parities]
+        if args.staged:
+            step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
+                                       stages=phases, before=before) for par in parities]
+        else:
+            # each tensor's phases chained on its own branch, no join between
+            # phases (the tensors are independent); the optimizer's step
+            # counter advances once, before the branches fork
+            step_graphs = [BranchGraph(len(ts), lambda i, par=par: [ts[i].run(ph, par) for ph in phases],
+                                       device, before=lambda _stage: before("bwd")) for par in parities]
     n_replay = [0]
 
     def step():
@@ -927,6 +934,9 @@ def main():
                     help="backward fused with the AdamW step on the learned arrays")
     ap.add_argument("--io", default="", choices=["", "bf16", "f16", "f32"],
                     help="element type of x, y, g, gx (default: the workload's)")
+    ap.add_argument("--staged", action="store_true",
+                    help="step graph with a join of all tensors between phases (default: each "
+                         "tensor's phases chained on its own branch)")
     ap.add_argument("--group", action="store_true",
                     help="one group launch per phase for all tensors instead of per-tensor launches")
     ap.add_argument("--gemm", action="store_true",
@@ -996,7 +1006,10 @@ def main():
                                     "per-block CRS + per-sub-block DGS"),
                    "scales": "learnable S^fp (+ dL/dS^fp)" if case.sfp else "absmax",
                    "launch": "one group launch per phase" if r["grouped"] else
-                             "one launch per tensor and phase, tensors on parallel graph branches",
+                             ("one launch per tensor and phase, tensors on parallel graph branches, "
+                              "phases joined" if args.staged else
+                              "one launch per tensor and phase, each tensor's phases chained on its "
+                              "own graph branch (programmatic dependent launches)"),
                    "step": "+".join(case.phases()) + " over all tensors " +
                            ("(bwd: gx + AdamW on the learned arrays)" if case.adam else
                             "(bwd: gx + gcrs + gdgs)"),

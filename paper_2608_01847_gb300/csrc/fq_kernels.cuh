@@ -845,6 +845,11 @@ template <int FMT, int DT, int SUB, int MODE>
 __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
     fq_block_kernel(const KParams p)
 {
+    // launched as a programmatic dependent of the previous kernel in the
+    // stream: wait until that one has completed (its results visible), then
+    // let the next one be scheduled behind this grid
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     block_loop<FMT, DT, SUB, MODE>(OneTensor<FMT>(p));
 }
 

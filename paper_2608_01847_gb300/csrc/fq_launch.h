@@ -83,14 +83,31 @@ inline uint32_t stream_grid(Kern kern, int& occ_cache, uint32_t n_chunks, uint32
     return static_cast<uint32_t>(std::max<uint64_t>(1, grid));
 }
 
+// Programmatic dependent launch: the grid may be scheduled while the
+// previous kernel in the stream is still running; the kernel itself waits
+// (griddepcontrol.wait) for that kernel's completion before touching memory.
+template <typename Kern, typename... Args>
+inline cudaError_t launch_dependent(Kern kern, uint32_t grid, cudaStream_t st, const Args&... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.stream = st;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 template <int FMT, int DT, int SUB, int MODE>
 cudaError_t run_block(const KParams& p, cudaStream_t st)
 {
     static int occ = 0;
     auto kern = fq_block_kernel<FMT, DT, SUB, MODE>;
     const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Unroll<FMT, DT, MODE>::U * kThreads);
-    kern<<<grid, kThreads, 0, st>>>(p);
-    return cudaGetLastError();
+    return launch_dependent(kern, grid, st, p);
 }
 
 // Dispatch over the sub-block size for one (format, dtype, mode).
