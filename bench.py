@@ -873,13 +873,21 @@ def gemm_arm(args, device):
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize(device)
+    # the step's GEMMs as one CUDA graph (no host launch gaps between them)
+    graph = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream(device)
+    cap.wait_stream(torch.cuda.current_stream(device))
+    with torch.cuda.graph(graph, stream=cap):
+        step()
+    torch.cuda.current_stream(device).wait_stream(cap)
+    graph.replay()
+    torch.cuda.synchronize(device)
     stream = torch.cuda.current_stream(device)
-    per = []
     with ClockSampler(device.index if device.index is not None else 0) as clk:
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
-            step()
+            graph.replay()
         e1.record(stream)
         torch.cuda.synchronize(device)
     ms = e0.elapsed_time(e1) / args.steps

@@ -152,6 +152,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::cluster_sync();   // every barrier of the cluster initialised before any multicast
     tc::tc_fence_after();
     const uint32_t tb = tbase;
+    // launched as a programmatic dependent: the set-up above overlaps the
+    // previous kernel in the stream; nothing it wrote is read before this
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     // tile groups: kCluster consecutive 128-row tiles of A (one per CTA of
     // the cluster; the last group may have CTAs past M, which load no A,
@@ -548,16 +552,18 @@ cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorM
     });
     if (attr != cudaSuccess) return attr;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute at[1];
+    cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = kCluster;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = kSmemBytes;
     cfg.stream = st;
     cfg.attrs = at;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;   // the occupancy query below takes the cluster shape only
     // persistent: as many clusters as are resident at once (one CTA per SM)
     static int resident = 0;
     if (resident <= 0) {
@@ -569,6 +575,7 @@ cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorM
     }
     const uint32_t groups = ((p.tiles_m + kCluster - 1) / kCluster) * p.tiles_n;
     cfg.gridDim = dim3(kCluster * std::min<uint32_t>(groups, static_cast<uint32_t>(resident)));
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, fp4_gemm_kernel<FMT>, ma, mb, md, p);
 }
 
