@@ -33,44 +33,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity)
     return ok != 0;
 }
 
-__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Wait for the phase with the given parity to complete; false after
-// `limit` unsuccessful polls (the caller records the failure).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit)
-{
-    for (uint32_t i = 0; i < limit; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (i > 64) __nanosleep(64);
-    }
-    return false;
-}
-
-// The same wait without sleeping between polls (try_wait itself suspends
-// the thread for a while): for waits on the critical path of a pipeline.
+// Wait for the phase with the given parity to complete; false after `limit`
+// unsuccessful polls (the caller records the failure).  No sleep between
+// polls: try_wait itself suspends the thread for a while.
 __device__ __forceinline__ bool mbar_wait_hot(uint64_t* bar, uint32_t parity, uint32_t limit)
 {
     for (uint32_t i = 0; i < limit; ++i)
         if (mbar_try_wait(bar, parity)) return true;
-    return false;
-}
-
-// The same wait by polling test_wait (the thread is never suspended).
-__device__ __forceinline__ bool mbar_wait_spin(uint64_t* bar, uint32_t parity, uint32_t limit)
-{
-    for (uint32_t i = 0; i < limit; ++i)
-        if (mbar_test_wait(bar, parity)) return true;
     return false;
 }
 
@@ -166,17 +135,10 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
-// One 32-bit column per lane of the warp's 32-lane quarter (x4: 4 columns).
+// One 32-bit column per lane of the warp's 32-lane quarter.
 __device__ __forceinline__ void tmem_st_x1(uint32_t taddr, uint32_t a)
 {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(a) : "memory");
-}
-
-__device__ __forceinline__ void tmem_st_x4(uint32_t taddr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
-{
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(a), "r"(b),
-                 "r"(c), "r"(d)
-                 : "memory");
 }
 
 // The same, 8 columns.
@@ -208,19 +170,6 @@ __device__ __forceinline__ void tmem_ld_x32(uint32_t taddr, uint32_t (&r)[32])
 }
 
 // ---- descriptors ----------------------------------------------------------------
-// Shared-memory matrix descriptor, K-major operand without swizzling: core
-// matrices of 8 rows x 16 bytes; `lbo` = byte distance between core matrices
-// adjacent along K, `sbo` = between core matrices adjacent along M / N.
-__device__ __forceinline__ uint64_t smem_desc_kmajor(uint32_t saddr, uint32_t lbo, uint32_t sbo)
-{
-    uint64_t d = 0;
-    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);          // bits 0-13: start address
-    d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;       // bits 16-29: leading byte offset
-    d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;       // bits 32-45: stride byte offset
-    d |= static_cast<uint64_t>(1) << 46;                          // bits 46-48: descriptor version 1
-    // base offset 0, relative leading offset, no swizzle (bits 61-63 = 0)
-    return d;
-}
 
 // K-major operand in 128-byte swizzled rows (as a TMA SWIZZLE_128B load
 // writes them): 8-row groups 1024 bytes apart; the tile must be 1024-byte
@@ -234,16 +183,6 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
     d |= static_cast<uint64_t>(1) << 46;                          // descriptor version 1
     d |= static_cast<uint64_t>(2) << 61;                          // 128-byte swizzle
     return d;
-}
-
-// Scale factors: shared memory -> tensor memory, 32 rows x 16 bytes (one
-// 128 x 4 export tile, line l = row l), copied to lane l of all four lane
-// quarters, columns taddr .. taddr + 3.  Ordered before later MMAs issued
-// by the same thread.
-__device__ __forceinline__ void tmem_cp_32x128b_x4(uint32_t taddr, uint32_t saddr)
-{
-    const uint64_t desc = smem_desc_kmajor(saddr, 16, 128);
-    asm volatile("tcgen05.cp.cta_group::1.32x128b.warpx4 [%0], %1;" ::"r"(taddr), "l"(desc) : "memory");
 }
 
 // Instruction descriptor of the block-scaled FP4 MMA (.kind::mxf4 and
