@@ -44,6 +44,7 @@ def main():
     ap.add_argument("--sub", type=int, default=8)
     ap.add_argument("--shared", action="store_true")
     ap.add_argument("--no-gx", action="store_true")
+    ap.add_argument("--sfp", action="store_true", help="bwd: learnable S^fp and its gradient")
     ap.add_argument("--launches", type=int, default=3)
     a = ap.parse_args()
 
@@ -59,6 +60,13 @@ def main():
     y = torch.empty_like(x)
     gx = None if a.no_gx else torch.empty_like(x)
     gc, gd = torch.empty_like(crs), torch.empty_like(dgs)
+    sfp = gsfp = None
+    if a.sfp:
+        # S^fp at its absmax initialisation (fp32 per block), as the benchmark's --sfp
+        m = x.float().abs().reshape(x.shape[0], -1, blk).amax(-1)
+        den = 6.0 if fmt == F.FOCUS_MXFP4 else float(alpha.item()) * 6.0
+        sfp = (m / den).contiguous()
+        gsfp = torch.empty_like(sfp)
     rows, cols = x.shape
     codes = torch.empty((rows, cols // 2), dtype=torch.uint8, device="cuda")
     sb = torch.empty((rows, cols // blk), dtype=torch.uint8, device="cuda")
@@ -90,7 +98,7 @@ def main():
                          scale_bytes=sb)
         else:
             F.focus_fq_bwd(x, g, fmt, crs, dgs, alpha, sub_block=a.sub, shared=a.shared, gx=gx,
-                           want_gx=not a.no_gx, gcrs=gc, gdgs=gd, ws=ws)
+                           want_gx=not a.no_gx, gcrs=gc, gdgs=gd, ws=ws, sfp=sfp, gsfp=gsfp)
 
     torch.cuda.synchronize()
     times = []
@@ -109,6 +117,8 @@ def main():
         return
     n = rows * cols
     bpe = bytes_per_elem(a.phase, a.fmt, a.sub, a.shared, not a.no_gx)
+    if a.sfp and a.phase == "bwd":
+        bpe += 2 * 4 / blk   # S^fp in, its gradient out
     print(json.dumps({"phase": a.phase, "tensor": f"{a.workload}/{a.tensor}", "shape": [rows, cols],
                       "fmt": a.fmt, "sub": a.sub, "shared": a.shared, "ms": times,
                       "algorithmic_bytes": n * bpe,
