@@ -746,6 +746,20 @@ def pool_fits(samples) -> bool:
     return 2 * need <= st.f_bavail * st.f_frsize
 
 
+def host_cpu() -> str:
+    """The host CPU as the OS names it (lscpu's model name, else the machine)."""
+    import platform
+    import subprocess
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() == "Model name":
+                return f"{line.split(':', 1)[1].strip()} ({platform.machine()})"
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.machine() or "unknown"
+
+
 def host_cores() -> int:
     try:
         return max(1, len(os.sched_getaffinity(0)))
@@ -778,7 +792,7 @@ def cpu_baseline(case, target_s=15.0):
             "sample": f"first {rows} rows of each tensor of {case.workload} ({n} elements; "
                       f"{'+'.join(case.phases())}), row slices on {procs} processes, median of {len(times)} "
                       f"passes {dt:.2f} s",
-            "elems_per_s": round(n / dt, 1),
+            "elems_per_s": round(n / dt, 1), "cpu": host_cpu(),
             "single_thread": {"value": round(nbytes / dt1 / 1e9, 6), "unit": "GB/s", "cores": 1,
                               "seconds": round(dt1, 2)}}
 
@@ -824,7 +838,7 @@ def reference_arm(case, args):
                        "elements_per_step": n},
             "cpu_baseline": {"value": round(value, 6), "unit": "GB/s", "cores": procs, "kind": "oracle",
                              "sample": f"first {rows} rows of each tensor per step, CPU oracle "
-                                       f"on row slices in {procs} processes"},
+                                       f"on row slices in {procs} processes", "cpu": host_cpu()},
             "e2e": {"value": round(value, 6), "unit": "GB/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
