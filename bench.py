@@ -943,7 +943,7 @@ def gemm_arm(args, device):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=4000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="focus", choices=["focus", "reference"])
     ap.add_argument("--workload", default="qwen3_4b_layer")
