@@ -189,8 +189,50 @@ def aggregate_gbs(bytes_per_rank_step: float, world: int, max_ms_per_step: float
 # ----------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------
+ARENA_ALIGN = 256
+
+
+def pack_arena(obj, names, device):
+    """Moves the tensor attributes `names` of `obj` into one allocation on
+    `device`, in that order, each at an ARENA_ALIGN-byte aligned offset, and
+    returns the allocation (uint8); the attributes become views of it with
+    their values, shapes and dtypes."""
+    import torch
+    arrs = [getattr(obj, n) for n in names]
+    offs, end = [], 0
+    for a in arrs:
+        offs.append(end)
+        end += -(-a.numel() * a.element_size() // ARENA_ALIGN) * ARENA_ALIGN
+    buf = torch.empty(max(end, ARENA_ALIGN), dtype=torch.uint8, device=device)
+    for n, a, off in zip(names, arrs, offs):
+        v = buf[off:off + a.numel() * a.element_size()].view(a.dtype).view(a.shape)
+        v.copy_(a)
+        setattr(obj, n, v)
+    return buf
+
+
+def arena_spans(buf, arrays):
+    """Byte ranges [start, end) of `buf` that cover `arrays` (views of it),
+    neighbours merged (across their alignment padding): the copies that move
+    those arrays between `buf` and a mirror of the same layout."""
+    base, size = buf.data_ptr(), buf.numel()
+    spans = []
+    for s, e in sorted((a.data_ptr() - base, a.data_ptr() - base + a.numel() * a.element_size())
+                       for a in arrays):
+        if s < 0 or e > size:
+            raise ValueError("array outside the arena")
+        if spans and s - spans[-1][1] < ARENA_ALIGN:
+            spans[-1][1] = max(spans[-1][1], e)
+        else:
+            spans.append([s, e])
+    return [tuple(sp) for sp in spans]
+
+
 class Tensor:
-    """Device tensors of one projection (or activation) plus its outputs."""
+    """Device tensors of one projection (or activation) plus its outputs.
+    The inputs a step takes from the host share one allocation, and so do
+    the outputs it returns, so that the end-to-end step moves each tensor
+    with one copy per direction."""
 
     def __init__(self, case: Case, w, idx, device, step=None):
         import torch
@@ -229,13 +271,20 @@ class Tensor:
             self.sfp = (m / den * jit).contiguous()
             self.gsfp = torch.empty_like(self.sfp)
         if case.adam:
-            # optimizer state resident in HBM; the paper's learning rates
-            # (Sec. 4.1); two synthetic batches alternate, the second's
-            # output gradient the negation of the first's, so that a fixed
-            # gradient does not drive the parameters out of range over
-            # thousands of steps
-            self.step = step
+            # two synthetic batches alternate, the second's output gradient
+            # the negation of the first's, so that a fixed gradient does not
+            # drive the parameters out of range over thousands of steps
             self.g_alt = -self.g
+            in_names = ("g_alt", "x", "g")   # either batch's (x, g) is one span
+        else:
+            in_names = ("x", "g", "crs", "dgs") + (("sfp",) if case.sfp else ())
+        out_names = ("y", "gx", "codes", "scales", "gcrs", "gdgs") + (("gsfp",) if case.sfp else ())
+        self.in_buf = pack_arena(self, in_names, device)
+        self.out_buf = pack_arena(self, out_names, device)
+        if case.adam:
+            # optimizer state resident in HBM; the paper's learning rates
+            # (Sec. 4.1)
+            self.step = step
             learned = {"crs": self.crs, "dgs": self.dgs}
             if self.sfp is not None:
                 learned["sfp"] = self.sfp
@@ -374,18 +423,23 @@ class BranchGraph:
 
 
 class PipelineGraph:
-    """End-to-end step as a graph of three chained streams: H2D copies of
-    each tensor's inputs, then its phases, then D2H copies of its outputs."""
+    """End-to-end step as a graph of three chained streams: the H2D copy of
+    each tensor's inputs, then its phases, then the D2H copy of its outputs
+    (one copy per tensor and direction: the inputs, and the outputs, share
+    an allocation, mirrored by pinned host buffers of the same layout), so
+    that tensor k's D2H overlaps tensor k+1's H2D on the full-duplex link."""
 
-    def __init__(self, ts, host_in, host_out, phases, device, parity=0, before=None):
+    def __init__(self, ts, phases, device, parity=0, before=None):
         import torch
         # the smallest tensor first (short pipeline fill: its H2D runs alone)
         # and the second smallest last (short drain: its D2H runs alone)
         order = sorted(range(len(ts)), key=lambda i: ts[i].n)
         order = order[:1] + order[2:] + order[1:2] if len(order) > 2 else order
         ts = [ts[i] for i in order]
-        host_in = [host_in[i] for i in order]
-        host_out = [host_out[i] for i in order]
+        spans_in = [arena_spans(t.in_buf, t.inputs(parity)) for t in ts]
+        spans_out = [arena_spans(t.out_buf, t.outputs()) for t in ts]
+        self.h2d = sum(e - s for sp in spans_in for s, e in sp)
+        self.d2h = sum(e - s for sp in spans_out for s, e in sp)
         self.graph = torch.cuda.CUDAGraph()
         s_in, s_cmp, s_out = (torch.cuda.Stream(device) for _ in range(3))
         cap = torch.cuda.Stream(device)
@@ -396,18 +450,18 @@ class PipelineGraph:
                 before()
             for st in (s_in, s_cmp, s_out):
                 st.wait_stream(main)
-            for t, hin, hout in zip(ts, host_in, host_out):
+            for t, sin, sout in zip(ts, spans_in, spans_out):
                 with torch.cuda.stream(s_in):
-                    for d, h in zip(t.inputs(parity), hin):
-                        d.copy_(h, non_blocking=True)
+                    for s, e in sin:
+                        t.in_buf[s:e].copy_(t.host_in[s:e], non_blocking=True)
                 s_cmp.wait_stream(s_in)
                 with torch.cuda.stream(s_cmp):
                     for ph in phases:
                         t.run(ph, parity)
                 s_out.wait_stream(s_cmp)
                 with torch.cuda.stream(s_out):
-                    for h, d in zip(hout, t.outputs()):
-                        h.copy_(d, non_blocking=True)
+                    for s, e in sout:
+                        t.host_out[s:e].copy_(t.out_buf[s:e], non_blocking=True)
             for st in (s_in, s_cmp, s_out):
                 main.wait_stream(st)
         torch.cuda.current_stream(device).wait_stream(cap)
@@ -551,14 +605,12 @@ def gpu_arm(case, args, rank, world, device):
     # (tensor after tensor), a compute chain (tensor k's phases once its
     # inputs are in HBM) and a D2H chain (tensor k's outputs once computed),
     # so that tensor k's D2H overlaps tensor k+1's H2D on the full-duplex link.
-    host_out = [[torch.empty_like(a, device="cpu").pin_memory() for a in t.outputs()] for t in ts]
-    e2e_graphs = []
-    for par in parities:
-        host_in = [[a.cpu().pin_memory() for a in t.inputs(par)] for t in ts]
-        e2e_graphs.append(PipelineGraph(ts, host_in, host_out, phases, device, par,
-                                        before=lambda: before("bwd")))
-    h2d = sum(a.numel() * a.element_size() for h in host_in for a in h)
-    d2h = sum(a.numel() * a.element_size() for h in host_out for a in h)
+    for t in ts:
+        t.host_in = t.in_buf.cpu().pin_memory()   # every batch's inputs
+        t.host_out = torch.empty_like(t.out_buf, device="cpu").pin_memory()
+    e2e_graphs = [PipelineGraph(ts, phases, device, par, before=lambda: before("bwd"))
+                  for par in parities]
+    h2d, d2h = e2e_graphs[-1].h2d, e2e_graphs[-1].d2h
     e2e_steps = max(3, min(args.steps, 20))
     e2e_steps += e2e_steps % len(parities)
     e2e_graphs[0].replay()
