@@ -189,8 +189,15 @@ uint8_t focus_oracle_e4m3_encode(float r)
 /* ------------------------------------------------------------------ */
 /* Shared exponent e of an MXFP4 block with absmax m, clamped to [-127, 127]
  * (E8M0 byte e + 127; 255 is NaN and never produced).
- *   CEIL  (default): e = ceil(log2(fl(m / 6)))  -- the paper's "typically
- *                    ceiling", which never lets |x / 2^e| exceed 6.
+ *   CEIL  (default): e = ceil(log2(m / 6)) of the exact quotient (Eq. 3 with
+ *                    the paper's "typically ceiling"), so |x / 2^e| <= 6.
+ *                    m / 6 is evaluated in binary64: a binary32 m other
+ *                    than 6 * 2^k is at least a relative 2^-23.6 away from
+ *                    it (one ulp of m over 6 * 2^k), far more than binary64
+ *                    rounding moves the quotient, so that quotient is a power
+ *                    of two exactly when m / 6 is.  (The binary32 quotient
+ *                    is not decisive: where it is subnormal, m = 0x01400001
+ *                    rounds to 2^-127.)
  *   FLOOR (option):  e = floor(log2 m) - 2      -- OCP MX v1.0, 2 being the
  *                    largest E2M1 exponent. */
 int focus_oracle_e8m0_exponent(float m, int rule)
@@ -199,14 +206,10 @@ int focus_oracle_e8m0_exponent(float m, int rule)
     if (m == 0.0f) {
         e = -127;
     } else if (rule == OR_MX_CEIL) {
-        float t = m / 6.0f;
-        if (t == 0.0f) {
-            e = -127;                      /* underflowed: below every scale */
-        } else {
-            int E;
-            float f = frexpf(t, &E);       /* t = f * 2^E, f in [0.5, 1) */
-            e = (f == 0.5f) ? E - 1 : E;   /* exact power of two or not */
-        }
+        double t = (double)m / 6.0;
+        int E;
+        double f = frexp(t, &E);           /* t = f * 2^E, f in [0.5, 1) */
+        e = (f == 0.5) ? E - 1 : E;        /* exact power of two or not */
     } else {
         int E;
         frexpf(m, &E);                     /* floor(log2 m) = E - 1 */
@@ -240,7 +243,7 @@ static float block_scale(int fmt, int mx_rule, float m, float alpha, uint8_t* by
  * S^dq = Q_fmt(S^fp), the scale kept in full precision and quantized to the
  * hardware format on the fly.  MXFP4: S^fp is the block scale, rounded up to
  * a power of two (the ceiling reading of Eq. 3, so that S^fp = fl(m/6) gives
- * the absmax scale).  NVFP4: alpha stays frozen and S^fp is the learnable
+ * the absmax scale wherever fl(m/6) is a normal number).  NVFP4: alpha stays frozen and S^fp is the learnable
  * Delta^fp, S^dq = alpha * Q_E4M3(Delta^fp) (so that S^fp = fl(m/fl(alpha*6))
  * gives the absmax scale). */
 static float block_scale_fp(int fmt, float sfp, float alpha, uint8_t* byte)

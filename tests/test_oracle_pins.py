@@ -8,6 +8,7 @@ in the oracle (dropped term, sign, index, transposed operand, off-by-one in an
 exponent rule, wrong tie rule) fails at least one of them.
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -45,12 +46,17 @@ def code_to_value(code):
 
 
 def e8m0_ceil_ref(m):
-    """Smallest e with fl(m/6) <= 2^e, clamped to [-127, 127]."""
-    m = f32(m)
-    t = (m / np.float32(6)).astype(np.float32)
+    """Smallest e with m <= 6 * 2^e (Eq. 3's ceiling of log2(m / 6), exact),
+    clamped to [-127, 127]: start one below floor(log2 m) - 2 and step up
+    while 6 * 2^e < m (binary64 products, exact)."""
+    m = f32(m).astype(np.float64)
     out = np.full(m.shape, -127, np.int64)
-    nz = t > 0
-    out[nz] = np.ceil(np.log2(t[nz].astype(np.float64))).astype(np.int64)
+    nz = m > 0
+    _, ex = np.frexp(m[nz])                       # m in [2^(ex-1), 2^ex)
+    e = ex.astype(np.int64) - 4
+    for _ in range(3):
+        e = np.where(6.0 * np.exp2(e.astype(np.float64)) < m[nz], e + 1, e)
+    out[nz] = e
     return np.clip(out, -127, 127)
 
 
@@ -223,11 +229,58 @@ def test_e8m0_ceil_and_floor_rules():
     assert np.array_equal(O.e8m0_exponent(m, O.MX_FLOOR), e8m0_floor_ref(m))
 
 
+CHUNK = 1 << 24
+
+
+def _sweep(kind, top, first, switch_bits, cap):
+    """Every binary32 pattern below `top` (from 1; from 0 for E4M3), in
+    chunks over a spawn-started process pool."""
+    import concurrent.futures as cf
+    import multiprocessing as mp
+    import oracle_pool
+    lo0 = 0 if kind == "e4m3" else 1
+    jobs = [(kind, lo, min(lo + CHUNK, top), first, switch_bits, cap) for lo in range(lo0, top, CHUNK)]
+    with cf.ProcessPoolExecutor(max_workers=min(16, os.cpu_count() or 1),
+                                mp_context=mp.get_context("spawn")) as ex:
+        bad = [b for b in ex.map(oracle_pool.format_sweep_chunk, jobs) if b >= 0]
+    assert not bad, (kind, hex(bad[0]))
+
+
+def test_e8m0_exhaustive():
+    """Every positive finite binary32 m: the ceiling rule is the smallest e
+    with m <= 6 * 2^e (it steps up right after each 6 * 2^e), the floor rule
+    floor(log2 m) - 2 (it steps up at each power of two), both clamped to
+    [-127, 127]."""
+    six = [int(np.float32(6.0 * 2.0 ** e).view(np.uint32)) + 1 for e in range(-127, 126)]
+    pow2 = [int(np.float32(2.0 ** k).view(np.uint32)) for k in range(-124, 128)]
+    _sweep("e8m0_ceil", 0x7F800000, -127, six, 127)
+    _sweep("e8m0_floor", 0x7F800000, -127, pow2, 127)
+
+
+def test_e4m3_exhaustive():
+    """Every binary32 r in [0, 500]: the code is the nearest finite E4M3
+    value (the table decoded from bias-7 arithmetic), ties to the even code,
+    saturating at 448 -- a step function that switches at each midpoint of
+    two neighbouring values, after it when the lower code is even."""
+    vals = [O.e4m3_decode(b) for b in range(0x7F)]          # 0x00 .. 0x7E, increasing
+    assert all(a < b for a, b in zip(vals, vals[1:]))
+    switches = []
+    for c in range(0x7E):
+        mid = (vals[c] + vals[c + 1]) / 2.0
+        assert float(np.float32(mid)) == mid                  # every midpoint is a binary32
+        bits = int(np.float32(mid).view(np.uint32))
+        switches.append(bits + 1 if c % 2 == 0 else bits)
+    _sweep("e4m3", int(np.float32(500.0).view(np.uint32)) + 1, 0, switches, 0x7E)
+
+
 def test_e8m0_ceil_never_saturates():
     """Under the ceiling rule the block maximum never exceeds 6 * 2^e, so at
     c = 1 no element saturates; and 2^e is the tightest such power."""
     rng = np.random.default_rng(9)
     m = rng.integers(0x00800000, 0x7F000000, 1_000_000, dtype=np.uint32).view(np.float32)
+    # where fl(m / 6) is subnormal it can round onto 2^-127: 0x01400001 is
+    # just above 6 * 2^-127 and needs e = -126
+    m = np.concatenate([m, np.array([0x01400000, 0x01400001, 0x01400002], np.uint32).view(np.float32)])
     e = O.e8m0_exponent(m, O.MX_CEIL).astype(np.float64)
     ok = e < 127
     ratio = m[ok].astype(np.float64) / np.exp2(e[ok])
