@@ -140,18 +140,23 @@ __device__ __forceinline__ float e4m3_decode(uint32_t byte)
 // ---------------------------------------------------------------------------
 // E8M0 (Eq. 3): shared exponent of an MXFP4 block with absmax m >= 0,
 // clamped to [-127, 127].  rule 0 (ceiling, the paper's "typically ceiling"):
-// e = ceil(log2(fl(m / 6))), read exactly off the bits of the quotient;
-// rule 1 (OCP MX v1.0): e = floor(log2 m) - 2.
+// e = ceil(log2(m / 6)), so that no |x| / 2^e exceeds 6; rule 1 (OCP MX
+// v1.0): e = floor(log2 m) - 2.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int mx_exponent(float m, int rule)
 {
     int e;
     if (rule == 0) {
+        // ceil(log2(m / 6)) of the exact quotient.  A normal binary32
+        // quotient is a power of two only when m / 6 is one (m other than
+        // 6 * 2^k is a relative 2^-23.6 or more away from it, fl moves by
+        // 2^-24 at most); a subnormal one is not decisive (m = 0x01400001
+        // rounds to 2^-127), so there m is compared with 6 * 2^-127 itself.
         const uint32_t b = __float_as_uint(__fdiv_rn(m, 6.0f));
         const int E = static_cast<int>(b >> 23);
         const uint32_t M = b & 0x7fffffu;
-        // subnormal or zero quotient: only values above 2^-127 reach -126
-        e = (E == 0) ? (M > 0x400000u ? -126 : -127) : (E - 127 + (M != 0u ? 1 : 0));
+        e = (E == 0) ? (m > __uint_as_float(0x01400000u) ? -126 : -127)
+                     : (E - 127 + (M != 0u ? 1 : 0));
     } else {
         const int E = static_cast<int>(__float_as_uint(m) >> 23);
         e = (E == 0) ? -127 : E - 129;
@@ -246,7 +251,8 @@ __device__ __forceinline__ float nv_scale(float m, float alpha, float den, const
 }
 
 // MXFP4 ceiling exponent with the quotient m / 6 estimated (see above):
-// only whether fl(m/6) is a power of two, and its binade, matter.
+// only whether m / 6 is a power of two, and its binade, matter; quotients
+// near the subnormal range take the exact path.
 __device__ __forceinline__ int mx_exponent_fast(float m, int rule)
 {
     if (rule == 0) {

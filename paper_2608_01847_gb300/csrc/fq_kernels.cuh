@@ -445,24 +445,24 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
         for (int k = 0; k < K; ++k) br[k] = make_bracket(sq[k]);
     }
     uint32_t cw = 0u;
-    const float rs = SFPG ? rcp_approx(sdq) : 0.0f;
     gS = {0.0f, 0.0f};
+    Sum2x2 accq;   // sum of g q over the block: q = 0 on dead sub-blocks
 #pragma unroll
     for (int k = 0; k < K; ++k) {
-        Sum2x2 acc, accq;
+        Sum2x2 acc;
 #pragma unroll
         for (int e = k * SUB; e < (k + 1) * SUB; e += 2) {
             const float2 x2 = elem_pair<DT>(xw, e / 2);
             float2 g2 = elem_pair<DT>(gw, e / 2);
             if constexpr (SFPG) {
-                // g * q over the sub-block (q: 2 significant bits, so exact
-                // for bf16 g); the q term of dy/dS^dq is not masked
+                // g * q over the block (q: 2 significant bits, so exact for
+                // bf16 g); the q term of dy/dS^dq is not masked
                 if (e % 8 == 0) cw = word_codes<DT, B, K>(xw, e / 8, sq, dead, br);
                 const uint32_t cb = (cw >> (4 * (e % 8))) & 0xffu;
                 const uint32_t h2 = e2m1x2_to_f16x2(cb);
                 const float2 q2 = __half22float2(*reinterpret_cast<const __half2*>(&h2));
                 const float2 p = mul2(g2, q2);
-                if (e == k * SUB) {
+                if (e == 0) {
                     accq.s = p;
                     accq.c = make_float2(0.0f, 0.0f);
                 } else {
@@ -499,16 +499,18 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
             const df qk = df_div_f(T[k], d[k], rd);
             gd[k] = -__fmul_rn(__fmul_rn(df_to_f(qk), rd), rc);
             Q = (k == 0) ? qk : df_add(Q, qk);
-            if constexpr (SFPG) {
-                // dL/dS^dq over the sub-block: sum g q - T_k / (S^dq c c^k)
-                if (!dead[k]) {
-                    const df u = df_div_f(df_div_f(qk, c, rc), sdq, rs);
-                    gS = df_add(gS, df_add(sum2x2_merge(accq), df{-u.h, -u.l}));
-                }
-            }
         }
     }
     gc = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
+    if constexpr (SFPG) {
+        // dL/dS^dq = sum_k (sum g q - T_k / (S^dq c c^k)) over the live
+        // sub-blocks = sum g q - Q / (c S^dq), Q = sum_k T_k / c^k (dead
+        // sub-blocks have q = 0 and T_k = 0)
+        if (sdq != 0.0f) {
+            const df u = df_div_f(df_div_f(Q, c, rc), sdq, rcp_approx(sdq));
+            gS = df_add(sum2x2_merge(accq), df{-u.h, -u.l});
+        }
+    }
 }
 
 // Coefficient gradients from finished sub-block sums (the shared-row
