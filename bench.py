@@ -969,6 +969,27 @@ def gemm_arm(args, device):
     big_ms = e0.elapsed_time(e1) / n_rep
     big_flops = 2 * GEMM_TOKENS * w.tensors[big].rows * w.tensors[big].cols
     assert int(flag.item()) == 0, "a GEMM wait gave up"
+    # context: NVIDIA's block-scaled GEMM (cuBLASLt through torch._scaled_mm)
+    # on the same exports and the same largest projection, where the
+    # installed torch has the FP4 path (NVFP4 only; alpha applied outside)
+    library = None
+    if fmt == F.FOCUS_NVFP4 and hasattr(torch, "float4_e2m1fn_x2"):
+        try:
+            a4, w4 = ac.view(torch.float4_e2m1fn_x2), wc.view(torch.float4_e2m1fn_x2).t()
+            sa, sw = at.view(torch.float8_e4m3fn), wt.view(torch.float8_e4m3fn)
+            for _ in range(3):
+                torch._scaled_mm(a4, w4, sa, sw, out_dtype=torch.bfloat16)
+            e0.record(stream)
+            for _ in range(n_rep):
+                torch._scaled_mm(a4, w4, sa, sw, out_dtype=torch.bfloat16)
+            e1.record(stream)
+            torch.cuda.synchronize(device)
+            lib_ms = e0.elapsed_time(e1) / n_rep
+            library = {"call": "torch._scaled_mm (cuBLASLt block-scaled NVFP4, bf16 out) on the same exports",
+                       "kernel": w.tensors[big].name,
+                       "tflops": round(big_flops / (lib_ms * 1e-3) / 1e12, 1)}
+        except (RuntimeError, TypeError, NotImplementedError) as e:
+            library = {"unavailable": str(e).splitlines()[0][:160]}
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             bf16 = float(json.load(f)["bf16_tflops"])
@@ -989,6 +1010,7 @@ def gemm_arm(args, device):
                      "achieved": round(big_tflops, 1), "peak": round(peak, 1), "peak_kind": peak_kind,
                      "unit": "TFLOP/s", "frac": round(big_tflops / peak, 4), "traffic": None},
         "clocks": clk.summary(), "gpu_launches": args.steps * len(jobs),
+        **({"library_reference": library} if library is not None else {}),
     }
 
 
