@@ -157,3 +157,52 @@ def test_fp4_gemm_bf16_output(fmt):
     assert torch.equal(d16, d32.to(torch.bfloat16))
     assert torch.equal(wide[:, :N], d16)
     assert torch.count_nonzero(wide[:, N:]) == 0
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+def test_fp4_gemm_full_size_sampled(fmt):
+    """The benchmark's largest Qwen3-4B GEMM at full size (8192 tokens x
+    gate_proj [9728, 2560]: 1216 tile pairs, 16 per cluster, so every
+    barrier of the ring and of the accumulator wraps many times), with fp32
+    and with bf16 output: D on 32 sampled rows x 32 sampled columns (first,
+    last, random) against the oracle's contraction of the oracle's export of
+    those rows, whose codes and scale bytes also match the GPU export."""
+    f = FMT[fmt]
+    M, N, K = 8192, 9728, 2560
+    block = 32 if f == O.MXFP4 else 16
+    _, xa = operand(M, K, 21, "act")
+    _, xb = operand(N, K, 22, "weight")
+    aa = O.alpha(xa) if f == O.NVFP4 else 0.0
+    ab = O.alpha(xb) if f == O.NVFP4 else 0.0
+    da, db = dev(xa), dev(xb)
+    aa_dev = torch.tensor([aa], dtype=torch.float32, device="cuda")
+    ab_dev = torch.tensor([ab], dtype=torch.float32, device="cuda")
+    ac, at = F.focus_pack_mma(da, f, alpha=aa_dev)
+    bc, bt = F.focus_pack_mma(db, f, alpha=ab_dev)
+    # the same exports, row-major scale bytes (to compare sampled rows)
+    ac2, as2 = F.focus_pack(da, f, alpha=aa_dev)
+    bc2, bs2 = F.focus_pack(db, f, alpha=ab_dev)
+    flag = torch.zeros(1, dtype=torch.int32, device="cuda")
+    d32 = F.focus_fp4_gemm(f, ac, at, bc, bt, aa_dev, ab_dev, timeout_flag=flag)
+    d16 = F.focus_fp4_gemm(f, ac, at, bc, bt, aa_dev, ab_dev, out_dtype=torch.bfloat16, timeout_flag=flag)
+    torch.cuda.synchronize()
+    assert int(flag.item()) == 0, "MMA wait gave up"
+    rng = np.random.default_rng(7 + f)
+    ma = np.unique(np.concatenate([[0, M - 1], rng.choice(M, 30, replace=False)]))
+    nb = np.unique(np.concatenate([[0, N - 1], rng.choice(N, 30, replace=False)]))
+    ra = O.fwd(xa[ma], f, alpha=aa, want_y=False, want_codes=True)
+    rb = O.fwd(xb[nb], f, alpha=ab, want_y=False, want_codes=True)
+    assert_bits_equal(host(ac2)[ma], ra["codes"], "A codes")
+    assert_bits_equal(host(as2)[ma], ra["scales"], "A scale bytes")
+    assert_bits_equal(host(bc2)[nb], rb["codes"], "B codes")
+    assert_bits_equal(host(bs2)[nb], rb["scales"], "B scale bytes")
+    assert torch.equal(ac, ac2) and torch.equal(bc, bc2)
+    ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], f, aa, ab)
+    mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], f, aa, ab)
+    bound = (K / 16 + 8) * 2.0 ** -23 * mag + 2.0 ** -23 * np.abs(ref) + 1e-30
+    ia, ib = torch.from_numpy(ma).cuda(), torch.from_numpy(nb).cuda()
+    got32 = host(d32[ia][:, ib]).astype(np.float64)
+    got16 = host(d16[ia][:, ib].float()).astype(np.float64)
+    assert np.all(np.abs(got32 - ref) <= bound), "fp32 output"
+    # bf16 output: the fp32 result rounded once more (half an ulp of bf16)
+    assert np.all(np.abs(got16 - ref) <= bound + 2.0 ** -8 * (np.abs(ref) + bound)), "bf16 output"
