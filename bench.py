@@ -39,6 +39,10 @@ if ROOT not in sys.path:
 
 METRIC = "fake-quant fwd+bwd GB/s and elems/s vs GB300 HBM peak; pack GB/s"
 L2_BYTES = 129 * 1024 * 1024
+# phase split: each phase captured this many times in one graph (the tensors
+# joined between repetitions), so that a phase's time excludes the gap
+# between graph replays
+PHASE_REPS = 8
 
 
 @dataclasses.dataclass(frozen=True)
@@ -509,15 +513,25 @@ def gpu_arm(case, args, rank, world, device):
             for t in ts:
                 t.run(ph)
     torch.cuda.synchronize(device)
-    # one graph per phase (for the phase split) and one for the whole step;
-    # with the optimizer, one of each per batch parity (alternating batches)
+    # Inputs that fit in L2 would stay there between back-to-back steps: then
+    # every timed step (and phase) follows a write of twice the L2 size, and
+    # the events bracket each step alone; the back-to-back figure is kept as
+    # the "L2-resident" one.
+    in_bytes = sum(t.x.numel() * t.x.element_size() * 2 for t in ts)
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device) if in_bytes <= L2_BYTES else None
+
+    # one graph per phase (for the phase split: PHASE_REPS repetitions, or
+    # one per flushed replay) and one for the whole step; with the optimizer,
+    # one of each per batch parity (alternating batches)
     parities = (0, 1) if case.adam else (0,)
+    reps = 1 if flush is not None else PHASE_REPS
     if grouped:
-        graphs = {ph: [SeqGraph(runner.run, device, (ph,))] for ph in phases}
+        graphs = {ph: [SeqGraph(runner.run, device, (ph,) * reps)] for ph in phases}
         step_graphs = [SeqGraph(runner.run, device, phases)]
     else:
-        graphs = {ph: [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
-                                   stages=(ph,), before=before) for par in parities]
+        graphs = {ph: [BranchGraph(len(ts), lambda i, st: ts[i].run(st[0], st[1]), device,
+                                   stages=tuple((ph, (par + r) % len(parities)) for r in range(reps)),
+                                   before=lambda st: before(st[0])) for par in parities]
                   for ph in phases}
         if args.staged:
             step_graphs = [BranchGraph(len(ts), lambda i, st, par=par: ts[i].run(st, par), device,
@@ -542,13 +556,6 @@ def gpu_arm(case, args, rank, world, device):
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize(device)
-
-    # Inputs that fit in L2 would stay there between back-to-back steps: then
-    # every timed step (and phase) follows a write of twice the L2 size, and
-    # the events bracket each step alone; the back-to-back figure is kept as
-    # the "L2-resident" one.
-    in_bytes = sum(t.x.numel() * t.x.element_size() * 2 for t in ts)
-    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device) if in_bytes <= L2_BYTES else None
 
     def timed(run, n):
         """ms of n runs: back to back, or (flush) each after an L2 flush."""
@@ -580,7 +587,7 @@ def gpu_arm(case, args, rank, world, device):
     phase_ms = {}
     n_split = max(1, min(args.steps, 100))
     for name, gph in graphs.items():
-        phase_ms[name] = timed(lambda k: gph[k % len(parities)].replay(), n_split) * args.steps / n_split
+        phase_ms[name] = timed(lambda k: gph[k % len(parities)].replay(), n_split) * args.steps / n_split / reps
     total_ms = max_over_ranks(total_ms, world, device)
     l2_resident_ms = None
     if flush is not None:
@@ -592,7 +599,7 @@ def gpu_arm(case, args, rank, world, device):
         torch.cuda.synchronize(device)
         l2_resident_ms = max_over_ranks(a.elapsed_time(b), world, device)
 
-    res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, clocks=clk.summary(),
+    res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, phase_reps=reps, clocks=clk.summary(),
                l2_flushed=flush is not None, l2_resident_ms=l2_resident_ms,
                ntensors=len(ts), grouped=grouped,
                launches_per_step=(sum(GroupRunner.launches(ph) for ph in phases) if grouped else
@@ -1115,7 +1122,10 @@ def main():
                           "each step" if r["l2_flushed"] else
                           f"inputs larger than L2: x+g = {r['n_elem'] * 2 * r['esz'] / 2**20:.0f} MiB"
                           " per step"),
-                   "parallelism": f"replicas x{world}"},
+                   "parallelism": f"replicas x{world}",
+                   "phase_split": (f"each phase captured {r['phase_reps']} times in one graph (tensors joined "
+                                   "between repetitions), timed per repetition" if r["phase_reps"] > 1 else
+                                   "each phase graph timed per replay")},
         "elems_per_s": round(world * r["n_elem"] / (ms_step * 1e-3), 1),
         "fwd_bwd_gbs": round(fb_bytes / ((ph["fwd"] + ph["bwd"]) * 1e-3) / 1e9, 2),
         "pack_gbs": round(gbs["pack"], 2),
