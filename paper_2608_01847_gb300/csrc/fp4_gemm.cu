@@ -306,31 +306,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
             for (uint32_t c = 0; c < n_chunks; ++c, ++k) {
-                bool got = tc::mbar_wait_hot(&full[s], ph, kWaitLimit);
-                if (kChunksPerSet == 1 && k >= kSfSets) {
-                    const uint32_t k2 = k - kSfSets;
-                    got = got && tc::mbar_wait_hot(&empty[k2 % kStages], (k2 / kStages) & 1u, kWaitLimit);
-                }
-                if (!__all_sync(0xffffffffu, got)) {
+                // the chunk's scale lines into registers as soon as its stage
+                // has landed, before waiting for its scale set to be free
+                if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&full[s], ph, kWaitLimit))) {
                     if (lane == 0) give_up(p);
                     ok = false;
                     break;
                 }
-                tc::tc_fence_after();
                 const uint32_t steps = min(4u, p.n_steps - 4 * c);
                 const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
+                uint32_t la[kTilesPerChunk];
+                uint4 lb[kTilesPerChunk], lh[kTilesPerChunk];
+#pragma unroll
+                for (uint32_t j = 0; j < kTilesPerChunk; ++j) {
+                    if (j < sf_tiles) {
+                        // A: quarter q reads only column q of the region (row q * 32 + lane)
+                        la[j] = *reinterpret_cast<const uint32_t*>(stage_sfa(s) + 512 * j + 16 * lane + 4 * q);
+                        lb[j] = *reinterpret_cast<const uint4*>(stage_sfb(s) + 512 * j + 16 * lane);
+                        lh[j] = *reinterpret_cast<const uint4*>(stage_sfb(s) + kSfBytes + 512 * j + 16 * lane);
+                    }
+                }
+                if (kChunksPerSet == 1 && k >= kSfSets) {
+                    const uint32_t k2 = k - kSfSets;
+                    if (!__all_sync(0xffffffffu,
+                                    tc::mbar_wait_hot(&empty[k2 % kStages], (k2 / kStages) & 1u, kWaitLimit))) {
+                        if (lane == 0) give_up(p);
+                        ok = false;
+                        break;
+                    }
+                }
+                tc::tc_fence_after();
                 const uint32_t set = (k / kChunksPerSet) % kSfSets;
                 const uint32_t sfbase =
                     lane_addr + kSfBase + kSfSet * set + kSfStep * kTilesPerChunk * (k % kChunksPerSet);
-                for (uint32_t j = 0; j < sf_tiles; ++j) {
-                    // A: quarter q reads only column q of the region (row q * 32 + lane)
-                    const uint32_t la = *reinterpret_cast<const uint32_t*>(stage_sfa(s) + 512 * j + 16 * lane + 4 * q);
-                    const uint4 lb = *reinterpret_cast<const uint4*>(stage_sfb(s) + 512 * j + 16 * lane);
-                    const uint4 lh = *reinterpret_cast<const uint4*>(stage_sfb(s) + kSfBytes + 512 * j + 16 * lane);
-                    tc::tmem_st_x1(sfbase + kSfStep * j + q, la);
-                    // rows 128-255 of B (stale but finite-or-not bytes when B has no such
-                    // rows: they only reach columns of D that are not stored)
-                    tc::tmem_st_x8(sfbase + kSfb + kSfStep * j, lb.x, lb.y, lb.z, lb.w, lh.x, lh.y, lh.z, lh.w);
+#pragma unroll
+                for (uint32_t j = 0; j < kTilesPerChunk; ++j) {
+                    if (j < sf_tiles) {
+                        tc::tmem_st_x1(sfbase + kSfStep * j + q, la[j]);
+                        // rows 128-255 of B (stale but finite-or-not bytes when B has no
+                        // such rows: they only reach columns of D that are not stored)
+                        tc::tmem_st_x8(sfbase + kSfb + kSfStep * j, lb[j].x, lb[j].y, lb[j].z, lb[j].w, lh[j].x,
+                                       lh[j].y, lh[j].z, lh[j].w);
+                    }
                 }
                 tc::tmem_wait_st();
                 tc::tc_fence_before();
