@@ -413,15 +413,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // accumulator is released before any staging
                     uint32_t w[kTileN / 2];
 #pragma unroll
-                    for (int cb = 0; cb < kTileN / 32; ++cb) {
-                        uint32_t r[32];
-                        tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * cb, r);
+                    for (int cb = 0; cb < kTileN / 32; cb += 2) {
+                        // two loads in flight per wait
+                        uint32_t r[2][32];
+                        tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * cb, r[0]);
+                        tc::tmem_ld_x32(lane_addr + acc * kTileN + 32 * (cb + 1), r[1]);
                         tc::tmem_wait_ld();
 #pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const __nv_bfloat162 h = __floats2bfloat162_rn(
-                                __fmul_rn(__uint_as_float(r[2 * e]), scale), __fmul_rn(__uint_as_float(r[2 * e + 1]), scale));
-                            w[16 * cb + e] = *reinterpret_cast<const uint32_t*>(&h);
+                        for (int hb = 0; hb < 2; ++hb) {
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const __nv_bfloat162 h = __floats2bfloat162_rn(__fmul_rn(__uint_as_float(r[hb][2 * e]), scale),
+                                                                               __fmul_rn(__uint_as_float(r[hb][2 * e + 1]), scale));
+                                w[16 * (cb + hb) + e] = *reinterpret_cast<const uint32_t*>(&h);
+                            }
                         }
                     }
                     tc::tc_fence_before();
