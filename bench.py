@@ -5,18 +5,26 @@ decoder layer (7 bf16 projections, 100.9 M elements), NVFP4 (block 16, E4M3
 + fp32 alpha), per-block CRS and per-sub-block (8) DGS coefficients:
   alpha (per tensor)  ->  fake-quant forward  ->  STE backward (input
   gradient + both coefficient gradients)  ->  export pack,
-each phase over all tensors before the next (as a calibration step runs all
-forwards, then all backwards), inputs resident in HBM.  The step is captured
-once as a CUDA graph: the phases in order, each phase's tensors on parallel
-branches that join before the next phase.  `value` is the algorithmic bytes of the
-step (per-element figures in bytes_per_elem) over the step time.
+inputs resident in HBM.  The step is captured once as a CUDA graph: each
+tensor's four phases chained on its own branch (programmatic dependent
+launches), the tensors' branches side by side; `--staged` joins all tensors
+between phases instead, `--group` runs each phase as one group launch.
+`value` is the algorithmic bytes of the step (per-element figures in
+bytes_per_elem) over the step time.  The JSON line also carries the phase
+split, the roofline of the dominant kernel, the end-to-end figure (pinned
+host buffers, copies inside the timed region), the CPU oracle baseline and
+the SM clocks sampled during the timed region.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
-                  [--workload NAME --fmt mxfp4|nvfp4 --shared]
+                  [--workload NAME --fmt mxfp4|nvfp4 --shared --sfp --adam
+                   --io f16 --sub B --staged --group --no-e2e --no-cpu-baseline]
+  python bench.py --gemm [--fmt mxfp4] [--workload NAME]
 
 Other workloads (the Llama-3-8B block, the 70B layer set, the W4A4
-activations, a sweep tensor) are measured the same way with --workload; the
-driver's line is the default case.
+activations, sweep tensors) are measured the same way with --workload; the
+default line is the Qwen3-4B layer.  `--impl reference` times the CPU
+oracle on a bounded sample of the same workload.  `--gemm` times the W4A4
+FP4 GEMMs of a layer's projections on their exports.
 
 Under torchrun (N > 1) every rank runs the same workload on its own GPU
 (replicas; no data-path collective), the step time is the max over ranks and
