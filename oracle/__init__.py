@@ -1,7 +1,7 @@
 """CPU oracle for the FOCUS FP4 fake-quantizer -- TEST INFRASTRUCTURE ONLY.
 
-Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
-``bench.py`` may import this package.  The product path (the CUDA library
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU legs of ``bench.py``
+(the CPU baseline and ``--impl reference``) may import this package.  The product path (the CUDA library
 under ``paper_2608_01847_gb300``) never imports it and shares no code with it.
 
 The arithmetic lives in ``focus_oracle.c`` (plain scalar C, binary32 forward,
