@@ -55,7 +55,7 @@ PHASE_REPS = 8
 
 @dataclasses.dataclass(frozen=True)
 class Case:
-    workload: str = "qwen3_4b_layer"
+    workload: str = "act_262144x4096"
     fmt: str = "nvfp4"
     sub: int = 8
     shared: bool = False       # one coefficient set for all rows (activations)
@@ -87,12 +87,12 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
     return out
 
 
-# DRAM traffic (read + write) of one backward phase of the default case,
-# from an ncu launch list of this benchmark (gpu__time_duration,
-# dram__bytes_read, dram__bytes_write; --cache-control none), and the sha256
-# prefix of the kernel sources it was taken on.  Reported only for the
-# default case and while the sources are unchanged.
-BWD_TRAFFIC = {"sources": "c7a077727c6cb778", "bytes_per_step": 702.7e6}
+# DRAM traffic (read + write) of the dominant kernel of the default line,
+# per element, from one ncu capture of that kernel on a smaller case of the
+# same workload (DRAM bytes scale with the elements processed), keyed by
+# (workload, format, phase), with the sha256 prefix of the kernel sources it
+# was taken on.  Reported only while the sources are unchanged.
+TRAFFIC = {}
 
 # AdamW hyper-parameters of the fused optimizer: the paper's learning rates
 # per format (Sec. 4.1: block scale / relaxation coefficients) and PyTorch's
@@ -131,50 +131,144 @@ def load_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clocks, power and throttle reasons of one GPU, sampled every
+    `period_s` in a background thread while the benchmark runs, read-only:
+    through NVML (the driver's libnvidia-ml, queried with ctypes), else by
+    an nvidia-smi child process.  `mark(name)` stamps the host time of a
+    moment of the run (after a device synchronize, so the stamps bracket the
+    device work); `summary(a, b)` reduces the samples taken between two
+    stamps."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+    # NVML clock-event reason bits (nvml.h): SW power cap 0x4, HW slowdown
+    # 0x8, SW thermal 0x20, HW thermal 0x40, HW power brake 0x80 (a HW slowdown)
+    REASON_BITS = {"hw_slowdown": 0x8 | 0x80, "hw_thermal_slowdown": 0x40,
+                   "sw_thermal_slowdown": 0x20, "sw_power_cap": 0x4}
 
-    def __init__(self, index):
-        self.index = index
-        self.proc = None
-        self.out = ""
+    def __init__(self, index, uuid=None, period_s=0.01):
+        self.index, self.uuid, self.period = index, uuid, period_s
+        self.samples = []          # (host time, sm MHz, max sm MHz, power W, [reason names])
+        self.marks = {}
+        self.source = None
+        self.error = None
+        self._stop = None
+        self._thread = None
+        self._proc = None
+
+    # -- NVML -------------------------------------------------------------
+    def _nvml_open(self):
+        import ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit_v2 failed")
+        h = ctypes.c_void_p()
+        ok = False
+        if self.uuid:
+            ok = lib.nvmlDeviceGetHandleByUUID(("GPU-" + self.uuid).encode(), ctypes.byref(h)) == 0
+        if not ok and lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(self.index), ctypes.byref(h)) != 0:
+            lib.nvmlShutdown()
+            raise OSError("no NVML handle for the device")
+        reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        return lib, h, reasons_fn
+
+    def _nvml_loop(self, lib, h, reasons_fn):
+        import ctypes
+        clk, mx, pw, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        try:
+            while not self._stop.is_set():
+                if (lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and
+                        lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0 and
+                        reasons_fn(h, ctypes.byref(rs)) == 0):
+                    power = pw.value / 1000.0 if lib.nvmlDeviceGetPowerUsage(h, ctypes.byref(pw)) == 0 else None
+                    names = [n for n, bit in self.REASON_BITS.items() if rs.value & bit]
+                    self.samples.append((time.monotonic(), float(clk.value), float(mx.value), power, names))
+                self._stop.wait(self.period)
+        finally:
+            lib.nvmlShutdown()
+
+    # -- nvidia-smi ---------------------------------------------------------
+    def _smi_loop(self):
+        names = list(self.REASON_BITS)
+        for ln in self._proc.stdout:
+            f = [v.strip() for v in ln.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                power = float(f[2]) if f[2] not in ("", "[N/A]") else None
+                self.samples.append((time.monotonic(), float(f[0]), float(f[1]), power,
+                                     [n for n, v in zip(names, f[3:7]) if v.lower() == "active"]))
+            except ValueError:
+                continue
 
     def __enter__(self):
+        import threading
+        self._stop = threading.Event()
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-        except Exception:
-            self.proc = None
+            lib, h, reasons_fn = self._nvml_open()
+            self.source = "nvml"
+            self._thread = threading.Thread(target=self._nvml_loop, args=(lib, h, reasons_fn), daemon=True)
+        except (OSError, AttributeError) as e:
+            self.error = f"nvml: {e}"
+            try:
+                self._proc = subprocess.Popen(
+                    ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                     "--format=csv,noheader,nounits", "-lms", str(max(20, int(self.period * 1000)))],
+                    stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True)
+                self.source = "nvidia-smi"
+                self._thread = threading.Thread(target=self._smi_loop, daemon=True)
+            except OSError as e2:
+                self.error += f"; nvidia-smi: {e2}"
+        if self._thread is not None:
+            self._thread.start()
+        self.mark("start")
         return self
 
     def __exit__(self, *a):
-        if self.proc is not None:
-            self.proc.terminate()
+        self.mark("end")
+        if self._stop is not None:
+            self._stop.set()
+        if self._proc is not None:
+            self._proc.terminate()
             try:
-                self.out, _ = self.proc.communicate(timeout=5)
+                _, err = self._proc.communicate(timeout=5)
+                if not self.samples and err:
+                    self.error = (self.error or "") + "; nvidia-smi: " + err.strip()[:200]
             except Exception:
-                self.proc.kill()
+                self._proc.kill()
+        if self._thread is not None:
+            self._thread.join(timeout=5)
 
-    def summary(self):
-        rows = []
-        for ln in (self.out or "").splitlines():
-            f = [s.strip() for s in ln.split(",")]
-            if len(f) < 9:
-                continue
-            try:
-                rows.append((float(f[1]), float(f[2]), f[5:9], f[4]))
-            except ValueError:
-                continue
+    def mark(self, name):
+        self.marks[name] = time.monotonic()
+
+    def summary(self, a="start", b="end"):
+        t0, t1 = self.marks.get(a, 0.0), self.marks.get(b, float("inf"))
+        rows = [r for r in self.samples if t0 <= r[0] <= t1]
+        out = {"source": self.source, "window": f"{a}..{b}", "samples": len(rows),
+               "period_ms": round(self.period * 1e3, 1)}
         if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[2]) if v.lower() == "active"})
-        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
-                "reasons": reasons, "samples": len(rows)}
+            out.update(sm_mhz=None, sm_max_mhz=None, reasons=["unavailable"])
+            if self.error:
+                out["error"] = self.error
+            return out
+        pw = [r[3] for r in rows if r[3] is not None]
+        out.update(sm_mhz=statistics.median(r[1] for r in rows), sm_min_mhz=min(r[1] for r in rows),
+                   sm_max_mhz=max(r[2] for r in rows),
+                   reasons=sorted({n for r in rows for n in r[4]}),
+                   power_w_max=round(max(pw), 1) if pw else None)
+        return out
+
+
+def device_uuid(device):
+    """The CUDA device's UUID as NVML spells it after "GPU-", or None."""
+    try:
+        import torch
+        u = str(torch.cuda.get_device_properties(device).uuid)
+        return u if len(u) >= 32 else None
+    except Exception:
+        return None
 
 
 # ----------------------------------------------------------------------------
@@ -556,9 +650,9 @@ def gpu_arm(case, args, rank, world, device):
         step_graphs[n_replay[0] % len(parities)].replay()
         n_replay[0] += 1
 
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize(device)
+    # clocks sampled from the warm-up to the end of the phase split; the
+    # line's `clocks` covers the timed steps alone
+    clk = ClockSampler(device.index if device.index is not None else 0, device_uuid(device))
 
     def barrier():
         if world > 1:
@@ -587,15 +681,25 @@ def gpu_arm(case, args, rank, world, device):
         return sum(a.elapsed_time(b) for a, b in evs)
 
     # ---- device-resident timing: K steps ----
-    with ClockSampler(device.index if device.index is not None else 0) as clk:
+    clk.__enter__()
+    try:
+        for _ in range(args.warmup):
+            step()
         barrier()
+        clk.mark("timed_start")
         total_ms = timed(lambda k: step(), args.steps)
         barrier()
-    # phase split: each phase graph replayed on its own, timed the same way
-    phase_ms = {}
-    n_split = max(1, min(args.steps, 100))
-    for name, gph in graphs.items():
-        phase_ms[name] = timed(lambda k: gph[k % len(parities)].replay(), n_split) * args.steps / n_split / reps
+        clk.mark("timed_end")
+        # phase split: each phase graph replayed on its own, timed the same way
+        phase_ms = {}
+        n_split = max(1, min(args.steps, 100))
+        for name, gph in graphs.items():
+            phase_ms[name] = timed(lambda k: gph[k % len(parities)].replay(), n_split) * args.steps / n_split / reps
+        torch.cuda.synchronize(device)
+    finally:
+        clk.__exit__()
+    clocks = clk.summary("timed_start", "timed_end")
+    clocks["run"] = {k: v for k, v in clk.summary().items() if k not in ("source", "period_ms")}
     total_ms = max_over_ranks(total_ms, world, device)
     l2_resident_ms = None
     if flush is not None:
@@ -607,7 +711,7 @@ def gpu_arm(case, args, rank, world, device):
         torch.cuda.synchronize(device)
         l2_resident_ms = max_over_ranks(a.elapsed_time(b), world, device)
 
-    res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, phase_reps=reps, clocks=clk.summary(),
+    res = dict(n_elem=n_elem, esz=esz, total_ms=total_ms, phase_ms=phase_ms, phase_reps=reps, clocks=clocks,
                l2_flushed=flush is not None, l2_resident_ms=l2_resident_ms,
                ntensors=len(ts), grouped=grouped,
                launches_per_step=(sum(GroupRunner.launches(ph) for ph in phases) if grouped else
@@ -964,13 +1068,16 @@ def gemm_arm(args, device):
     graph.replay()
     torch.cuda.synchronize(device)
     stream = torch.cuda.current_stream(device)
-    with ClockSampler(device.index if device.index is not None else 0) as clk:
+    with ClockSampler(device.index if device.index is not None else 0, device_uuid(device)) as clk:
+        torch.cuda.synchronize(device)
+        clk.mark("timed_start")
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
             graph.replay()
         e1.record(stream)
         torch.cuda.synchronize(device)
+        clk.mark("timed_end")
     ms = e0.elapsed_time(e1) / args.steps
     # dominant launch: the largest projection alone
     big = max(range(len(jobs)), key=lambda j: jobs[j][2].numel() * w.tensors[j].cols)
@@ -1024,7 +1131,7 @@ def gemm_arm(args, device):
         "roofline": {"bound": "tensor", "kernel": f"fp4_gemm_kernel ({w.tensors[big].name})",
                      "achieved": round(big_tflops, 1), "peak": round(peak, 1), "peak_kind": peak_kind,
                      "unit": "TFLOP/s", "frac": round(big_tflops / peak, 4), "traffic": None},
-        "clocks": clk.summary(), "gpu_launches": args.steps * len(jobs),
+        "clocks": clk.summary("timed_start", "timed_end"), "gpu_launches": args.steps * len(jobs),
         **({"library_reference": library} if library is not None else {}),
     }
 
@@ -1032,10 +1139,11 @@ def gemm_arm(args, device):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="focus", choices=["focus", "reference"])
-    ap.add_argument("--workload", default="qwen3_4b_layer")
+    ap.add_argument("--workload", default=None,
+                    help="default: act_262144x4096 (qwen3_4b_layer with --gemm)")
     ap.add_argument("--fmt", default="nvfp4", choices=["nvfp4", "mxfp4"])
     ap.add_argument("--sub", type=int, default=8)
     ap.add_argument("--shared", action="store_true", help="coefficients shared by all rows")
@@ -1055,6 +1163,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args()
+    if args.workload is None:
+        args.workload = "qwen3_4b_layer" if args.gemm else Case().workload
     case = Case(args.workload, args.fmt, args.sub, args.shared, args.sfp, args.adam, args.io)
     default_case = case == Case()
 
@@ -1087,12 +1197,44 @@ def main():
             print(json.dumps(gemm_arm(args, device)))
         return
     r = gpu_arm(case, args, rank, world, device)
+    # the default line also carries the other format on the same workload
+    # (device-resident timing only)
+    other = None
+    if default_case:
+        import gc
+        gc.collect()
+        torch.cuda.empty_cache()
+        other_case = dataclasses.replace(case, fmt="mxfp4")
+        other = (other_case, gpu_arm(other_case, argparse.Namespace(**{**vars(args), "no_e2e": True}), rank, world, device))
     if rank != 0:
         if world > 1:
             import torch.distributed as dist
             dist.destroy_process_group()
         return
 
+    out = device_line(case, r, args, world, default_case)
+    if other is not None:
+        o = device_line(other[0], other[1], args, world, False)
+        out["other_format"] = {k: o[k] for k in ("value", "unit", "ms_per_step", "elems_per_s", "fwd_bwd_gbs",
+                                                 "pack_gbs", "phase_gbs", "phase_ms", "roofline", "clocks",
+                                                 "gpu_launches")}
+        out["other_format"]["config"] = {k: o["config"][k] for k in ("fmt", "sub_block", "coefficients",
+                                                                     "bytes_per_elem")}
+        out["gpu_launches"] += o["gpu_launches"]
+    if "e2e_ms" in r:
+        step_bytes = r["n_elem"] * sum(bytes_per_elem(case, r["esz"]).values())
+        out["e2e"] = {"value": round(aggregate_gbs(step_bytes, world, r["e2e_ms"]), 2),
+                      "unit": "GB/s", "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]}
+    if not args.no_cpu_baseline and world == 1:
+        out["cpu_baseline"] = cpu_baseline(case)
+    print(json.dumps(out))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def device_line(case, r, args, world, default_case):
+    """The JSON line of one device-resident run (gpu_arm's result)."""
     peak, peak_kind = load_peaks()
     K = args.steps
     ms_step = r["total_ms"] / K
@@ -1104,14 +1246,16 @@ def main():
     dom = max(ph, key=ph.get)
     fb_bytes = r["n_elem"] * (bpe["fwd"] + bpe["bwd"])
     traffic = None
-    if default_case and dom == "bwd" and kernel_sources_sha() == BWD_TRAFFIC["sources"]:
-        traffic = BWD_TRAFFIC["bytes_per_step"]
+    tr = TRAFFIC.get((case.workload, case.fmt, dom))
+    if default_case and tr is not None and kernel_sources_sha() == tr["sources"]:
+        traffic = round(tr["bytes_per_elem"] * r["n_elem"] / r["ntensors"])
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": case.workload, "tensors": r["ntensors"], "elements": r["n_elem"],
-                   "fmt": case.fmt, "io_dtype": case.io or ("bf16" if r["esz"] == 2 else "f32"),
+                   "fmt": case.fmt, "io_dtype": case.io or {4: "f32", 2: "bf16"}[r["esz"]],
+                   "arithmetic": "binary32 (coefficient gradients in double-binary32)",
                    "sub_block": case.sub,
                    "coefficients": ("shared by all rows" if case.shared else
                                     "per-block CRS + per-sub-block DGS"),
@@ -1142,7 +1286,8 @@ def main():
         "roofline": {"bound": "hbm", "kernel": f"fq_{dom}", "achieved": round(gbs[dom], 2),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(gbs[dom] / peak, 4), "traffic": traffic,
-                     "traffic_unit": "bytes per phase (one launch per tensor)"},
+                     "traffic_unit": "bytes per launch (DRAM read + write)",
+                     "algorithmic_bytes": round(r["n_elem"] * bpe[dom] / r["ntensors"])},
         "clocks": r["clocks"],
         "gpu_launches": K * r["launches_per_step"],
     }
@@ -1150,15 +1295,7 @@ def main():
         out["l2_resident"] = {"value": round(aggregate_gbs(step_bytes, world, r["l2_resident_ms"] / K), 2),
                               "unit": "GB/s", "ms_per_step": round(r["l2_resident_ms"] / K, 4),
                               "note": "steps back to back, inputs left in L2 by the previous step"}
-    if "e2e_ms" in r:
-        out["e2e"] = {"value": round(aggregate_gbs(step_bytes, world, r["e2e_ms"]), 2),
-                      "unit": "GB/s", "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]}
-    if not args.no_cpu_baseline and world == 1:
-        out["cpu_baseline"] = cpu_baseline(case)
-    print(json.dumps(out))
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+    return out
 
 
 if __name__ == "__main__":

@@ -127,8 +127,11 @@ int focus_nvfp4_alpha(const focus_desc_t* desc, const void* x, float* alpha_out,
  * path because that call can synchronise the device.  It calls no
  * allocating routine.
  * - The first call on a device looks up the array's device address (with
- *   that device current) and caches it; make that first call before any
- *   stream capture.
+ *   that device current) and caches it for the life of the process; make
+ *   that first call before any stream capture.  The cached address belongs
+ *   to the device's current context: after cudaDeviceReset (or anything else
+ *   that destroys the primary context) this entry point must not be called
+ *   again in the same process.
  * - Every call on a device shares the one array, so calls that overlap on
  *   the GPU (e.g. on two streams at once) race and may return wrong values;
  *   serialise them.  Nothing in the array needs clearing between calls.
@@ -283,7 +286,7 @@ size_t focus_mma_scale_bytes(const focus_desc_t* desc);
  * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
  * kernel whose wait on its pipeline gives up sets it to 1 (the output is
  * then incomplete) instead of waiting for ever.  Enqueued on `stream`; the
- * kernel runs as clusters of two CTAs. */
+ * kernel is persistent (one CTA per SM, each loading its own operand tiles). */
 int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
                    const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
                    const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,

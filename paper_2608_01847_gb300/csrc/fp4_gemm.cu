@@ -7,15 +7,13 @@
 // exported codes and hardware scales enter the product.
 //
 // Persistent, warp-specialised kernel, one CTA per SM, 128 x 256 tiles of D
-// (one M = 128, N = 256 MMA per K = 64 step), CTA pairs in clusters:
+// (one M = 128, N = 256 MMA per K = 64 step):
 //   warp 0     TMA producer: per K chunk of 256 elements (128 bytes of codes
-//              per row) the CTA's A tile and its half of the pair's B tile
-//              (2D TMA, 128-byte swizzle; the B half multicast to both CTAs
-//              of the cluster) and the chunk's scale tiles (1D bulk copies)
-//              into a ring of stages;
+//              per row) the CTA's A tile and its B tile (2D TMA, 128-byte
+//              swizzle) and the chunk's scale tiles (1D bulk copies) into a
+//              ring of stages;
 //   warp 1     MMA issuer: four K = 64 block-scaled MMAs per chunk into an
-//              accumulator in tensor memory, a commit to free the stage on
-//              both CTAs;
+//              accumulator in tensor memory, a commit to free the stage;
 //   warps 2-5  epilogue: accumulator -> registers (one lane quarter each),
 //              alpha scaling, then 32-row x 128-byte boxes of D staged in
 //              shared memory and written by TMA stores;
@@ -23,6 +21,9 @@
 //              (tcgen05.st, one lane quarter each), alternating between two
 //              sets of scale regions (an NVFP4 chunk fills a set, an MXFP4
 //              set holds two chunks), handed to the MMA warp by mbarrier.
+// Every CTA loads its own operands from this GPU's memory: consecutive CTAs
+// take consecutive 128-row tiles of A with the same tile of B, so B is read
+// from L2 by neighbours at about the same time.
 // The producer and MMA warps run their loops converged (all lanes wait,
 // lane 0 issues).  Writing the scales with tcgen05.st from their own warps
 // keeps them off the tensor pipe: copied there with tcgen05.cp they
@@ -74,13 +75,6 @@ constexpr int kOutBox = 32 * 128;
 constexpr int kOutBufs = 2;
 constexpr int kSmemBytes = kStages * kStageBytes + 4 * kOutBufs * kOutBox + 1024;   // + alignment slack
 constexpr int kThreads = 320;         // producer, MMA, four epilogue warps, four scale warps
-// CTAs of a cluster: consecutive 128-row tiles of A with the same 256-row
-// tile of B; each CTA loads 1 / kCluster of the B tile and multicasts it to
-// all of them, so B is read from L2 once per cluster.
-constexpr int kCluster = 2;
-constexpr int kSliceRows = kTileN / kCluster;
-constexpr int kSliceBytes = kTileBytesB / kCluster;
-constexpr uint16_t kClusterMask = static_cast<uint16_t>((1u << kCluster) - 1);
 // tensor memory: the 256-column accumulator, then two sets of scale regions
 // used by chunks in turn (set k % 2); inside a set, the four steps of a chunk
 // at + 16 j (A, 4 columns) and + 64 + 16 j (B, 8 columns: B rows 0-127 in
@@ -134,7 +128,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(&full[s], 1);
-            tc::mbar_init(&empty[s], kCluster);   // the MMA commits of every CTA of the cluster
+            tc::mbar_init(&empty[s], 1);   // the MMA warp's commit
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(&acc_full[b], 1);
@@ -149,7 +143,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::tc_fence_before();
     __syncthreads();
-    tc::cluster_sync();   // every barrier of the cluster initialised before any multicast
     tc::tc_fence_after();
     const uint32_t tb = tbase;
     // launched as a programmatic dependent: the set-up above overlaps the
@@ -157,13 +150,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    // tile groups: kCluster consecutive 128-row tiles of A (one per CTA of
-    // the cluster; the last group may have CTAs past M, which load no A,
-    // store nothing and keep the cluster's pipeline going) x one tile of B
-    const uint32_t rank = tc::cluster_rank();
-    const uint32_t tiles_mg = (p.tiles_m + kCluster - 1) / kCluster;
-    const uint32_t n_groups = tiles_mg * p.tiles_n;
-    const uint32_t group0 = tc::cluster_id(), groups_step = tc::cluster_count();
+    // tiles: u = tn * tiles_m + tm, so that consecutive CTAs take
+    // consecutive 128-row tiles of A with the same 256-row tile of B
+    const uint32_t n_groups = p.tiles_m * p.tiles_n;
+    const uint32_t group0 = blockIdx.x, groups_step = gridDim.x;
     const uint32_t n_chunks = (p.n_steps + 3) / 4;
     constexpr uint32_t steps_per_tile = FMT == 0 ? 2 : 1;   // K steps one scale tile covers
     // chunks per scale set: an MXFP4 chunk has two scale tiles, so a set
@@ -178,8 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t s = 0, ph = 0;
         bool ok = true;
         for (uint32_t u = group0; u < n_groups && ok; u += groups_step) {
-            const uint32_t tm = (u % tiles_mg) * kCluster + rank, tn = u / tiles_mg;
-            const bool valid = tm < p.tiles_m;
+            const uint32_t tm = u % p.tiles_m, tn = u / p.tiles_m;
             for (uint32_t c = 0; c < n_chunks; ++c) {
                 if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit))) {
                     ok = false;
@@ -191,18 +180,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t sf_tiles = (steps + steps_per_tile - 1) / steps_per_tile;
                     const uint32_t tile0 = (4 * c) / steps_per_tile;
                     const bool hi = 2 * tn + 1 < p.tile_rows_b;   // second 128-row half of B exists
-                    // this CTA's A tile and scales, the whole B tile (one slice from
-                    // each CTA of the cluster) and the B scales
-                    tc::mbar_arrive_expect_tx(&full[s], (valid ? kTileBytes + sf_tiles * 512 : 0) + kTileBytesB +
-                                                            (hi ? 2 : 1) * sf_tiles * 512);
-                    tc::tma_load_2d_mc(stage_b(s) + rank * kSliceBytes, &tma_b, static_cast<int32_t>(c * kChunk),
-                                       static_cast<int32_t>(tn * kTileN + rank * kSliceRows), &full[s], kClusterMask);
-                    if (valid) {
-                        tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
-                                        static_cast<int32_t>(tm * kTile), &full[s]);
-                        tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
-                                      sf_tiles * 512, &full[s]);
-                    }
+                    // the A and B tiles and their scales (rows past M or N are
+                    // filled with zeros by the tensor maps)
+                    tc::mbar_arrive_expect_tx(&full[s], kTileBytes + kTileBytesB + (hi ? 3 : 2) * sf_tiles * 512);
+                    tc::tma_load_2d(stage_b(s), &tma_b, static_cast<int32_t>(c * kChunk),
+                                    static_cast<int32_t>(tn * kTileN), &full[s]);
+                    tc::tma_load_2d(stage_a(s), &tma_a, static_cast<int32_t>(c * kChunk),
+                                    static_cast<int32_t>(tm * kTile), &full[s]);
+                    tc::bulk_load(stage_sfa(s), p.sfa + (static_cast<size_t>(tm) * p.tiles_k + tile0) * 512,
+                                  sf_tiles * 512, &full[s]);
                     tc::bulk_load(stage_sfb(s), p.sfb + (static_cast<size_t>(2 * tn) * p.tiles_k + tile0) * 512,
                                   sf_tiles * 512, &full[s]);
                     if (hi)
@@ -217,8 +203,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-        // every stage released by every CTA of the cluster: no commit of
-        // another CTA still to arrive on this CTA's barriers
+        // every stage released: no commit still to arrive on this CTA's
+        // barriers when it exits
         for (int i = 0; i < kStages && ok; ++i) {
             if (!__all_sync(0xffffffffu, tc::mbar_wait_hot(&empty[s], ph ^ 1, kWaitLimit))) {
                 if (lane == 0) give_up(p);
@@ -272,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         else
                             tc::mma_nvf4(d_tmem, ad, bd, tc::idesc_fp4(kTile, kTileN, false), sfa, sfb, accumulate);
                     }
-                    tc::mma_commit_mc(&empty[s], kClusterMask);
+                    tc::mma_commit(&empty[s]);
                 }
                 __syncwarp();
                 if (++s == kStages) {
@@ -294,8 +280,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // and scale set (k / kChunksPerSet) % 2.  Before a set is rewritten,
         // the MMAs of the chunks that last used it must be complete.  NVFP4
         // (one chunk per set): those of chunk k - 2, whose commit completed
-        // the empty barrier of that chunk's stage (on every CTA of the
-        // cluster).  MXFP4 (pairs of chunks): the last of them is chunk
+        // the empty barrier of that chunk's stage.  MXFP4 (pairs of
+        // chunks): the last of them is chunk
         // 2 p - 3 for pair p, and the producer loaded chunk 2 p into the stage
         // that chunk freed (three stages), so the full barrier of chunk 2 p
         // already implies it.
@@ -392,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++obuf;
         };
         for (uint32_t u = group0; u < n_groups; u += groups_step) {
-            const uint32_t tm = (u % tiles_mg) * kCluster + rank, tn = u / tiles_mg;
+            const uint32_t tm = u % p.tiles_m, tn = u / p.tiles_m;
             const bool got = __all_sync(0xffffffffu, tc::mbar_wait_hot(&acc_full[acc], acc_ph, kWaitLimit));
             if (!got) {
                 if (lane == 0) give_up(p);
@@ -500,7 +486,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp >= 2 && warp < 6 && lane == 0) tc::bulk_wait_all();   // output stores complete
     tc::tc_fence_before();
     __syncthreads();
-    tc::cluster_sync();
     tc::tc_fence_after();
     if (warp == 0) tc::tmem_dealloc(tb, kTmemCols);
 }
@@ -574,30 +559,26 @@ cudaError_t launch(const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorM
     });
     if (attr != cudaSuccess) return attr;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute at[2];
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = kCluster;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = kSmemBytes;
     cfg.stream = st;
     cfg.attrs = at;
-    cfg.numAttrs = 1;   // the occupancy query below takes the cluster shape only
-    // persistent: as many clusters as are resident at once (one CTA per SM)
+    cfg.numAttrs = 1;
+    // persistent: as many CTAs as are resident at once (one per SM)
     static int resident = 0;
     if (resident <= 0) {
-        cfg.gridDim = dim3(kCluster * static_cast<uint32_t>(device_sm_count() / kCluster));
         int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, fp4_gemm_kernel<FMT>, &cfg) != cudaSuccess || n <= 0)
-            n = device_sm_count() / kCluster;
-        resident = std::max(n, 1);
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fp4_gemm_kernel<FMT>, kThreads, kSmemBytes) !=
+                cudaSuccess ||
+            n <= 0)
+            n = 1;
+        resident = std::max(n * device_sm_count(), 1);
     }
-    const uint32_t groups = ((p.tiles_m + kCluster - 1) / kCluster) * p.tiles_n;
-    cfg.gridDim = dim3(kCluster * std::min<uint32_t>(groups, static_cast<uint32_t>(resident)));
-    cfg.numAttrs = 2;
+    const uint32_t tiles = p.tiles_m * p.tiles_n;
+    cfg.gridDim = dim3(std::min<uint32_t>(tiles, static_cast<uint32_t>(resident)));
     return cudaLaunchKernelEx(&cfg, fp4_gemm_kernel<FMT>, ma, mb, md, p);
 }
 
@@ -634,7 +615,7 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
         return FOCUS_ERR_MISALIGNED;
     CUtensorMap ma, mb, md;
     if (!make_map(&ma, CU_TENSOR_MAP_DATA_TYPE_UINT8, a_codes, M, K / 2, K / 2, 1, kTile) ||
-        !make_map(&mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, b_codes, N, K / 2, K / 2, 1, kSliceRows))
+        !make_map(&mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, b_codes, N, K / 2, K / 2, 1, kTileN))
         return FOCUS_ERR_CUDA;
     GemmParams p;
     p.sfa = a_scale_tiles;

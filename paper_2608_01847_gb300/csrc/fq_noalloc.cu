@@ -39,7 +39,8 @@ float* g_partials_addr[kMaxDevices] = {nullptr};
 std::mutex g_setup_mutex;
 
 // Device address of g_alpha_partials on the current device (looked up once
-// per device, with that device current).
+// per device, with that device current, and kept for the life of the
+// process: it is not valid across a reset of the device's context).
 int static_partials(float** out)
 {
     int dev = 0;
