@@ -1,30 +1,34 @@
 """Benchmark of the FOCUS FP4 fake-quantizer hot path on GB300.
 
-Default case: one step = one pass of the whole hot path over the Qwen3-4B
-decoder layer (7 bf16 projections, 100.9 M elements), NVFP4 (block 16, E4M3
-+ fp32 alpha), per-block CRS and per-sub-block (8) DGS coefficients:
+Default case: one step = one pass of the whole hot path over the W4A4
+calibration activations of the paper's setup (Sec. 4.1: 128 sequences x
+2048 tokens x hidden 4096 = 1.07 G bf16 elements, 2 GiB), NVFP4 (block 16,
+E4M3 + a per-call fp32 alpha), per-block CRS and per-sub-block (8) DGS
+coefficients:
   alpha (per tensor)  ->  fake-quant forward  ->  STE backward (input
   gradient + both coefficient gradients)  ->  export pack,
-inputs resident in HBM.  The step is captured once as a CUDA graph: each
-tensor's four phases chained on its own branch (programmatic dependent
-launches), the tensors' branches side by side; `--staged` joins all tensors
-between phases instead, `--group` runs each phase as one group launch.
-`value` is the algorithmic bytes of the step (per-element figures in
-bytes_per_elem) over the step time.  The JSON line also carries the phase
-split, the roofline of the dominant kernel, the end-to-end figure (pinned
-host buffers, copies inside the timed region), the CPU oracle baseline and
-the SM clocks sampled during the timed region.
+inputs resident in HBM.  The same workload under MXFP4 (block 32, E8M0) is
+timed after it and reported under "other_format".  The step is captured once
+as a CUDA graph: each tensor's phases chained on its own branch
+(programmatic dependent launches), the tensors' branches side by side;
+`--staged` joins all tensors between phases instead, `--group` runs each
+phase as one group launch.  `value` is the algorithmic bytes of the step
+(per-element figures in bytes_per_elem) over the step time.  The JSON line
+also carries the phase split, the roofline of the dominant kernel, the
+end-to-end figure (pinned host buffers, copies inside the timed region), the
+CPU oracle baseline and the SM clocks sampled (NVML, read-only) during the
+timed steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
                   [--workload NAME --fmt mxfp4|nvfp4 --shared --sfp --adam
                    --io f16 --sub B --staged --group --no-e2e --no-cpu-baseline]
   python bench.py --gemm [--fmt mxfp4] [--workload NAME]
 
-Other workloads (the Llama-3-8B block, the 70B layer set, the W4A4
-activations, sweep tensors) are measured the same way with --workload; the
-default line is the Qwen3-4B layer.  `--impl reference` times the CPU
-oracle on a bounded sample of the same workload.  `--gemm` times the W4A4
-FP4 GEMMs of a layer's projections on their exports.
+Other workloads (the Qwen3-4B layer, the Llama-3-8B block, the 70B layer
+set, sweep tensors) are measured the same way with --workload.
+`--impl reference` times the CPU oracle on a bounded sample of the same
+workload.  `--gemm` times the W4A4 FP4 GEMMs of a layer's projections on
+their exports (default: the Qwen3-4B layer x 8192 tokens).
 
 Under torchrun (N > 1) every rank runs the same workload on its own GPU
 (replicas; no data-path collective), the step time is the max over ranks and
@@ -803,7 +807,10 @@ def calibrate_oracle(case, target_s):
     oracle_step(case, probe)
     dt = max(time.perf_counter() - t0, 1e-6)
     from paper_2608_01847_gb300 import workloads as W
-    most = max(t.rows for t in W.WORKLOADS[case.workload].tensors)
+    tensors = W.WORKLOADS[case.workload].tensors
+    # at most 2^28 elements of the largest tensor (a bounded sample of the
+    # 2 GiB activations; every layer's weights fit whole)
+    most = min(max(t.rows for t in tensors), max(1, (1 << 28) // max(t.cols for t in tensors)))
     return max(1, min(int(8 * target_s / dt), most))
 
 
