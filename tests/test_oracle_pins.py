@@ -109,6 +109,40 @@ def test_hand_mxfp4_block_crs():
     assert expect == pytest.approx(-1.3248, abs=1e-6)
 
 
+def test_hand_gx_rounding_order():
+    """The STE input gradient rounds the scale ratio once (dy/dx = S^dq / S^q,
+    Sec. 3.2): gx = fl(g * fl(S^dq / S^q)).  Evaluating the chain rule term by
+    term instead, fl(fl(g * S^dq) / S^q), rounds differently for some g; this
+    block is one of them.  Worked by hand, binary32, integers x 2^-k exact:
+
+      S^dq = 0.25 (the block above, m = 1.5), c = 1.25, S^q = 0.3125 (exact)
+      rho  = fl(0.25 / 0.3125) = fl(0.8):  0.8 * 2^24 = 13421772.8
+             -> 13421773 * 2^-24                              (0x3F4CCCCD)
+      g    = 1.125 = 9 / 8
+      ratio order:   g * rho = 9 * 13421773 * 2^-27 = 120795957 * 2^-27
+             in [0.5, 1) the spacing is 2^-24: 120795957 / 8 = 15099494.625
+             -> 15099495 * 2^-24 = 0.90000004                  (0x3F666667)
+      chain order:   fl(g * S^dq) = 0.28125 (exact), 0.28125 / 0.3125 = 0.9:
+             0.9 * 2^24 = 15099494.4 -> 15099494 * 2^-24 = 0.9 (0x3F666666)
+    The oracle (and the kernels, which it checks bit for bit) take the ratio
+    order: the expected bits are the first ones."""
+    x = np.zeros((1, 32), np.float32)
+    x[0, :4] = [0.7, -0.26, 0.13, 1.5]
+    crs = np.array([[1.25]], np.float32)
+    g = np.zeros_like(x)
+    g[0, :4] = 1.125
+    gx = O.bwd(x, g, O.MXFP4, crs=crs)["gx"]
+    assert list(gx[0, :4].view(np.uint32)) == [0x3F666667] * 4
+    assert np.all(gx[0, 4:] == 0)
+    # the two orders really differ here (numpy binary32 arithmetic)
+    chain = np.float32(np.float32(np.float32(1.125) * np.float32(0.25)) / np.float32(0.3125))
+    assert chain.view(np.uint32) == 0x3F666666
+    # the same bits through a DGS coefficient (c_eff = c^k = 1.25), sub-block 8
+    dgs = np.array([[1.25, 1.0, 1.0, 1.0]], np.float32)
+    gx = O.bwd(x, g, O.MXFP4, dgs=dgs)["gx"]
+    assert list(gx[0, :4].view(np.uint32)) == [0x3F666667] * 4
+
+
 def test_hand_mxfp4_ties():
     # S^q = 0.25 (m = 1.5): 0.625 -> u = 2.5 (tie 2|3 -> 2, code 4); 1.25 -> 5
     # (tie 4|6 -> 4, code 6); 0.0625 -> 0.25 (tie 0|0.5 -> 0); -0.0625 -> -0 (0x8)

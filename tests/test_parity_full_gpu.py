@@ -87,14 +87,95 @@ def test_full_size_per_row(name, fmt):
         _check_tensor(w, idx, fmt)
 
 
-def test_full_size_sweep_4gb():
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_full_size_sweep_4gb(fmt):
+    """The sweep's largest point: one [262144, 8192] bf16 tensor, 2^31
+    elements (4 GiB), the largest size the descriptor allows."""
     w = W.sweep_workload(1 << 32)
-    _check_tensor(w, 0, O.NVFP4)
+    _check_tensor(w, 0, fmt)
+
+
+def test_full_size_coefficients_at_one():
+    """The Qwen3-4B layer (NVFP4) with no coefficient arrays, i.e. c = c^k = 1,
+    the method's starting point, which Sec. 3.3 states is the baseline: every
+    tensor at full size, sampled rows bit for bit against the oracle (itself
+    pinned to standard RTN on the CPU), and against an independent RTN
+    (numpy, torch's E4M3); the input gradient is g itself wherever the block
+    is live (S^dq / S^q = 1), with -0 written as +0; the coefficient
+    gradients at c = 1 within tolerance."""
+    from test_oracle_pins import rtn_reference
+    w = W.WORKLOADS["qwen3_4b_layer"]
+    for idx in range(len(w.tensors)):
+        x, g = W.device_tensor(w, idx, "cuda")
+        rows, cols = x.shape
+        a_dev = F.focus_nvfp4_alpha(x)
+        y, sb = F.focus_fq_fwd(x, O.NVFP4, None, None, a_dev, want_scales=True)
+        codes, sb2 = F.focus_pack(x, O.NVFP4, None, None, a_dev)
+        gx, gc, gd = F.focus_fq_bwd(x, g, O.NVFP4, None, None, a_dev, want_gcrs=True, want_gdgs=True)
+        torch.cuda.synchronize()
+        xh = host(x)
+        a = O.alpha(xh)
+        assert_bits_equal(host(a_dev), np.array([a], np.float32), "alpha")
+        rng = np.random.default_rng(300 + idx)
+        rs = np.unique(np.concatenate([[0, rows - 1], rng.choice(rows, 30, replace=False)]))
+        ri = torch.from_numpy(rs).cuda()
+        sel = lambda t: host(t.index_select(0, ri))
+        xs, gs = xh[rs], sel(g)
+        ref = O.fwd(xs, O.NVFP4, alpha=a, want_codes=True)
+        rb = O.bwd(xs, gs, O.NVFP4, alpha=a, want_abs=True)
+        name = f"c=1 {w.tensors[idx].name}"
+        assert_bits_equal(sel(y), ref["y"], f"{name} y")
+        assert_bits_equal(sel(sb), ref["scales"], f"{name} scale bytes")
+        assert_bits_equal(sel(sb2), ref["scales"], f"{name} scale bytes (pack)")
+        assert_bits_equal(sel(codes), ref["codes"], f"{name} codes")
+        assert_bits_equal(sel(gx), rb["gx"], f"{name} gx")
+        rtn = O.bf16_rne(rtn_reference(W.bf16_bits_to_f32(xs), O.NVFP4, alpha=a))
+        assert_bits_equal(sel(y), rtn, f"{name} y against RTN")
+        live = np.repeat(ref["scales"] != 0, 16, axis=1)
+        expect_gx = np.where(live & (gs != 0x8000), gs, np.uint16(0))
+        assert_bits_equal(sel(gx), expect_gx, f"{name} gx = g")
+        assert_grad_close(sel(gc), rb["gcrs"], rb["gcrs_abs"], FLOOR_ROW, f"{name} dL/dc at 1")
+        assert_grad_close(sel(gd), rb["gdgs"], rb["gdgs_abs"], FLOOR_ROW, f"{name} dL/dc^k at 1")
+        del x, g, y, sb, sb2, codes, gx, gc, gd
+        torch.cuda.empty_cache()
 
 
 # ---------------------------------------------------------------------------
 # shared-row coefficients over all rows of the activation workload
 # ---------------------------------------------------------------------------
+def _pooled_shared_oracle(x, g, fmt, a, ch, dh, sub, tmp_path):
+    """The oracle's shared-row gradient sums over every row of (x, g): rows
+    split across a spawn-started process pool, inputs through one
+    memory-mapped file, partial sums added in binary64.  Returns the sums,
+    their |term| sums, and the memory-mapped inputs (x, g as bf16 bits)."""
+    rows, cols = x.shape
+    path = os.path.join(tmp_path, "xg.npy")
+    arr = np.lib.format.open_memmap(path, mode="w+", dtype=np.uint16, shape=(2, rows, cols))
+    arr[0] = host(x)
+    arr[1] = host(g)
+    arr.flush()
+    del arr
+    nproc = max(1, min(32, os.cpu_count() or 1))
+    bounds = np.linspace(0, rows, nproc + 1).astype(int)
+    jobs = [(path, int(bounds[i]), int(bounds[i + 1]), fmt, a, ch, dh, sub)
+            for i in range(nproc) if bounds[i + 1] > bounds[i]]
+    with cf.ProcessPoolExecutor(max_workers=nproc, mp_context=mp.get_context("spawn")) as ex:
+        parts = list(ex.map(oracle_pool.shared_rows_chunk, jobs))
+    sums = tuple(sum(p[i] for p in parts) for i in range(4))   # dL/dc, dL/dc^k, |terms| of each
+    return sums, np.load(path, mmap_mode="r")
+
+
+def _check_shared_gx(gx, xg, fmt, a, ch, dh, sub, what):
+    """Input gradient of the shared-row backward on sampled rows against the
+    per-row oracle (same formula, one coefficient row for all rows)."""
+    rows = xg.shape[1]
+    rng = np.random.default_rng(5)
+    rs = np.unique(np.concatenate([[0, rows - 1], rng.choice(rows, 30, replace=False)]))
+    rb = O.bwd(np.ascontiguousarray(xg[0][rs]), np.ascontiguousarray(xg[1][rs]), fmt, crs=ch, dgs=dh,
+               alpha=a, sub=sub, shared=True)
+    assert_bits_equal(host(gx.index_select(0, torch.from_numpy(rs).cuda())), rb["gx"], what)
+
+
 @pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
 def test_full_size_shared_rows(fmt, tmp_path):
     w = W.WORKLOADS["act_262144x4096"]
@@ -105,40 +186,54 @@ def test_full_size_shared_rows(fmt, tmp_path):
     a_dev = F.focus_nvfp4_alpha(x) if fmt == O.NVFP4 else None
     gx, gc, gd = F.focus_fq_bwd(x, g, fmt, crs, dgs, a_dev, sub_block=sub, shared=True)
     torch.cuda.synchronize()
-    rows, cols = x.shape
     a = float(host(a_dev)[0]) if fmt == O.NVFP4 else 0.0
-    # inputs for the pool through one memory-mapped file
-    path = os.path.join(tmp_path, "xg.npy")
-    arr = np.lib.format.open_memmap(path, mode="w+", dtype=np.uint16, shape=(2, rows, cols))
-    arr[0] = host(x)
-    arr[1] = host(g)
-    arr.flush()
-    del arr
     ch, dh = host(crs), host(dgs)
+    (ref_c, ref_d, abs_c, abs_d), xg = _pooled_shared_oracle(x, g, fmt, a, ch, dh, sub, tmp_path)
     if fmt == O.NVFP4:
-        assert a == O.alpha(np.load(path, mmap_mode="r")[0])
-    nproc = max(1, min(32, os.cpu_count() or 1))
-    bounds = np.linspace(0, rows, nproc + 1).astype(int)
-    jobs = [(path, int(bounds[i]), int(bounds[i + 1]), fmt, a, ch, dh, sub)
-            for i in range(nproc) if bounds[i + 1] > bounds[i]]
-    with cf.ProcessPoolExecutor(max_workers=nproc, mp_context=mp.get_context("spawn")) as ex:
-        parts = list(ex.map(oracle_pool.shared_rows_chunk, jobs))
-    ref_c = sum(p[0] for p in parts)
-    ref_d = sum(p[1] for p in parts)
-    abs_c = sum(p[2] for p in parts)
-    abs_d = sum(p[3] for p in parts)
+        assert a == O.alpha(xg[0])
     # the partials are added in binary64 from unrounded values: the tolerance
     # is the shared-row one (1e-5 relative, 2^-30 cancellation floor)
     assert_grad_close(host(gc)[0], ref_c[0], abs_c[0], FLOOR_SHARED, "shared dL/dc")
     assert_grad_close(host(gd)[0], ref_d[0], abs_d[0], FLOOR_SHARED, "shared dL/dc^k")
-    # input gradient: sampled rows against the per-row oracle (same formula)
-    rng = np.random.default_rng(5)
-    rs = np.unique(np.concatenate([[0, rows - 1], rng.choice(rows, 30, replace=False)]))
-    xs = np.load(path, mmap_mode="r")[0][rs]
-    gs = np.load(path, mmap_mode="r")[1][rs]
-    rb = O.bwd(np.ascontiguousarray(xs), np.ascontiguousarray(gs), fmt, crs=ch, dgs=dh, alpha=a,
-               sub=sub, shared=True)
-    assert_bits_equal(host(gx.index_select(0, torch.from_numpy(rs).cuda())), rb["gx"], "shared gx")
+    _check_shared_gx(gx, xg, fmt, a, ch, dh, sub, "shared gx")
+
+
+@pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
+def test_full_size_shared_rows_adamw(fmt, tmp_path):
+    """The W4A4 activation calibration step with channel-block coefficients
+    shared by all 262,144 rows, fused with the AdamW step (Sec. 4.1): the
+    device's new c_i, c_i^k and moments must lie in the interval that the
+    gradient tolerance and binary32 rounding allow around the oracle's exact
+    step from its gradient summed over every row."""
+    from gpu_helpers import assert_adamw_close
+    hp = dict(lr_coef=5e-2 if fmt == O.MXFP4 else 1e-3, lr_scale=0.0, beta1=0.9, beta2=0.999, eps=1e-8,
+              weight_decay=0.01)
+    w = W.WORKLOADS["act_262144x4096"]
+    block = 32 if fmt == O.MXFP4 else 16
+    sub = 8
+    x, g = W.device_tensor(w, 0, "cuda")
+    crs, dgs = W.device_coefs(w, 0, block, sub, "cuda", shared=True)
+    a_dev = F.focus_nvfp4_alpha(x) if fmt == O.NVFP4 else None
+    ch, dh = host(crs), host(dgs)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(31 + fmt)
+    params = {"crs": crs, "dgs": dgs}
+    moments = {k: ((torch.rand(v.shape, generator=gen, device="cuda") - 0.5) * 0.1,
+                   torch.rand(v.shape, generator=gen, device="cuda") * 0.01) for k, v in params.items()}
+    m0 = {k: (host(m), host(v)) for k, (m, v) in moments.items()}
+    step = torch.tensor([3], dtype=torch.int64, device="cuda")
+    gx = F.focus_fq_bwd_adamw(x, g, fmt, step, hp, crs=crs, dgs=dgs, moments=moments, alpha=a_dev,
+                              sub_block=sub, shared=True)
+    torch.cuda.synchronize()
+    a = float(host(a_dev)[0]) if fmt == O.NVFP4 else 0.0
+    (ref_c, ref_d, abs_c, abs_d), xg = _pooled_shared_oracle(x, g, fmt, a, ch, dh, sub, tmp_path)
+    _check_shared_gx(gx, xg, fmt, a, ch, dh, sub, "shared gx (AdamW)")
+    for k, p0, grad, gabs in (("crs", ch, ref_c, abs_c), ("dgs", dh, ref_d, abs_d)):
+        pn, mn, vn = O.adamw(p0, grad, m0[k][0], m0[k][1], hp["lr_coef"], hp["beta1"], hp["beta2"],
+                             hp["eps"], hp["weight_decay"], 3)
+        ref = {"grad": grad, "grad_abs": gabs, "p": pn}
+        assert_adamw_close((host(params[k]), host(moments[k][0]), host(moments[k][1])), p0, m0[k][0],
+                           m0[k][1], ref, FLOOR_SHARED, hp["lr_coef"], hp, 3, f"shared AdamW {k}")
 
 
 # ---------------------------------------------------------------------------
@@ -155,7 +250,12 @@ def _sfp_init(x, fmt, a_dev, seed):
     return (m / den * (torch.rand(m.shape, generator=gen, device=x.device) * 0.2 + 0.9)).contiguous()
 
 
-@pytest.mark.parametrize("name,fmt,idx", [("qwen3_4b_layer", O.NVFP4, 4), ("llama_70b_layer", O.MXFP4, 6)])
+# every tensor of the Qwen3-4B layer (NVFP4) and of the 70B layer set (both formats)
+EVERY_TENSOR = [(n, f, i) for n, fs in (("qwen3_4b_layer", (O.NVFP4,)), ("llama_70b_layer", (O.MXFP4, O.NVFP4)))
+                for f in fs for i in range(len(W.WORKLOADS[n].tensors))]
+
+
+@pytest.mark.parametrize("name,fmt,idx", EVERY_TENSOR)
 def test_full_size_learnable_scale(name, fmt, idx):
     w = W.WORKLOADS[name]
     block = 32 if fmt == O.MXFP4 else 16
@@ -185,7 +285,7 @@ def test_full_size_learnable_scale(name, fmt, idx):
     assert_grad_close(sel(gs), rb["gsfp"], rb["gsfp_abs"], FLOOR_ROW, f"{name} dL/dS^fp")
 
 
-@pytest.mark.parametrize("name,fmt,idx", [("qwen3_4b_layer", O.NVFP4, 4), ("llama_70b_layer", O.MXFP4, 6)])
+@pytest.mark.parametrize("name,fmt,idx", EVERY_TENSOR)
 def test_full_size_fused_adamw(name, fmt, idx):
     from gpu_helpers import assert_adamw_close
     hp = dict(lr_coef=5e-2 if fmt == O.MXFP4 else 1e-3, lr_scale=2e-2 * 2.0 ** -7 if fmt == O.MXFP4 else 5e-3,

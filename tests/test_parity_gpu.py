@@ -237,6 +237,31 @@ def test_degenerate_blocks():
     run_case(xn, g, O.NVFP4, crs=rng.uniform(0.9, 1.1, (48, 16)).astype(np.float32))
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_gradient_overflow_rule(dtype):
+    """Sub-blocks of alternating +a, -a with g = 1 cancel exactly (T = 0).
+    The kernels sum even and odd elements in two interleaved binary32 chains:
+    at a = 2^125 each chain peaks at 4a = 2^127, nothing overflows, and the
+    gradient is exactly 0; at a = 2^126 a chain reaches 2^128 and overflows,
+    and the pair turns into NaN -- allowed only because the sum of |terms|
+    (2^129) is beyond the binary32 range (the comparison rule of
+    assert_grad_close)."""
+    x = np.ones((2, 64), np.float32)
+    x[0, :32] = np.float32(2.0 ** 125) * np.tile(np.float32([1, -1]), 16)
+    x[1, :32] = np.float32(2.0 ** 126) * np.tile(np.float32([1, -1]), 16)
+    g = np.ones_like(x)
+    if dtype == "bf16":
+        x, g = W.to_bf16_bits(x), W.to_bf16_bits(g)
+    crs = np.ones((2, 2), np.float32)
+    dgs = np.ones((2, 8), np.float32)
+    out = run_case(x, g, O.MXFP4, crs=crs, dgs=dgs)
+    gc, gd = host(out["gcrs"]), host(out["gdgs"])
+    assert gc[0, 0] == 0 and np.all(gd[0, :4] == 0)
+    assert np.isnan(gc[1, 0]) and np.all(np.isnan(gd[1, :4]))
+    # the second block of each row (ones) is unaffected
+    assert np.isfinite(gc[:, 1]).all() and np.isfinite(gd[:, 4:]).all()
+
+
 def test_nvfp4_all_zero_tensor():
     x = np.zeros((8, 64), np.float32)
     g = np.ones_like(x)
