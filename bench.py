@@ -532,49 +532,142 @@ class BranchGraph:
         self.graph.replay()
 
 
-class PipelineGraph:
-    """End-to-end step as a graph of three chained streams: the H2D copy of
-    each tensor's inputs, then its phases, then the D2H copy of its outputs
-    (one copy per tensor and direction: the inputs, and the outputs, share
-    an allocation, mirrored by pinned host buffers of the same layout), so
-    that tensor k's D2H overlaps tensor k+1's H2D on the full-duplex link."""
+# arrays of a Tensor that hold one row (or one row's coefficients) per row
+ROW_ARRAYS = ("x", "g", "g_alt", "y", "gx", "crs", "dgs", "sfp", "gcrs", "gdgs", "gsfp", "codes", "scales")
+# outputs that only the forward-side phases (forward, pack) write
+FRONT_OUTPUTS = ("y", "codes", "scales")
 
-    def __init__(self, ts, phases, device, parity=0, before=None):
+
+def tensor_piece(t, r0, r1):
+    """Rows [r0, r1) of Tensor t: a shallow copy whose row arrays (and
+    moments) are views of t's rows -- the C ABI computes a row range of a
+    tensor exactly as the whole call would -- sharing t's alpha and scratch."""
+    import copy
+    p = copy.copy(t)
+    for n in ROW_ARRAYS:
+        a = getattr(t, n, None)
+        if a is not None:
+            setattr(p, n, a[r0:r1])
+    if getattr(t, "moments", None) is not None:
+        p.moments = {k: (m[r0:r1], v[r0:r1]) for k, (m, v) in t.moments.items()}
+    p.n = (r1 - r0) * t.x.shape[1]
+    return p
+
+
+class PipelineGraph:
+    """End-to-end step as a graph of three chained streams: the H2D copies
+    of each tensor's inputs, then its phases, then the D2H copies of its
+    outputs (the inputs, and the outputs, of a tensor share an allocation
+    mirrored by pinned host buffers of the same layout), so that one
+    tensor's D2H overlaps the next one's H2D on the full-duplex link.
+
+    A tensor of more than 2 * piece_elems elements (per-row coefficients) is
+    moved and computed in row pieces of about piece_elems elements: the
+    pieces' forward-side inputs (x and coefficients) first, then their
+    upstream gradients; the forward and pack of a piece start once its rows
+    have arrived (NVFP4: once all of x has, for the per-tensor alpha), its
+    values, codes and scale bytes leave while the gradients still arrive,
+    and its backward outputs follow its backward.  With the fused optimizer
+    the phases keep their order (the pack reads the updated coefficients)."""
+
+    def __init__(self, ts, phases, device, parity=0, before=None, piece_elems=1 << 27):
         import torch
         # the smallest tensor first (short pipeline fill: its H2D runs alone)
         # and the second smallest last (short drain: its D2H runs alone)
         order = sorted(range(len(ts)), key=lambda i: ts[i].n)
         order = order[:1] + order[2:] + order[1:2] if len(order) > 2 else order
         ts = [ts[i] for i in order]
-        spans_in = [arena_spans(t.in_buf, t.inputs(parity)) for t in ts]
-        spans_out = [arena_spans(t.out_buf, t.outputs()) for t in ts]
-        self.h2d = sum(e - s for sp in spans_in for s, e in sp)
-        self.d2h = sum(e - s for sp in spans_out for s, e in sp)
+        self.h2d = self.d2h = 0
         self.graph = torch.cuda.CUDAGraph()
         s_in, s_cmp, s_out = (torch.cuda.Stream(device) for _ in range(3))
         cap = torch.cuda.Stream(device)
         cap.wait_stream(torch.cuda.current_stream(device))
+
+        def h2d(t, arrays):
+            for s, e in arena_spans(t.in_buf, arrays):
+                t.in_buf[s:e].copy_(t.host_in[s:e], non_blocking=True)
+                self.h2d += e - s
+
+        def d2h(t, arrays):
+            for s, e in arena_spans(t.out_buf, arrays):
+                t.host_out[s:e].copy_(t.out_buf[s:e], non_blocking=True)
+                self.d2h += e - s
+
         with torch.cuda.graph(self.graph, stream=cap):
             main = torch.cuda.current_stream(device)
             if before is not None:
                 before()
             for st in (s_in, s_cmp, s_out):
                 st.wait_stream(main)
-            for t, sin, sout in zip(ts, spans_in, spans_out):
-                with torch.cuda.stream(s_in):
-                    for s, e in sin:
-                        t.in_buf[s:e].copy_(t.host_in[s:e], non_blocking=True)
-                s_cmp.wait_stream(s_in)
-                with torch.cuda.stream(s_cmp):
-                    for ph in phases:
-                        t.run(ph, parity)
-                s_out.wait_stream(s_cmp)
-                with torch.cuda.stream(s_out):
-                    for s, e in sout:
-                        t.host_out[s:e].copy_(t.out_buf[s:e], non_blocking=True)
+            for t in ts:
+                rows = t.x.shape[0]
+                n_p = 1 if t.case.shared else min(rows, t.n // piece_elems)
+                if n_p < 2:
+                    with torch.cuda.stream(s_in):
+                        h2d(t, t.inputs(parity))
+                    s_cmp.wait_stream(s_in)
+                    with torch.cuda.stream(s_cmp):
+                        for ph in phases:
+                            t.run(ph, parity)
+                    s_out.wait_stream(s_cmp)
+                    with torch.cuda.stream(s_out):
+                        d2h(t, t.outputs())
+                    continue
+                self._pieces(t, n_p, phases, parity, s_in, s_cmp, s_out, h2d, d2h)
             for st in (s_in, s_cmp, s_out):
                 main.wait_stream(st)
         torch.cuda.current_stream(device).wait_stream(cap)
+
+    @staticmethod
+    def _pieces(t, n_p, phases, parity, s_in, s_cmp, s_out, h2d, d2h):
+        import torch
+        rows = t.x.shape[0]
+        bounds = [rows * k // n_p for k in range(n_p + 1)]
+        pcs = [tensor_piece(t, bounds[k], bounds[k + 1]) for k in range(n_p)]
+        ids = lambda arrs: {id(a) for a in arrs}
+        grad_in = ids((t.g_alt if parity else t.g,) if t.case.adam else (t.g,))
+        work = [ph for ph in phases if ph != "alpha"]
+        if t.case.adam:
+            front, back = work[:work.index("bwd")], work[work.index("bwd"):]
+        else:
+            front, back = [ph for ph in work if ph != "bwd"], [ph for ph in work if ph == "bwd"]
+        front_out = {n for n in FRONT_OUTPUTS if not t.case.adam or n == "y"}
+        e_x, e_g, e_f, e_b = ([torch.cuda.Event() for _ in pcs] for _ in range(4))
+
+        in_names = [n for n in ROW_ARRAYS if getattr(t, n, None) is not None and
+                    id(getattr(t, n)) in ids(t.inputs(parity))]
+        out_names = [n for n in ROW_ARRAYS if getattr(t, n, None) is not None and
+                     id(getattr(t, n)) in ids(t.outputs())]
+        fwd_in = [n for n in in_names if id(getattr(t, n)) not in grad_in]
+        g_in = [n for n in in_names if id(getattr(t, n)) in grad_in]
+        with torch.cuda.stream(s_in):
+            for p, e in zip(pcs, e_x):
+                h2d(t, [getattr(p, n) for n in fwd_in])
+                e.record()
+            for p, e in zip(pcs, e_g):
+                h2d(t, [getattr(p, n) for n in g_in])
+                e.record()
+        with torch.cuda.stream(s_cmp):
+            if "alpha" in phases:
+                s_cmp.wait_event(e_x[-1])
+                t.run("alpha", parity)
+            for p, ex, ef in zip(pcs, e_x, e_f):
+                s_cmp.wait_event(ex)
+                for ph in front:
+                    p.run(ph, parity)
+                ef.record()
+            for p, eg, eb in zip(pcs, e_g, e_b):
+                s_cmp.wait_event(eg)
+                for ph in back:
+                    p.run(ph, parity)
+                eb.record()
+        with torch.cuda.stream(s_out):
+            for p, ef in zip(pcs, e_f):
+                s_out.wait_event(ef)
+                d2h(t, [getattr(p, n) for n in out_names if n in front_out])
+            for p, eb in zip(pcs, e_b):
+                s_out.wait_event(eb)
+                d2h(t, [getattr(p, n) for n in out_names if n not in front_out])
 
     def replay(self):
         self.graph.replay()

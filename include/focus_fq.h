@@ -26,8 +26,12 @@
  *   default stream) and completes asynchronously.
  * - x, y, g and gx are row-major [rows, ld] arrays of desc->dtype; only the
  *   first `cols` elements of each row are read or written.  Every row must
- *   start on a 32-byte boundary: the arrays 32-byte aligned (16 bytes suffice
- *   for the alpha pass) and ld * sizeof(element) a multiple of 32.
+ *   start on a 16-byte boundary: the arrays 16-byte aligned and
+ *   ld * sizeof(element) a multiple of 16 (FOCUS_ERR_MISALIGNED otherwise).
+ *   When every row of every array of a call starts on a 32-byte boundary
+ *   (arrays 32-byte aligned, ld * sizeof(element) a multiple of 32) the
+ *   kernels move each 32-byte piece of a row with one 256-bit access, else
+ *   with two 128-bit accesses; the results are the same.
  * - Coefficient arrays are dense fp32: crs / gcrs are [rows, cols/block] and
  *   dgs / gdgs are [rows, cols/sub_block]; with coef_shared_rows = 1 both are
  *   a single row ([cols/block], [cols/sub_block]) shared by all rows.  They

@@ -17,6 +17,14 @@ cudaError_t launch_bwd_nv(int dt, int sub, const KParams& p, cudaStream_t st);
 cudaError_t launch_bwd_shared_mx(int dt, int sub, const KParams& p, uint32_t ny, cudaStream_t st);
 cudaError_t launch_bwd_shared_nv(int dt, int sub, const KParams& p, uint32_t ny, cudaStream_t st);
 
+int shared_bwd_occupancy_mx(int dt, int sub);
+int shared_bwd_occupancy_nv(int dt, int sub);
+
+int shared_bwd_occupancy(int fmt, int dt, int sub)
+{
+    return fmt == 0 ? shared_bwd_occupancy_mx(dt, sub) : shared_bwd_occupancy_nv(dt, sub);
+}
+
 cudaError_t launch_bwd(int fmt, int dt, int sub, const KParams& p, cudaStream_t st)
 {
     return fmt == 0 ? launch_bwd_mx(dt, sub, p, st) : launch_bwd_nv(dt, sub, p, st);
@@ -43,8 +51,9 @@ int check_desc(const focus_desc_t* d, bool method)
     if (d->rows < 0 || d->cols < 0 || d->ld < d->cols || d->ld < 0) return FOCUS_ERR_INVALID_ARG;
     if (d->dtype != FOCUS_F32 && d->dtype != FOCUS_BF16 && d->dtype != FOCUS_F16) return FOCUS_ERR_INVALID_ARG;
     if (d->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
-    // rows start on 32-byte boundaries (256-bit accesses)
-    if ((d->ld * (d->dtype == FOCUS_F32 ? 4 : 2)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
+    // rows start on 16-byte boundaries (128-bit accesses; 256-bit ones when
+    // every row of every array starts on a 32-byte boundary)
+    if ((d->ld * (d->dtype == FOCUS_F32 ? 4 : 2)) % 16 != 0) return FOCUS_ERR_MISALIGNED;
     if (d->rows > 0 && d->cols > 0 && d->rows > kMaxChunks / (d->cols / 8)) return FOCUS_ERR_UNSUPPORTED;
     if (!method) return FOCUS_OK;
     if (d->fmt != FOCUS_MXFP4 && d->fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;
@@ -83,6 +92,20 @@ KParams make_params(const focus_desc_t* d)
 
 int map_cuda(cudaError_t e) { return e == cudaSuccess ? FOCUS_OK : FOCUS_ERR_CUDA; }
 
+// The element arrays of a call (x, y, g, gx; NULL ones ignored) must start
+// on 16-byte boundaries; the kernels take 256-bit accesses when every row of
+// every one of them starts on a 32-byte boundary, else two 128-bit ones.
+bool rows_misaligned(const void* a, const void* b, const void* c)
+{
+    return misaligned(a, 16) || misaligned(b, 16) || misaligned(c, 16);
+}
+
+int rows_half(const focus_desc_t* d, const void* a, const void* b, const void* c)
+{
+    const bool pitch32 = (d->ld * (d->dtype == FOCUS_F32 ? 4 : 2)) % 32 == 0;
+    return (!pitch32 || misaligned(a, 32) || misaligned(b, 32) || misaligned(c, 32)) ? 1 : 0;
+}
+
 // Sub-block size the kernels run with: without DGS coefficients (and without
 // their gradient) every sub-block of a block shares S^q, so one sub-block per
 // block gives identical results.
@@ -99,6 +122,18 @@ int check_coef_ptrs(const float* a, const float* b, const float* c, const float*
 }
 
 size_t bwd_ws_bytes(const focus_desc_t* d);
+
+// Row groups of the shared-row backward for a descriptor: a function of the
+// descriptor and the device only (the occupancy of the kernel for the
+// descriptor's sub-block size), so the workspace query and the launch agree;
+// a call without DGS runs the block-sized sub-block kernel with the same row
+// groups, whose partials then fit in less of the workspace.
+uint32_t shared_groups(const focus_desc_t* d)
+{
+    const uint32_t bpr = static_cast<uint32_t>(d->cols / d->block);
+    return shared_row_groups(static_cast<uint32_t>(d->rows), bpr,
+                             shared_bwd_occupancy(d->fmt, d->dtype, d->sub_block));
+}
 
 // Bytes of the scale tiles of the MMA layout: 128-row x 4-column tiles of
 // the [rows, cols/block] scale matrix, 512 bytes each.
@@ -198,11 +233,11 @@ int run_bwd(const focus_desc_t* desc, const void* x, const float* crs, const flo
     if (opt && (rc = check_opt(*opt))) return rc;
     const bool learn = opt && (opt->crs || opt->dgs || opt->sfp);
     const bool want_T = gcrs != nullptr || gdgs != nullptr || (learn && (crs || dgs));
-    if (misaligned(x, 32) || misaligned(g, 32) || misaligned(gx, 32) || misaligned(alpha, 4) ||
-        misaligned(sfp, 4) || misaligned(gsfp, 4))
+    if (rows_misaligned(x, g, gx) || misaligned(alpha, 4) || misaligned(sfp, 4) || misaligned(gsfp, 4))
         return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, gcrs, gdgs))) return rc;
     KParams p = make_params(desc);
+    p.half = rows_half(desc, x, g, gx);
     p.x = x;
     p.g = g;
     p.gx = gx;
@@ -238,7 +273,7 @@ int run_bwd(const focus_desc_t* desc, const void* x, const float* crs, const flo
         if (misaligned(ws, 16)) return FOCUS_ERR_MISALIGNED;
         p.ws = static_cast<float*>(ws);
         p.nsub = static_cast<uint32_t>(desc->cols / sub);
-        const uint32_t ny = shared_row_groups(p.rows, p.bpr);
+        const uint32_t ny = shared_groups(desc);
         return map_cuda(launch_bwd_shared(desc->fmt, desc->dtype, sub, p, ny, st));
     }
     return map_cuda(launch_bwd(desc->fmt, desc->dtype, sub, p, st));
@@ -247,8 +282,7 @@ int run_bwd(const focus_desc_t* desc, const void* x, const float* crs, const flo
 size_t bwd_ws_bytes(const focus_desc_t* d)
 {
     if (!d->coef_shared_rows || d->rows == 0 || d->cols == 0) return 0;
-    const uint32_t bpr = static_cast<uint32_t>(d->cols / d->block);
-    const uint32_t ny = shared_row_groups(static_cast<uint32_t>(d->rows), bpr);
+    const uint32_t ny = shared_groups(d);
     return static_cast<size_t>(ny) * static_cast<size_t>(d->cols / d->sub_block) * 2 * sizeof(float);
 }
 
@@ -311,10 +345,11 @@ FOCUS_API int focus_fq_fwd(const focus_desc_t* desc, const void* x, const float*
     if (sfp && desc->coef_shared_rows) return FOCUS_ERR_INVALID_ARG;
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !y || (desc->fmt == FOCUS_NVFP4 && !alpha)) return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 32) || misaligned(y, 32) || misaligned(alpha, 4) || misaligned(sfp, 4))
+    if (rows_misaligned(x, y, nullptr) || misaligned(alpha, 4) || misaligned(sfp, 4))
         return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
+    p.half = rows_half(desc, x, y, nullptr);
     p.x = x;
     p.y = y;
     p.crs = crs;
@@ -339,11 +374,13 @@ int run_pack(const focus_desc_t* desc, const void* x, const float* crs, const fl
     if (desc->rows == 0 || desc->cols == 0) return FOCUS_OK;
     if (!x || !codes || !scale_bytes || (desc->fmt == FOCUS_NVFP4 && !alpha))
         return FOCUS_ERR_INVALID_ARG;
-    if (misaligned(x, 32) || misaligned(codes, 16) || misaligned(alpha, 4) || misaligned(sfp, 4))
+    if (rows_misaligned(x, nullptr, nullptr) || misaligned(codes, 16) || misaligned(alpha, 4) ||
+        misaligned(sfp, 4))
         return FOCUS_ERR_MISALIGNED;
     if (mma_layout && misaligned(scale_bytes, 16)) return FOCUS_ERR_MISALIGNED;
     if ((rc = check_coef_ptrs(crs, dgs, nullptr, nullptr))) return rc;
     KParams p = make_params(desc);
+    p.half = rows_half(desc, x, nullptr, nullptr);
     p.x = x;
     p.crs = crs;
     p.dgs = dgs;
@@ -454,20 +491,22 @@ int build_group(const focus_tensor_t* t, int n, GroupMode mode, KGroup& g, int& 
             break;
         case kGroupFwd:
             if (!a.y) return FOCUS_ERR_INVALID_ARG;
-            if (misaligned(a.x, 32) || misaligned(a.y, 32)) return FOCUS_ERR_MISALIGNED;
+            if (rows_misaligned(a.x, a.y, nullptr)) return FOCUS_ERR_MISALIGNED;
             break;
         case kGroupPack:
             if (!a.codes || !a.scale_bytes) return FOCUS_ERR_INVALID_ARG;
-            if (misaligned(a.x, 32) || misaligned(a.codes, 16)) return FOCUS_ERR_MISALIGNED;
+            if (rows_misaligned(a.x, nullptr, nullptr) || misaligned(a.codes, 16)) return FOCUS_ERR_MISALIGNED;
             break;
         case kGroupBwd:
             if (!a.g) return FOCUS_ERR_INVALID_ARG;
-            if (misaligned(a.x, 32) || misaligned(a.g, 32) || misaligned(a.gx, 32)) return FOCUS_ERR_MISALIGNED;
+            if (rows_misaligned(a.x, a.g, a.gx)) return FOCUS_ERR_MISALIGNED;
             if (!a.gx && !a.gcrs && !a.gdgs && !a.gsfp) continue;   // nothing asked of this tensor
             break;
         }
         KParams& p = g.p[g.n];
         p = make_params(&d);
+        p.half = mode == kGroupBwd ? rows_half(&d, a.x, a.g, a.gx)
+                                   : rows_half(&d, a.x, mode == kGroupFwd ? a.y : nullptr, nullptr);
         p.x = a.x;
         if (mode != kGroupAlpha) {
             p.crs = a.crs;

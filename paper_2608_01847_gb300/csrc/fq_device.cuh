@@ -405,6 +405,46 @@ __device__ __forceinline__ void st_v8(void* p, const uint32_t (&w)[8])
                  : "memory");
 }
 
+// The same 32 bytes as two 128-bit accesses, for rows that start on a
+// 16-byte but not on a 32-byte boundary.  Each of the two warp-wide loads
+// touches half of every lane's sector, so the loads allocate in L1: the
+// second finds the sector the first brought in.
+__device__ __forceinline__ void ld_v4x2(uint32_t (&w)[8], const void* p)
+{
+    asm("ld.global.nc.v4.b32 {%0, %1, %2, %3}, [%8];\n\t"
+        "ld.global.nc.v4.b32 {%4, %5, %6, %7}, [%8+16];"
+        : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]),
+          "=r"(w[7])
+        : "l"(p));
+}
+
+__device__ __forceinline__ void st_v4x2(void* p, const uint32_t (&w)[8])
+{
+    asm volatile("st.global.cs.v4.b32 [%0], {%1, %2, %3, %4};\n\t"
+                 "st.global.cs.v4.b32 [%0+16], {%5, %6, %7, %8};"
+                 :
+                 : "l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]),
+                   "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
+
+// 32 bytes at p: one 256-bit access, or two 128-bit ones when HALF (the
+// rows of the call start on 16-byte but not 32-byte boundaries; the host
+// picks the kernel instantiation).
+template <bool HALF>
+__device__ __forceinline__ void ld_32b(uint32_t (&w)[8], const void* p)
+{
+    if constexpr (HALF) ld_v4x2(w, p);
+    else ld_v8(w, p);
+}
+
+template <bool HALF>
+__device__ __forceinline__ void st_32b(void* p, const uint32_t (&w)[8])
+{
+    if constexpr (HALF) st_v4x2(p, w);
+    else st_v8(p, w);
+}
+
 // ---------------------------------------------------------------------------
 // Global memory: one "chunk" is 8 consecutive elements of a row (16 B bf16
 // or fp16, 32 B fp32), read with 128-bit non-coherent loads.

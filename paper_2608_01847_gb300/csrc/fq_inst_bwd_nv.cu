@@ -16,4 +16,6 @@ cudaError_t launch_bwd_shared_nv(int dt, int sub, const KParams& p, uint32_t ny,
     return bwd_shared_by_dt<1>(dt, sub, p, ny, st);
 }
 
+int shared_bwd_occupancy_nv(int dt, int sub) { return shared_occ_by<1>(dt, sub); }
+
 }  // namespace focus

@@ -4,7 +4,10 @@
 // elements for MXFP4, 16 for NVFP4, contiguous along a row): its absmax, its
 // scale, its coefficients and its coefficient gradients are computed once,
 // in registers, with no shuffles.  A block of bf16 is one (NVFP4) or two
-// (MXFP4) 256-bit loads, i.e. exactly one 32-byte sector per lane per load.
+// (MXFP4) 256-bit loads, i.e. exactly one 32-byte sector per lane per load
+// (two 128-bit loads per sector in the HALF instantiations, which the host
+// launches when the rows of a call start on 16-byte but not 32-byte
+// boundaries).
 // The streaming kernels walk a linear block index with a grid-stride loop
 // sized to the resident CTAs, issuing every load of a step before any
 // arithmetic; pairs of elements go through the packed f32x2 instructions.
@@ -47,6 +50,9 @@ struct KParams {
     uint8_t* scales;
     float* ws;            // scratch: per-CTA partials
     uint64_t ld;          // row pitch of x / y / g / gx in elements
+    int half;             // rows of x / y / g / gx start on 16-byte (not 32-byte)
+                          // boundaries: the launch takes the HALF kernels (32-byte
+                          // pieces as two 128-bit accesses)
     uint32_t n_chunks;    // rows * cols / 8 (alpha pass)
     uint32_t cpr;         // 8-element chunks per row
     FastDiv div_cpr;
@@ -85,29 +91,16 @@ struct Geo {
 // ---------------------------------------------------------------------------
 // block I/O
 // ---------------------------------------------------------------------------
-template <int W>
+template <int W, bool HALF>
 __device__ __forceinline__ void load_block(uint32_t (&w)[W], const void* base, uint64_t byte_off)
 {
     const char* p = static_cast<const char*>(base) + byte_off;
 #pragma unroll
     for (int i = 0; i < W / 8; ++i) {
         uint32_t t[8];
-        ld_v8(t, p + 32 * i);
+        ld_32b<HALF>(t, p + 32 * i);
 #pragma unroll
         for (int k = 0; k < 8; ++k) w[8 * i + k] = t[k];
-    }
-}
-
-template <int W>
-__device__ __forceinline__ void store_block(void* base, uint64_t byte_off, const uint32_t (&w)[W])
-{
-    char* p = static_cast<char*>(base) + byte_off;
-#pragma unroll
-    for (int i = 0; i < W / 8; ++i) {
-        uint32_t t[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) t[k] = w[8 * i + k];
-        st_v8(p + 32 * i, t);
     }
 }
 
@@ -424,7 +417,7 @@ __device__ __forceinline__ df sum2x2_merge(const Sum2x2& a)
 //   gd_k = -(T_k / d_k) / (c d_k),   gc = -(sum_k T_k / d_k) / c^2,
 // with T_k / d_k in double-fp32 and the sum over k compensated.
 // ---------------------------------------------------------------------------
-template <int DT, int B, int K, bool SFPG>
+template <int DT, int B, int K, bool SFPG, bool HALF>
 __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw,
                                           const float (&sq)[K], const bool (&dead)[K],
                                           const float (&rho)[K], float c, const float (&d)[K],
@@ -479,7 +472,7 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
                 put_pair<DT>(grp, (e % EPG) / 2,
                              fma2(g2, make_float2(rho[k], rho[k]), make_float2(0.0f, 0.0f)));
                 if (e % EPG == EPG - 2) {
-                    st_v8(static_cast<char*>(gx_base) + off + (e / EPG) * 32, grp);
+                    st_32b<HALF>(static_cast<char*>(gx_base) + off + (e / EPG) * 32, grp);
                 }
             }
             if (want_T) {
@@ -668,7 +661,7 @@ struct TensorGroup {
     __device__ __forceinline__ const TensorScale& ts(int t) const { return scale[t]; }
 };
 
-template <int FMT, int DT, int SUB, int MODE, class Src>
+template <int FMT, int DT, int SUB, int MODE, bool HALF, class Src>
 __device__ __forceinline__ void block_loop(const Src& src)
 {
     using G = Geo<FMT, DT, SUB>;
@@ -717,8 +710,8 @@ __device__ __forceinline__ void block_loop(const Src& src)
                 } else {
                     off[j] = static_cast<uint64_t>(blk) * (B * ESZ);
                 }
-                load_block<W>(xr[j], p.x, off[j]);
-                if constexpr (BWD) load_block<W>(gr[j], p.g, off[j]);
+                load_block<W, HALF>(xr[j], p.x, off[j]);
+                if constexpr (BWD) load_block<W, HALF>(gr[j], p.g, off[j]);
                 if (p.sfp) sv[j] = __ldg(p.sfp + blk);
                 const uint32_t q = p.shared ? cb : blk;
                 if (p.crs) cv[j] = __ldg(p.crs + q);
@@ -774,7 +767,7 @@ __device__ __forceinline__ void block_loop(const Src& src)
                             put_pair<DT>(grp, (el % EPG) / 2,
                                          mul2(make_float2(q[e], q[e + 1]), make_float2(sdq, sdq)));
                             if (el % EPG == EPG - 2)
-                                st_v8(static_cast<char*>(p.y) + off[j] + (el / EPG) * 32, grp);
+                                st_32b<HALF>(static_cast<char*>(p.y) + off[j] + (el / EPG) * 32, grp);
                         }
                     }
                 } else {
@@ -800,8 +793,8 @@ __device__ __forceinline__ void block_loop(const Src& src)
                 if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
                 float gd[K], gc;
                 df T[K], gS;
-                block_bwd<DT, B, K, SFPG>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], sdq, p.ste,
-                                          want_gx, want_T, p.gx, off[j], gd, gc, T, gS);
+                block_bwd<DT, B, K, SFPG, HALF>(xr[j], gr[j], sq, dead, rho, cv[j], dv[j], sdq, p.ste,
+                                                want_gx, want_T, p.gx, off[j], gd, gc, T, gS);
                 if (want_T) {
                     if (p.gdgs) store_coefs<K>(p.gdgs + static_cast<size_t>(blk) * K, gd);
                     if (p.gcrs) p.gcrs[blk] = gc;
@@ -843,7 +836,7 @@ __device__ __forceinline__ void block_loop(const Src& src)
 }
 
 
-template <int FMT, int DT, int SUB, int MODE>
+template <int FMT, int DT, int SUB, int MODE, bool HALF>
 __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
     fq_block_kernel(const KParams p)
 {
@@ -852,10 +845,10 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value)
     // let the next one be scheduled behind this grid
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    block_loop<FMT, DT, SUB, MODE>(OneTensor<FMT>(p));
+    block_loop<FMT, DT, SUB, MODE, HALF>(OneTensor<FMT>(p));
 }
 
-template <int FMT, int DT, int SUB, int MODE>
+template <int FMT, int DT, int SUB, int MODE, bool HALF>
 __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
     fq_group_kernel(const __grid_constant__ KGroup g)
 {
@@ -863,7 +856,7 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value)
     __shared__ TensorScale scale[kMaxGroup];
     if (threadIdx.x < g.n) scale[threadIdx.x] = tensor_scale<FMT>(g.p[threadIdx.x].alpha);
     __syncthreads();
-    block_loop<FMT, DT, SUB, MODE>(TensorGroup<FMT>{g, scale});
+    block_loop<FMT, DT, SUB, MODE, HALF>(TensorGroup<FMT>{g, scale});
 }
 
 // ---------------------------------------------------------------------------
@@ -875,8 +868,22 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value)
 // per (row group, sub-block column) to scratch; fq_bwd_shared_finalize sums
 // the row groups in a fixed order.
 // ---------------------------------------------------------------------------
+// Resident CTAs per SM the shared-row backward's registers must allow.  For
+// NVFP4 with 16-bit elements, 4 (64 registers, a few bytes of spills to L1),
+// as the per-row backward: with the whole-wave grid of shared_row_groups the
+// activations' shared-row backward ran at 6595 GB/s against 6407 at 3 CTAs
+// and a part-empty last wave.  MXFP4 keeps 2 (its unconstrained allocation
+// was 94 registers without spills for bf16 and sub-block 8; bounded to 3
+// CTAs it spilled and measured 6435 against 6763 GB/s), and 1 for 2-element
+// sub-blocks, whose per-sub-block state needs about 200 registers.
 template <int FMT, int DT, int SUB>
-__global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p)
+struct MinCtasShared {
+    static constexpr int value =
+        FMT == 1 ? (DT != 0 ? (SUB == 2 ? 3 : 4) : (SUB == 2 ? 2 : 3)) : (SUB == 2 ? 1 : 2);
+};
+
+template <int FMT, int DT, int SUB, bool HALF>
+__global__ void __launch_bounds__(kThreads, (MinCtasShared<FMT, DT, SUB>::value)) fq_bwd_shared_kernel(const KParams p)
 {
     using G = Geo<FMT, DT, SUB>;
     constexpr int B = G::B, K = G::K, W = G::W;
@@ -905,8 +912,8 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
             uint32_t xr[W], gr[W];
             const uint64_t off =
                 (static_cast<uint64_t>(r) * p.ld + static_cast<uint64_t>(cb) * B) * ESZ;
-            load_block<W>(xr, p.x, off);
-            load_block<W>(gr, p.g, off);
+            load_block<W, HALF>(xr, p.x, off);
+            load_block<W, HALF>(gr, p.g, off);
             uint32_t sbyte;
             const float sdq = block_scale<FMT>(block_absmax<DT, W>(xr), ts, p.mx_rule, sbyte);
             float sq[K];
@@ -916,8 +923,8 @@ __global__ void __launch_bounds__(kThreads) fq_bwd_shared_kernel(const KParams p
             if (want_gx) scale_ratios<K>(sdq, sq, dead, rho);
             float gd[K], gc;
             df T[K], gS;
-            block_bwd<DT, B, K, false>(xr, gr, sq, dead, rho, c, d, sdq, p.ste, want_gx, true,
-                                       p.gx, off, gd, gc, T, gS);
+            block_bwd<DT, B, K, false, HALF>(xr, gr, sq, dead, rho, c, d, sdq, p.ste, want_gx, true,
+                                             p.gx, off, gd, gc, T, gS);
 #pragma unroll
             for (int k = 0; k < K; ++k) acc[k] = df_add(acc[k], T[k]);
         }

@@ -23,9 +23,9 @@ inline int device_sms()
     return n;
 }
 
-// CTAs of the alpha pass and of the shared-row backward's row groups: a
-// fixed multiple of the SM count, so scratch sizes are a pure function of the
-// descriptor and the device.
+// CTAs of the alpha pass (and about as many for the shared-row backward's
+// row groups): a fixed multiple of the SM count, so scratch sizes are a pure
+// function of the descriptor and the device.
 constexpr int kCtasPerSm = 8;
 
 inline uint32_t alpha_grid(uint32_t n_chunks)
@@ -47,14 +47,25 @@ inline uint32_t shared_tx(uint32_t bpr)
 
 inline uint32_t shared_col_ctas(uint32_t bpr) { return (bpr + shared_tx(bpr) - 1) / shared_tx(bpr); }
 
-inline uint32_t shared_row_groups(uint32_t rows, uint32_t bpr)
+// Row groups of the shared-row backward for a kernel with `occ` resident
+// CTAs per SM: the grid (column CTAs x row groups) is a whole number of
+// waves of resident CTAs, about kCtasPerSm per SM, so that no last wave runs
+// part-empty (1216 CTAs at 3 per SM left the SMs a third idle in the last of
+// 2.67 waves), and each CTA walks an equal share of the rows.
+inline uint32_t shared_row_groups(uint32_t rows, uint32_t bpr, int occ)
 {
     const uint32_t nty = kThreads / shared_tx(bpr);
     const uint64_t need = (static_cast<uint64_t>(rows) + nty - 1) / nty;
+    const uint64_t o = static_cast<uint64_t>(std::max(occ, 1));
+    const uint64_t waves = (kCtasPerSm + o - 1) / o;
     const uint64_t cap = std::max<uint64_t>(
-        1, static_cast<uint64_t>(device_sms()) * kCtasPerSm / shared_col_ctas(bpr));
+        1, static_cast<uint64_t>(device_sms()) * o * waves / shared_col_ctas(bpr));
     return static_cast<uint32_t>(std::max<uint64_t>(1, std::min<uint64_t>({need, cap, 65535})));
 }
+
+// Resident CTAs per SM of the shared-row backward kernel (fmt, dtype, sub)
+// on the current device (defined in the backward instantiation units).
+int shared_bwd_occupancy(int fmt, int dt, int sub);
 
 // Grid of a grid-stride streaming kernel: enough CTAs for the work, at most
 // what is resident at once on the device -- except for large tensors (at
@@ -101,13 +112,20 @@ inline cudaError_t launch_dependent(Kern kern, uint32_t grid, cudaStream_t st, c
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+template <int FMT, int DT, int SUB, int MODE, bool HALF>
+cudaError_t run_block_as(const KParams& p, cudaStream_t st)
+{
+    static int occ = 0;
+    auto kern = fq_block_kernel<FMT, DT, SUB, MODE, HALF>;
+    const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Unroll<FMT, DT, MODE>::U * kThreads);
+    return launch_dependent(kern, grid, st, p);
+}
+
+// The 256-bit kernel, or (rows on 16-byte boundaries) the 128-bit one.
 template <int FMT, int DT, int SUB, int MODE>
 cudaError_t run_block(const KParams& p, cudaStream_t st)
 {
-    static int occ = 0;
-    auto kern = fq_block_kernel<FMT, DT, SUB, MODE>;
-    const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Unroll<FMT, DT, MODE>::U * kThreads);
-    return launch_dependent(kern, grid, st, p);
+    return p.half ? run_block_as<FMT, DT, SUB, MODE, true>(p, st) : run_block_as<FMT, DT, SUB, MODE, false>(p, st);
 }
 
 // Dispatch over the sub-block size for one (format, dtype, mode).
@@ -141,11 +159,11 @@ cudaError_t linear_by_dt(int dt, int sub, const KParams& p, cudaStream_t st)
 
 // Group launches: one kernel over the concatenated blocks of up to
 // kMaxGroup tensors that share format, element type and sub-block size.
-template <int FMT, int DT, int SUB, int MODE>
-cudaError_t run_group(const KGroup& g_blocks, cudaStream_t st)
+template <int FMT, int DT, int SUB, int MODE, bool HALF>
+cudaError_t run_group_as(const KGroup& g_blocks, cudaStream_t st)
 {
     static int occ = 0;
-    auto kern = fq_group_kernel<FMT, DT, SUB, MODE>;
+    auto kern = fq_group_kernel<FMT, DT, SUB, MODE, HALF>;
     // every tensor starts on a tile (one CTA step of U * kThreads blocks)
     constexpr uint32_t span = Unroll<FMT, DT, MODE>::U * kThreads;
     KGroup g = g_blocks;
@@ -158,6 +176,15 @@ cudaError_t run_group(const KGroup& g_blocks, cudaStream_t st)
     const uint32_t grid = stream_grid(kern, occ, at, 1);
     kern<<<grid, kThreads, 0, st>>>(g);
     return cudaGetLastError();
+}
+
+// 128-bit accesses for the whole group if any tensor's rows need them.
+template <int FMT, int DT, int SUB, int MODE>
+cudaError_t run_group(const KGroup& g, cudaStream_t st)
+{
+    bool half = false;
+    for (int i = 0; i < g.n; ++i) half = half || g.p[i].half;
+    return half ? run_group_as<FMT, DT, SUB, MODE, true>(g, st) : run_group_as<FMT, DT, SUB, MODE, false>(g, st);
 }
 
 template <int FMT, int DT, int MODE>
@@ -206,7 +233,8 @@ template <int FMT, int DT, int SUB>
 cudaError_t run_bwd_shared(const KParams& p, uint32_t ny, cudaStream_t st)
 {
     const dim3 grid(shared_col_ctas(p.bpr), ny);
-    fq_bwd_shared_kernel<FMT, DT, SUB><<<grid, kThreads, 0, st>>>(p);
+    if (p.half) fq_bwd_shared_kernel<FMT, DT, SUB, true><<<grid, kThreads, 0, st>>>(p);
+    else fq_bwd_shared_kernel<FMT, DT, SUB, false><<<grid, kThreads, 0, st>>>(p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess || (p.gcrs == nullptr && p.gdgs == nullptr && p.step == nullptr)) return e;
     return run_shared_finalize<FMT, SUB>(p, ny, st);
@@ -226,6 +254,49 @@ cudaError_t bwd_shared_by_sub(int sub, const KParams& p, uint32_t ny, cudaStream
     default: break;
     }
     return cudaErrorInvalidValue;
+}
+
+template <int FMT, int DT, int SUB>
+int shared_occ()
+{
+    static int occ = 0;
+    if (occ <= 0) {
+        int o = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fq_bwd_shared_kernel<FMT, DT, SUB, false>, kThreads,
+                                                          0) !=
+                cudaSuccess ||
+            o <= 0)
+            o = 1;
+        occ = o;
+    }
+    return occ;
+}
+
+template <int FMT, int DT>
+int shared_occ_by_sub(int sub)
+{
+    switch (sub) {
+    case 2: return shared_occ<FMT, DT, 2>();
+    case 4: return shared_occ<FMT, DT, 4>();
+    case 8: return shared_occ<FMT, DT, 8>();
+    case 16: return shared_occ<FMT, DT, 16>();
+    case 32:
+        if constexpr (FMT == 0) return shared_occ<FMT, DT, 32>();
+        break;
+    default: break;
+    }
+    return 1;
+}
+
+template <int FMT>
+int shared_occ_by(int dt, int sub)
+{
+    switch (dt) {
+    case 0: return shared_occ_by_sub<FMT, 0>(sub);
+    case 1: return shared_occ_by_sub<FMT, 1>(sub);
+    case 2: return shared_occ_by_sub<FMT, 2>(sub);
+    default: return 1;
+    }
 }
 
 template <int FMT>

@@ -73,7 +73,7 @@ FOCUS_API int focus_nvfp4_alpha_noalloc(const focus_desc_t* desc, const void* x,
     if (desc->dtype != FOCUS_F32 && desc->dtype != FOCUS_BF16 && desc->dtype != FOCUS_F16)
         return FOCUS_ERR_INVALID_ARG;
     if (desc->cols % 8 != 0) return FOCUS_ERR_INVALID_ARG;
-    if ((desc->ld * (desc->dtype == FOCUS_F32 ? 4 : 2)) % 32 != 0) return FOCUS_ERR_MISALIGNED;
+    if ((desc->ld * (desc->dtype == FOCUS_F32 ? 4 : 2)) % 16 != 0) return FOCUS_ERR_MISALIGNED;
     if (desc->rows > 0 && desc->cols > 0 && desc->rows > ((int64_t(1) << 31) - 1) / (desc->cols / 8))
         return FOCUS_ERR_UNSUPPORTED;
     const bool empty = desc->rows == 0 || desc->cols == 0;

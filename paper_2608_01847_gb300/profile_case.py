@@ -3,6 +3,13 @@ profiler captures (ncu) of a single launch on a case of known size.
 
   python -m paper_2608_01847_gb300.profile_case --phase bwd --workload qwen3_4b_layer \
       --tensor gate_proj --fmt nvfp4 --launches 3
+  python -m paper_2608_01847_gb300.profile_case --phase bwd --workload act_262144x4096 \
+      --tensor act --rows 32768 --shared --launches 3
+
+`--rows R` draws only the first R rows' worth of the tensor (the same
+recipe on an [R, cols] tensor), for captures of a smaller case of a large
+workload; `--adam` runs the backward fused with one AdamW step on the
+coefficients (and on S^fp with `--sfp`).
 
 Draws the tensor on the GPU (seeded, same recipe as the benchmark), runs the
 phase `--launches` times and prints the CUDA-event time per launch and the
@@ -45,20 +52,37 @@ def main():
     ap.add_argument("--shared", action="store_true")
     ap.add_argument("--no-gx", action="store_true")
     ap.add_argument("--sfp", action="store_true", help="bwd: learnable S^fp and its gradient")
+    ap.add_argument("--adam", action="store_true", help="bwd: fused with one AdamW step")
+    ap.add_argument("--rows", type=int, default=0, help="draw only this many rows of the tensor")
+    ap.add_argument("--pad", type=int, default=0,
+                    help="row pitch cols + PAD elements (PAD = 8 bf16: rows on 16-byte, not 32-byte, "
+                         "boundaries)")
     ap.add_argument("--launches", type=int, default=3)
     a = ap.parse_args()
 
     B.build()
     F.lib()
+    import dataclasses
     w = W.WORKLOADS[a.workload]
     idx = [t.name for t in w.tensors].index(a.tensor)
+    if a.rows:
+        t = w.tensors[idx]
+        specs = list(w.tensors)
+        specs[idx] = W.TensorSpec(t.name, min(a.rows, t.rows), t.cols)
+        w = dataclasses.replace(w, tensors=tuple(specs))
     fmt = F.FOCUS_MXFP4 if a.fmt == "mxfp4" else F.FOCUS_NVFP4
     blk = F.block_of(fmt)
     x, g = W.device_tensor(w, idx, "cuda")
+    if a.pad:
+        def padded(t):
+            b = torch.zeros((t.shape[0], t.shape[1] + a.pad), dtype=t.dtype, device=t.device)
+            b[:, :t.shape[1]] = t
+            return b[:, :t.shape[1]]
+        x, g = padded(x), padded(g)
     crs, dgs = W.device_coefs(w, idx, blk, a.sub, "cuda", shared=a.shared)
     alpha = F.focus_nvfp4_alpha(x)
-    y = torch.empty_like(x)
-    gx = None if a.no_gx else torch.empty_like(x)
+    y = F._like_x(x)
+    gx = None if a.no_gx else F._like_x(x)
     gc, gd = torch.empty_like(crs), torch.empty_like(dgs)
     sfp = gsfp = None
     if a.sfp:
@@ -86,8 +110,21 @@ def main():
         dmat = torch.empty((a.tokens, rows), dtype=torch.bfloat16, device="cuda")
         del act, g, gx, y
 
+    if a.adam:
+        # the paper's learning rates (Sec. 4.1), PyTorch's AdamW defaults
+        hp = dict(lr_coef=5e-2 if fmt == F.FOCUS_MXFP4 else 1e-3,
+                  lr_scale=2e-2 * 2.0 ** -7 if fmt == F.FOCUS_MXFP4 else 5e-3,
+                  beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01)
+        learned = {"crs": crs, "dgs": dgs, **({"sfp": sfp} if sfp is not None else {})}
+        moments = {k: (torch.zeros_like(v), torch.zeros_like(v)) for k, v in learned.items()}
+        step = torch.ones(1, dtype=torch.int64, device="cuda")
+
     def run():
-        if a.phase == "gemm":
+        if a.phase == "bwd" and a.adam:
+            F.focus_fq_bwd_adamw(x, g, fmt, step, hp, crs=crs, dgs=dgs, sfp=sfp, moments=moments,
+                                 alpha=alpha, sub_block=a.sub, shared=a.shared, gx=gx,
+                                 want_gx=not a.no_gx, ws=ws)
+        elif a.phase == "gemm":
             F.focus_fp4_gemm(fmt, ac, at, wc, wt, act_alpha, alpha, d=dmat)
         elif a.phase == "alpha":
             F.focus_nvfp4_alpha(x, alpha, ws)
@@ -119,8 +156,13 @@ def main():
     bpe = bytes_per_elem(a.phase, a.fmt, a.sub, a.shared, not a.no_gx)
     if a.sfp and a.phase == "bwd":
         bpe += 2 * 4 / blk   # S^fp in, its gradient out
+    if a.adam and a.phase == "bwd":
+        # per learned value p, m, v in and out instead of p in and gradient out
+        coef = 0.0 if a.shared else 4 / blk + 4 / a.sub
+        bpe += 4 * (coef + (4 / blk if a.sfp else 0.0))
     print(json.dumps({"phase": a.phase, "tensor": f"{a.workload}/{a.tensor}", "shape": [rows, cols],
-                      "fmt": a.fmt, "sub": a.sub, "shared": a.shared, "ms": times,
+                      "fmt": a.fmt, "sub": a.sub, "shared": a.shared, "adam": a.adam, "pad": a.pad,
+                      "ms": times,
                       "algorithmic_bytes": n * bpe,
                       "gbs_last": n * bpe / (times[-1] * 1e-3) / 1e9}))
 

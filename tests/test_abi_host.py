@@ -62,8 +62,8 @@ def _desc(rows=4, cols=64, ld=None, dtype=1, fmt=0, block=None, sub=8, shared=0,
 P = ctypes.c_void_p
 ALIGNED = P(0x100000)       # placeholder device addresses: never dereferenced
 ALIGNED2 = P(0x200000)
-ODD = P(0x100010)           # 16-byte aligned only (rows need 32)
-ODD8 = P(0x100008)          # 8-byte aligned only (coefficient arrays need 16)
+ODD = P(0x100008)           # 8-byte aligned only (rows and coefficient arrays need 16)
+ODD8 = ODD
 
 
 def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None, sfp=None):
@@ -74,8 +74,11 @@ def fwd(L, d, x=ALIGNED, crs=None, dgs=None, alpha=ALIGNED2, y=ALIGNED2, sb=None
 @pytest.mark.parametrize("kw,status", [
     (dict(block=64), -2), (dict(fmt=1, block=32), -2), (dict(sub=3), -2), (dict(sub=32, fmt=1), -2),
     (dict(sub=64), -2), (dict(cols=48), -1), (dict(ld=60), -1), (dict(ld=68), -3),
-    (dict(ld=72), -3), (dict(ld=72, dtype=0, rows=0), 0),
-    (dict(dtype=3), -1), (dict(dtype=2, rows=0), 0), (dict(dtype=2, ld=72), -3), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
+    (dict(ld=76), -3), (dict(ld=72, dtype=0, rows=0), 0), (dict(ld=66, dtype=0), -3),
+    # a row pitch of 16 (not 32) bytes passes the checks (shown on empty tensors,
+    # which return before anything is launched)
+    (dict(ld=72, rows=0), 0), (dict(ld=68, dtype=0, rows=0), 0),
+    (dict(dtype=3), -1), (dict(dtype=2, rows=0), 0), (dict(dtype=2, ld=68), -3), (dict(fmt=2), -1), (dict(ste=3), -1), (dict(rule=2), -1),
     (dict(shared=2), -1), (dict(rows=-1), -1), (dict(rows=1 << 40, cols=1 << 20), -2),
 ])
 def test_descriptor_rejections(L, kw, status):

@@ -28,18 +28,20 @@ FMT = {"mx": O.MXFP4, "nv": O.NVFP4}
 
 
 def run_case(x, g, fmt, crs=None, dgs=None, sub=8, shared=False, ste=O.STE_IDENTITY,
-             rule=O.MX_CEIL, alpha=None, pad=0, check_alpha=True):
-    """Run alpha (NVFP4), fwd, pack and bwd on GPU and oracle; compare all."""
+             rule=O.MX_CEIL, alpha=None, pad=0, check_alpha=True, offset=0):
+    """Run alpha (NVFP4), fwd, pack and bwd on GPU and oracle; compare all.
+    pad / offset: the device inputs are columns [offset, offset + cols) of
+    a buffer [rows, offset + cols + pad] (ld > cols, rows off 32-byte
+    boundaries when offset or the pitch is not a multiple of 32 bytes)."""
     rows, cols = x.shape
     block = 32 if fmt == O.MXFP4 else 16
-    # device inputs, optionally as a column slice of a wider buffer (ld > cols)
     xd, gd = dev(x), dev(g)
-    if pad:
-        xb = torch.zeros((rows, cols + pad), dtype=xd.dtype, device="cuda")
+    if pad or offset:
+        xb = torch.zeros((rows, offset + cols + pad), dtype=xd.dtype, device="cuda")
         gb = torch.zeros_like(xb)
-        xb[:, :cols] = xd
-        gb[:, :cols] = gd
-        xd, gd = xb[:, :cols], gb[:, :cols]
+        xb[:, offset:offset + cols] = xd
+        gb[:, offset:offset + cols] = gd
+        xd, gd = xb[:, offset:offset + cols], gb[:, offset:offset + cols]
     cd = dev(crs) if crs is not None else None
     dd = dev(dgs) if dgs is not None else None
     a_dev = None
@@ -106,6 +108,28 @@ def test_shapes(fmt, dtype, rows, cols, pad):
     crs = W.draw_coefs(w, rows * cols // block, 5).reshape(rows, -1)
     dgs = W.draw_coefs(w, rows * cols // 8, 6).reshape(rows, -1)
     run_case(x, g, FMT[fmt], crs, dgs, pad=pad)
+
+
+@pytest.mark.parametrize("fmt", ["mx", "nv"])
+@pytest.mark.parametrize("dtype", ["bf16", "f16", "f32"])
+@pytest.mark.parametrize("pad,offset", [(8, 0), (0, 8), (8, 8), (24, 0)])
+def test_rows_on_16_byte_boundaries(fmt, dtype, pad, offset):
+    """Rows that start on 16-byte but not 32-byte boundaries (row pitch
+    cols + 8 sixteen-bit elements, or a view starting 8 elements into a
+    wider buffer; for fp32, 4-element steps): the kernels take two 128-bit
+    accesses per 32-byte piece, results bit for bit the oracle's, with
+    every phase (and the shared-row backward) on several tiles and a ragged
+    tail."""
+    w, x, g = seeded(300, 672, dtype, seed=41 + pad + offset)
+    if dtype == "f32":
+        pad, offset = pad // 2, offset // 2
+    esz = 4 if dtype == "f32" else 2
+    assert ((672 + pad + offset) * esz) % 32 == 16 or (offset * esz) % 32 == 16
+    block = 32 if fmt == "mx" else 16
+    crs = W.draw_coefs(w, 300 * 672 // block, 5).reshape(300, -1)
+    dgs = W.draw_coefs(w, 300 * 672 // 8, 6).reshape(300, -1)
+    run_case(x, g, FMT[fmt], crs, dgs, pad=pad, offset=offset)
+    run_case(x, g, FMT[fmt], crs[:1], dgs[:1], shared=True, pad=pad, offset=offset)
 
 
 @pytest.mark.parametrize("fmt,sub", [("mx", 2), ("mx", 4), ("mx", 8), ("mx", 16), ("mx", 32),
