@@ -599,8 +599,11 @@ struct Unroll {
 // bound by memory latency: with 16-bit elements, one more CTA per SM than the
 // registers it would like (4 for NVFP4 at 64 registers, 3 for MXFP4 at 80)
 // is faster despite a few dozen bytes of spills to L1-cached local memory
-// (measured: NVFP4 Qwen3-4B backward 6124 -> 6543 GB/s).  The fused
-// optimizer's extra state spills too much there and keeps the lower count.
+// (measured: NVFP4 Qwen3-4B backward 6124 -> 6543 GB/s).  The backward fused
+// with AdamW on the coefficients takes the same counts (Llama-70B layer set,
+// NVFP4 6664 -> 6883 GB/s, MXFP4 6617 -> 6704; Qwen3-4B 6448 -> 6547, against
+// one CTA fewer); with S^fp learned as well its extra state spills too much
+// and keeps one fewer (at the backward's count: 70B NVFP4 6361 -> 6177).
 // The MXFP4 backward with binary16 elements is the exception: its
 // conversions spill three times as much at 3 CTAs, and 2 CTAs per SM are
 // faster (Llama-70B layer set, fp16 I/O: backward 5927 -> 6413 GB/s).
@@ -608,13 +611,16 @@ struct Unroll {
 // (pack phase: Qwen3-4B 5746 -> 5913 GB/s, Llama-70B layer 6715 -> 6796);
 // the MXFP4 export (70B: 6915 -> 6722) and the forward (Qwen3-4B NVFP4: 6409
 // -> 6282) do not.  One fewer for 2-element sub-blocks, whose per-sub-block
-// state is largest.
+// state is largest -- except the plain NVFP4 backward of 16-bit elements,
+// which is faster at the full count there too (70B 6058 -> 6231, Qwen3-4B
+// 5802 -> 5953 GB/s; the MXFP4 one is not: 5325 -> 4850).
 template <int FMT, int DT, int SUB, int MODE>
 struct MinCtas {
     static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT == 1 ? 3 : 2);
-    static constexpr int adam = FMT == 1 ? 3 : 2;
-    static constexpr int value =
-        ((MODE >= kBwdA) ? adam : (MODE >= kBwd) ? bwd : (MODE == kPack && FMT == 1) ? 5 : 4) - (SUB == 2 ? 1 : 0);
+    static constexpr int adam_sfp = FMT == 1 ? 3 : 2;
+    static constexpr int base =
+        MODE == kBwdSA ? adam_sfp : (MODE >= kBwd) ? bwd : (MODE == kPack && FMT == 1) ? 5 : 4;
+    static constexpr int value = base - ((SUB == 2 && !(FMT == 1 && DT != 0 && MODE == kBwd)) ? 1 : 0);
 };
 
 // Where a block's tensor comes from: one tensor (the per-tensor entry
