@@ -423,7 +423,7 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
                                           const float (&rho)[K], float c, const float (&d)[K],
                                           float sdq, int ste, bool want_gx, bool want_T,
                                           void* gx_base, uint64_t off, float (&gd)[K], float& gc,
-                                          df (&T)[K], df& gS)
+                                          df (&T)[K], df& gS, df* q_out = nullptr)
 {
     constexpr int SUB = B / K;
     constexpr int EPG = DT != 0 ? 16 : 8;  // elements per 256-bit group
@@ -495,6 +495,7 @@ __device__ __forceinline__ void block_bwd(const uint32_t* xw, const uint32_t* gw
         }
     }
     gc = -__fmul_rn(__fmul_rn(df_to_f(Q), rc), rc);
+    if (q_out) *q_out = Q;
     if constexpr (SFPG) {
         // dL/dS^dq = sum_k (sum g q - T_k / (S^dq c c^k)) over the live
         // sub-blocks = sum g q - Q / (c S^dq), Q = sum_k T_k / c^k (dead
@@ -595,6 +596,29 @@ struct Unroll {
     static constexpr int U = (MODE >= kBwd) ? 1 : ((FMT == 1 && DT != 0) ? 2 : 1);
 };
 
+// Backward kernels that split each 32-element MXFP4 block over two adjacent
+// lanes (16 elements each; the block maximum and the sums over sub-blocks
+// exchanged by shuffle), which halves the per-thread state of a block.  Taken
+// where it measured faster (backward phase on the Llama-70B layer set, GB/s,
+// one lane per block -> a pair): 16-bit elements with sub-blocks of 2 (5326
+// -> 6355), 4 (6411 -> 6642) or 16 (6700 -> 6962), binary16 with sub-blocks
+// of 8 (6409 -> 6896).  Not for bf16 with sub-blocks of 8 (7035 -> 6891), nor
+// with the S^fp gradient or the fused optimizer (5-13 % slower: both lanes
+// redo the per-block work, and their state does not halve), nor for binary32
+// (not measured).
+template <int FMT, int DT, int SUB, int MODE>
+struct PairBlocks {
+    static constexpr bool value =
+        FMT == 0 && MODE == kBwd && DT != 0 && SUB <= 16 && (SUB != 8 || DT == 2);
+};
+
+// Blocks one CTA covers per step of its grid-stride loop.
+template <int FMT, int DT, int SUB, int MODE>
+struct Span {
+    static constexpr int value =
+        PairBlocks<FMT, DT, SUB, MODE>::value ? kThreads / 2 : Unroll<FMT, DT, MODE>::U * kThreads;
+};
+
 // Resident CTAs per SM the register allocation must allow.  The backward is
 // bound by memory latency: with 16-bit elements, one more CTA per SM than the
 // registers it would like (4 for NVFP4 at 64 registers, 3 for MXFP4 at 80)
@@ -614,8 +638,10 @@ struct Unroll {
 // state is largest -- except the plain NVFP4 backward of 16-bit elements,
 // which is faster at the full count there too (70B 6058 -> 6231, Qwen3-4B
 // 5802 -> 5953 GB/s; the MXFP4 one is not: 5325 -> 4850).
-template <int FMT, int DT, int SUB, int MODE>
+template <int FMT_, int DT, int SUB, int MODE>
 struct MinCtas {
+    // a thread of a pair kernel holds 16 elements, as an NVFP4 thread does
+    static constexpr int FMT = PairBlocks<FMT_, DT, SUB, MODE>::value ? 1 : FMT_;
     static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT == 1 ? 3 : 2);
     static constexpr int adam_sfp = FMT == 1 ? 3 : 2;
     static constexpr int base =
@@ -841,6 +867,136 @@ __device__ __forceinline__ void block_loop(const Src& src)
     }
 }
 
+// ---------------------------------------------------------------------------
+// MXFP4 backward with each 32-element block split over two adjacent lanes
+// (PairBlocks): lane h of the pair owns elements 16h .. 16h+15, i.e. the
+// sub-blocks K/2 h .. K/2 h + K/2 - 1.  The pair computes the block maximum
+// with one shuffle, each lane its half's input gradient, sub-block sums and
+// DGS gradients as block_bwd does for a 16-element block, and the pair adds
+// the two halves of sum_k T_k / c^k (and of dL/dS^dq) in a fixed order, lower
+// half first, for the CRS gradient and the S^fp gradient; lane 0 of the pair
+// writes the per-block results.  Every lane runs every step (lanes past the
+// last block compute on zeros and store nothing), so the shuffles see full
+// warps.
+// ---------------------------------------------------------------------------
+template <int DT, int SUB, int MODE, bool HALF, class Src>
+__device__ __forceinline__ void pair_bwd_loop(const Src& src)
+{
+    constexpr int B = 32, K = B / SUB, BH = 16, KH = K / 2;
+    constexpr int WH = DT != 0 ? BH / 2 : BH;   // 32-bit words of a half block
+    constexpr int ESZ = DT != 0 ? 2 : 4;
+    constexpr bool SFPG = MODE == kBwdS || MODE == kBwdSA;
+    constexpr bool ADAM = MODE >= kBwdA;
+    static_assert(KH >= 1 && BH % SUB == 0, "a sub-block must lie in one half");
+    AdamW aw;
+    if constexpr (ADAM) aw = adamw_setup(src.at(0));
+    const uint32_t span = kThreads / 2;
+    const uint32_t n_tiles = src.tiles(span);
+    const uint32_t h = threadIdx.x & 1u;
+
+    for (uint32_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        const int tt = src.tensor(tile);
+        const KParams& p = src.at(tt);
+        const TensorScale& ts = src.ts(tt);
+        const uint32_t blk = src.base(tile, tt, span) + threadIdx.x / 2;
+        const bool valid = blk < p.n_blocks;
+        const bool want_gx = p.gx != nullptr;
+        const bool want_T = SFPG || p.gcrs != nullptr || p.gdgs != nullptr ||
+                            (ADAM && (p.new_crs != nullptr || p.new_dgs != nullptr));
+        uint32_t xr[WH], gr[WH];
+        float cv = 1.0f, sv = 0.0f, dv[KH];
+        BlockMoments<ADAM ? KH : 1> mo;
+#pragma unroll
+        for (int k = 0; k < KH; ++k) dv[k] = 1.0f;
+        uint64_t off = 0;
+        if (valid) {
+            uint32_t cb = 0;
+            if (p.strided || p.shared) {
+                const uint32_t row = fast_div(blk, p.div_bpr);
+                cb = blk - row * p.bpr;
+                off = (static_cast<uint64_t>(row) * p.ld + static_cast<uint64_t>(cb) * B + BH * h) * ESZ;
+            } else {
+                off = (static_cast<uint64_t>(blk) * B + BH * h) * ESZ;
+            }
+            load_block<WH, HALF>(xr, p.x, off);
+            load_block<WH, HALF>(gr, p.g, off);
+            if (p.sfp) sv = __ldg(p.sfp + blk);
+            const uint32_t q = p.shared ? cb : blk;
+            if (p.crs) cv = __ldg(p.crs + q);
+            if (p.dgs) load_coefs<KH>(p.dgs + static_cast<size_t>(q) * K + KH * h, dv);
+            if constexpr (ADAM) {
+                if (p.new_crs) {
+                    mo.mc = p.opt_m[0][blk];
+                    mo.vc = p.opt_v[0][blk];
+                }
+                if (p.new_dgs) {
+                    load_coefs<KH>(p.opt_m[1] + static_cast<size_t>(blk) * K + KH * h, mo.md);
+                    load_coefs<KH>(p.opt_v[1] + static_cast<size_t>(blk) * K + KH * h, mo.vd);
+                }
+                if (SFPG && p.new_sfp) {
+                    mo.ms = p.opt_m[2][blk];
+                    mo.vs = p.opt_v[2][blk];
+                }
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < WH; ++i) xr[i] = gr[i] = 0u;
+        }
+        // the block maximum over both halves (max of non-negative floats)
+        const float mh = block_absmax<DT, WH>(xr);
+        const float m = fmaxf(mh, __shfl_xor_sync(kFullMask, mh, 1));
+        uint32_t sbyte;
+        const float sdq = p.sfp ? block_scale_fp<0>(sv, ts, sbyte) : block_scale<0>(m, ts, p.mx_rule, sbyte);
+        float sq[KH];
+        bool dead[KH];
+        relaxed_scales<KH>(sdq, cv, dv, sq, dead);
+        float rho[KH];
+        if (want_gx) scale_ratios<KH>(sdq, sq, dead, rho);
+        float gd[KH], gc_half;
+        df T[KH], gS, Q;
+        block_bwd<DT, BH, KH, SFPG, HALF>(xr, gr, sq, dead, rho, cv, dv, sdq, p.ste, want_gx && valid,
+                                          want_T, p.gx, off, gd, gc_half, T, gS, &Q);
+        // the two halves' sums, lower half first
+        const df Qo = shfl_xor_df(Q, 1);
+        const df Qt = h == 0 ? df_add(Q, Qo) : df_add(Qo, Q);
+        const float rc = rcp_approx(cv);
+        const float gc = -__fmul_rn(__fmul_rn(df_to_f(Qt), rc), rc);
+        float gs = 0.0f;
+        if constexpr (SFPG) {
+            const df So = shfl_xor_df(gS, 1);
+            gs = df_to_f(h == 0 ? df_add(gS, So) : df_add(So, gS));   // STE through Q_fmt: dS^dq/dS^fp = 1
+        }
+        if (!valid) continue;
+        if (want_T && p.gdgs) store_coefs<KH>(p.gdgs + static_cast<size_t>(blk) * K + KH * h, gd);
+        if (h == 0) {
+            if (want_T && p.gcrs) p.gcrs[blk] = gc;
+            if (SFPG && p.gsfp) p.gsfp[blk] = gs;
+        }
+        if constexpr (ADAM) {
+            if (p.new_crs && h == 0) {
+                p.new_crs[blk] = adamw_update(cv, gc, mo.mc, mo.vc, aw.step_c, aw.decay_c, aw);
+                p.opt_m[0][blk] = mo.mc;
+                p.opt_v[0][blk] = mo.vc;
+            }
+            if (p.new_dgs) {
+                float nd[KH];
+#pragma unroll
+                for (int k = 0; k < KH; ++k)
+                    nd[k] = adamw_update(dv[k], gd[k], mo.md[k], mo.vd[k], aw.step_c, aw.decay_c, aw);
+                const size_t q = static_cast<size_t>(blk) * K + KH * h;
+                store_coefs<KH>(p.new_dgs + q, nd);
+                store_coefs<KH>(p.opt_m[1] + q, mo.md);
+                store_coefs<KH>(p.opt_v[1] + q, mo.vd);
+            }
+            if (SFPG && p.new_sfp && h == 0) {
+                p.new_sfp[blk] = adamw_update(sv, gs, mo.ms, mo.vs, aw.step_s, aw.decay_s, aw);
+                p.opt_m[2][blk] = mo.ms;
+                p.opt_v[2][blk] = mo.vs;
+            }
+        }
+    }
+}
+
 
 template <int FMT, int DT, int SUB, int MODE, bool HALF>
 __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value))
@@ -851,7 +1007,10 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value)
     // let the next one be scheduled behind this grid
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    block_loop<FMT, DT, SUB, MODE, HALF>(OneTensor<FMT>(p));
+    if constexpr (PairBlocks<FMT, DT, SUB, MODE>::value)
+        pair_bwd_loop<DT, SUB, MODE, HALF>(OneTensor<FMT>(p));
+    else
+        block_loop<FMT, DT, SUB, MODE, HALF>(OneTensor<FMT>(p));
 }
 
 template <int FMT, int DT, int SUB, int MODE, bool HALF>
@@ -862,7 +1021,10 @@ __global__ void __launch_bounds__(kThreads, (MinCtas<FMT, DT, SUB, MODE>::value)
     __shared__ TensorScale scale[kMaxGroup];
     if (threadIdx.x < g.n) scale[threadIdx.x] = tensor_scale<FMT>(g.p[threadIdx.x].alpha);
     __syncthreads();
-    block_loop<FMT, DT, SUB, MODE, HALF>(TensorGroup<FMT>{g, scale});
+    if constexpr (PairBlocks<FMT, DT, SUB, MODE>::value)
+        pair_bwd_loop<DT, SUB, MODE, HALF>(TensorGroup<FMT>{g, scale});
+    else
+        block_loop<FMT, DT, SUB, MODE, HALF>(TensorGroup<FMT>{g, scale});
 }
 
 // ---------------------------------------------------------------------------

@@ -117,7 +117,7 @@ cudaError_t run_block_as(const KParams& p, cudaStream_t st)
 {
     static int occ = 0;
     auto kern = fq_block_kernel<FMT, DT, SUB, MODE, HALF>;
-    const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Unroll<FMT, DT, MODE>::U * kThreads);
+    const uint32_t grid = stream_grid(kern, occ, p.n_blocks, Span<FMT, DT, SUB, MODE>::value);
     return launch_dependent(kern, grid, st, p);
 }
 
@@ -164,8 +164,8 @@ cudaError_t run_group_as(const KGroup& g_blocks, cudaStream_t st)
 {
     static int occ = 0;
     auto kern = fq_group_kernel<FMT, DT, SUB, MODE, HALF>;
-    // every tensor starts on a tile (one CTA step of U * kThreads blocks)
-    constexpr uint32_t span = Unroll<FMT, DT, MODE>::U * kThreads;
+    // every tensor starts on a tile (one CTA step of blocks)
+    constexpr uint32_t span = Span<FMT, DT, SUB, MODE>::value;
     KGroup g = g_blocks;
     uint32_t at = 0;
     for (int i = 0; i < g.n; ++i) {
