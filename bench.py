@@ -100,7 +100,7 @@ TRAFFIC = {
     # fq_block_kernel<1,1,8,2> on [32768, 4096] of the activations: 637.6 MB
     # read + 336.8 MB written for 134,217,728 elements
     # (profiles/fq_bwd_nvfp4_act_32768rows.txt)
-    ("act_262144x4096", "nvfp4", "bwd"): {"sources": "a8fbe65a5cacc9ba", "bytes_per_elem": 7.2602},
+    ("act_262144x4096", "nvfp4", "bwd"): {"sources": "bcb91ae283e0cd82", "bytes_per_elem": 7.2602},
 }
 
 # AdamW hyper-parameters of the fused optimizer: the paper's learning rates
