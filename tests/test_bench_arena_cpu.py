@@ -81,3 +81,24 @@ def test_arena_mirror_round_trip():
         buf[s:e].copy_(mirror[s:e])
     for n in names:
         assert torch.equal(getattr(o, n), before[n]), n
+
+
+def test_tensor_piece_views_rows():
+    """A row piece of a benchmark tensor: every row array (and the optimizer
+    moments) becomes the view of rows [r0, r1) of the same storage, the
+    per-tensor arrays (alpha, scratch) stay shared, the element count
+    follows the rows."""
+    o = make()
+    o.case = types.SimpleNamespace(shared=False, adam=True)
+    o.alpha = torch.zeros(1)
+    o.moments = {"crs": (torch.rand(37, 4), torch.rand(37, 4))}
+    o.n = o.x.numel()
+    p = bench.tensor_piece(o, 5, 12)
+    for n in ("x", "g", "crs", "dgs", "codes", "scales"):
+        v, whole = getattr(p, n), getattr(o, n)
+        assert v.shape[0] == 7 and v.data_ptr() == whole[5].data_ptr(), n
+        assert torch.equal(v, whole[5:12]), n
+    m, vv = p.moments["crs"]
+    assert m.data_ptr() == o.moments["crs"][0][5].data_ptr() and vv.shape == (7, 4)
+    assert p.alpha is o.alpha and p.n == 7 * 64
+    assert o.x.shape[0] == 37 and o.n == 37 * 64      # the whole tensor is unchanged
