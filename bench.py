@@ -568,9 +568,10 @@ class PipelineGraph:
 
     A tensor of more than 2 * piece_elems elements (per-row coefficients) is
     moved and computed in row pieces of about piece_elems elements: the
-    pieces' forward-side inputs (x and coefficients) first, then their
-    upstream gradients; the forward and pack of a piece start once its rows
-    have arrived (NVFP4: once all of x has, for the per-tensor alpha), its
+    pieces' forward-side inputs (x and coefficients; NVFP4: all of x first,
+    then the coefficients) first, then their upstream gradients; the forward
+    and pack of a piece start once its rows have arrived (NVFP4: once all of
+    x has, for the per-tensor alpha), its
     values, codes and scale bytes leave while the gradients still arrive,
     and its backward outputs follow its backward.  With the fused optimizer
     the phases keep their order (the pack reads the updated coefficients)."""
@@ -645,16 +646,25 @@ class PipelineGraph:
                      id(getattr(t, n)) in ids(t.outputs())]
         fwd_in = [n for n in in_names if id(getattr(t, n)) not in grad_in]
         g_in = [n for n in in_names if id(getattr(t, n)) in grad_in]
+        # NVFP4: every output waits for the per-tensor alpha, i.e. for all of
+        # x, so x crosses first and the pieces' coefficients after it;
+        # without alpha a piece's x and coefficients travel together
+        x_first = "alpha" in phases and "x" in fwd_in
+        e_xall = torch.cuda.Event()
         with torch.cuda.stream(s_in):
+            if x_first:
+                for p in pcs:
+                    h2d(t, [p.x])
+                e_xall.record()
             for p, e in zip(pcs, e_x):
-                h2d(t, [getattr(p, n) for n in fwd_in])
+                h2d(t, [getattr(p, n) for n in fwd_in if not (x_first and n == "x")])
                 e.record()
             for p, e in zip(pcs, e_g):
                 h2d(t, [getattr(p, n) for n in g_in])
                 e.record()
         with torch.cuda.stream(s_cmp):
             if "alpha" in phases:
-                s_cmp.wait_event(e_x[-1])
+                s_cmp.wait_event(e_xall if x_first else e_x[-1])
                 t.run("alpha", parity)
             for p, ex, ef in zip(pcs, e_x, e_f):
                 s_cmp.wait_event(ex)
