@@ -87,6 +87,18 @@ def test_full_size_per_row(name, fmt):
         _check_tensor(w, idx, fmt)
 
 
+@pytest.mark.parametrize("fmt,sub,io", [(O.MXFP4, 2, "bf16"), (O.MXFP4, 4, "bf16"), (O.MXFP4, 8, "f16"),
+                                        (O.MXFP4, 16, "f16"), (O.NVFP4, 2, "bf16")])
+def test_full_size_variants(fmt, sub, io):
+    """Table 5's sub-block sizes and binary16 elements on the 70B gate_proj
+    [28672, 8192] at full size, in the launch configuration the benchmark
+    uses: the MXFP4 backward there splits each block over two lanes, the
+    NVFP4 one at sub-block 2 runs at four CTAs per SM."""
+    import dataclasses
+    w = dataclasses.replace(W.WORKLOADS["llama_70b_layer"], dtype=io)
+    _check_tensor(w, 4, fmt, sub=sub, seed=sub)
+
+
 @pytest.mark.parametrize("fmt", [O.MXFP4, O.NVFP4])
 def test_full_size_sweep_4gb(fmt):
     """The sweep's largest point: one [262144, 8192] bf16 tensor, 2^31
