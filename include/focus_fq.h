@@ -290,7 +290,9 @@ size_t focus_mma_scale_bytes(const focus_desc_t* desc);
  * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
  * kernel whose wait on its pipeline gives up sets it to 1 (the output is
  * then incomplete) instead of waiting for ever.  Enqueued on `stream`; the
- * kernel is persistent (one CTA per SM, each loading its own operand tiles). */
+ * kernel is persistent and launched in clusters of two CTAs (one per SM),
+ * each pair computing 256 x 256 tiles of D with the tensor cores of both of
+ * its SMs; every CTA loads its own operand tiles. */
 int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const uint8_t* a_codes,
                    const uint8_t* a_scale_tiles, const float* alpha_a, const uint8_t* b_codes,
                    const uint8_t* b_scale_tiles, const float* alpha_b, void* d, int32_t d_dtype,
