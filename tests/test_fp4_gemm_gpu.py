@@ -162,8 +162,9 @@ def test_fp4_gemm_bf16_output(fmt):
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
 def test_fp4_gemm_full_size_sampled(fmt):
     """The benchmark's largest Qwen3-4B GEMM at full size (8192 tokens x
-    gate_proj [9728, 2560]: 2432 tiles of 128 x 256 on one CTA per SM, so
-    every barrier of the ring and of the accumulator wraps many times), with fp32
+    gate_proj [9728, 2560]: 1216 tiles of 256 x 256 on 76 persistent CTA
+    pairs, so every barrier of the ring, of the scale sets and of the
+    accumulator wraps many times), with fp32
     and with bf16 output: D on 32 sampled rows x 32 sampled columns (first,
     last, random) against the oracle's contraction of the oracle's export of
     those rows, whose codes and scale bytes also match the GPU export."""
