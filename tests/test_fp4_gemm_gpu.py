@@ -85,7 +85,11 @@ def check_gemm(fmt, M, N, K, seed=0, crs=True):
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
 @pytest.mark.parametrize("M,N,K", [(128, 128, 64), (128, 128, 256), (256, 384, 512), (200, 130, 320),
                                    (1, 1, 64), (129, 257, 1024), (384, 128, 2560),
-                                   (200, 132, 320), (130, 260, 512), (300, 520, 256)])
+                                   (200, 132, 320), (130, 260, 512), (300, 520, 256),
+                                   # several 256 x 256 pair tiles both ways; the last tile row and
+                                   # column leave the second CTA of the pair without rows of A / B;
+                                   # K of 13 steps ends in a one-step chunk
+                                   (513, 770, 832)])
 def test_fp4_gemm_parity(fmt, M, N, K):
     check_gemm(FMT[fmt], M, N, K, seed=M + N + K)
 
