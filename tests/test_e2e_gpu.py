@@ -85,3 +85,50 @@ def test_pipeline_returns_the_step_results(fmt, shared, sfp, adam, piece_elems):
             assert torch.equal(got.view(torch.uint8), r.cpu().contiguous().view(torch.uint8)), (i, j)
     for a, r in zip(learned, ref_learned):   # the optimizer's step, in HBM
         assert torch.equal(a.view(torch.int32), r.view(torch.int32))
+
+
+@pytest.mark.parametrize("fmt,shared,sfp", [("nvfp4", False, False), ("mxfp4", False, True),
+                                            ("nvfp4", True, False)])
+def test_staged_steps_return_the_step_results(fmt, shared, sfp):
+    """The benchmark's end-to-end steps without the fused optimizer: two
+    buffer sets on two streams, each step an input graph, a compute graph
+    and an output graph, step k's inputs crossing while step k - 1 returns
+    its outputs.
+    Three steps (sets A, B, A) from poisoned device buffers: each set's host
+    mirror receives exactly the results of the phases called directly."""
+    w = W.Workload("e2e", tuple(W.TensorSpec(f"t{i}", r, c) for i, (r, c) in enumerate(SHAPES)), "bf16",
+                   ("mxfp4", "nvfp4"), "weight", 5.0, 0.02, "entries", 0.01, 20.0, (0.9, 1.1), 314)
+    case = bench.Case(workload="e2e", fmt=fmt, shared=shared, sfp=sfp)
+    dev = torch.device("cuda")
+    sets = [[bench.Tensor(case, w, i, dev, None) for i in range(len(SHAPES))] for _ in range(2)]
+    phases = case.phases()
+    for ph in phases:
+        for t in sets[0]:
+            t.run(ph)
+    torch.cuda.synchronize()
+    ref = [[o.clone() for o in t.outputs()] for t in sets[0]]
+    for t, t2 in zip(*sets):
+        t.host_in = t.in_buf.cpu().pin_memory()
+        t2.host_in = t.host_in
+        for u in (t, t2):
+            u.host_out = torch.full_like(u.out_buf, 0x5A, device="cpu").pin_memory()
+    staged = bench.StagedE2E(sets, phases, dev)
+    arrays = [a for t in sets[0] for a in t.inputs()]
+    extra = staged.h2d - sum(a.numel() * a.element_size() for a in arrays)
+    assert 0 <= extra < bench.ARENA_ALIGN * len(arrays), extra
+    for ts in sets:   # poison: every input must come in, every output go out
+        for t in ts:
+            t.in_buf.fill_(0xA5)
+            t.out_buf.fill_(0xC3)
+    torch.cuda.synchronize()
+    main = torch.cuda.current_stream()
+    staged.fork(main)
+    for _ in range(3):
+        staged.step()
+    staged.join(main)
+    torch.cuda.synchronize()
+    for ts in sets:
+        for i, t in enumerate(ts):
+            for j, (a, r) in enumerate(zip(t.outputs(), ref[i])):
+                got = host_view(t, t.host_out, t.out_buf, a)
+                assert torch.equal(got.view(torch.uint8), r.cpu().contiguous().view(torch.uint8)), (i, j)
