@@ -132,11 +132,13 @@ def adamw_bounds(p, m, v, g, g_abs, floor, lr, beta1, beta2, eps, wd, step):
     dh = np.sqrt(np.maximum(vh, 0.0)) * R
     dl = dl * (1 - 20 * U32) + eps * (1 - U32)
     dh = dh * (1 + 20 * U32) + eps * (1 + U32)
-    # m / den over the corners (den > 0), plus the division's rounding
+    # m / den over the corners (den > 0), plus the division's error (the
+    # device's approximate division: within 2 ulp; the square root's 2 ulp
+    # are inside the denominator's slack above)
     c = np.stack([ml / dl, ml / dh, mh / dl, mh / dh])
     ul, uh = c.min(0), c.max(0)
     umax = np.maximum(np.abs(ul), np.abs(uh))
-    ul, uh = ul - U32 * umax, uh + U32 * umax
+    ul, uh = ul - 3 * U32 * umax, uh + 3 * U32 * umax
     # p (1 - lr wd) - lr / (1 - beta1^t) * (m / den)
     S = lr / (1.0 - b1 ** step)
     pd = p * (1.0 - lr * wd)

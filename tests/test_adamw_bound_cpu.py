@@ -1,7 +1,8 @@
 """The AdamW tolerance of the GPU tests, checked on the CPU: a binary32
 evaluation in the device's operation order, from any gradient within the
-gradient tolerance, lies inside the interval; the same evaluation with a
-plausible mistake in the update does not."""
+gradient tolerance and with its square root and division off by up to 2 ulp
+(the device's approximate forms), lies inside the interval; the same
+evaluation with a plausible mistake in the update does not."""
 import numpy as np
 import pytest
 
@@ -11,8 +12,19 @@ from gpu_helpers import FLOOR_ROW, REL, adamw_bounds
 F = np.float32
 
 
-def device_order_f32(p, g, m, v, lr, b1, b2, eps, wd, t, mistake=None):
-    """The fused kernel's update in binary32 (each line one rounding)."""
+def ulps(a, k):
+    """Binary32 values a moved by k units in the last place."""
+    a = np.asarray(a, F)
+    towards = F(np.inf) if k > 0 else F(-np.inf)
+    for _ in range(abs(k)):
+        a = np.nextafter(a, towards)
+    return a
+
+
+def device_order_f32(p, g, m, v, lr, b1, b2, eps, wd, t, mistake=None, sqrt_ulps=0, div_ulps=0):
+    """The fused kernel's update in binary32 (each line one rounding); the
+    kernel's square root and division are approximations within 2 ulp,
+    modelled by moving the correctly rounded ones by sqrt_ulps / div_ulps."""
     p, g, m, v = (np.asarray(a, F) for a in (p, g, m, v))
     lr, b1, b2, eps, wd = F(lr), F(b1), F(b2), F(eps), F(wd)
     o1, o2 = F(1) - b1, F(1) - b2
@@ -30,10 +42,10 @@ def device_order_f32(p, g, m, v, lr, b1, b2, eps, wd, t, mistake=None):
         b1, b2, o1, o2 = b2, b1, o2, o1
     m = b1 * m + o1 * g
     v = b2 * v + o2 * (g * g)
-    den = np.sqrt(v) * rbc2 + eps
+    den = ulps(np.sqrt(v), sqrt_ulps) * rbc2 + eps
     if mistake == "eps_inside_sqrt":
         den = np.sqrt(v * rbc2 * rbc2 + eps)
-    return p * decay - step * (m / den), m, v
+    return p * decay - step * ulps(m / den, div_ulps), m, v
 
 
 def cases(rng, n):
@@ -67,10 +79,11 @@ def test_device_order_within_bound(step, lr):
     dg = REL * np.abs(g) + FLOOR_ROW * g_abs
     for s in (-1.0, 1.0, None):
         gd = g + (dg * s if s is not None else dg * rng.uniform(-1, 1, n))
-        pd, md, vd = device_order_f32(p, gd.astype(F), m, v, lr, *hp, step)
-        for val, lo, hi in ((pd, pl, ph), (md, ml, mh), (vd, vl, vh)):
-            val = val.astype(np.float64)
-            assert np.all((val >= lo) & (val <= hi))
+        for su, du in ((0, 0), (2, 2), (-2, -2), (2, -2), (-2, 2)):
+            pd, md, vd = device_order_f32(p, gd.astype(F), m, v, lr, *hp, step, sqrt_ulps=su, div_ulps=du)
+            for val, lo, hi in ((pd, pl, ph), (md, ml, mh), (vd, vl, vh)):
+                val = val.astype(np.float64)
+                assert np.all((val >= lo) & (val <= hi)), (su, du)
 
 
 @pytest.mark.parametrize("mistake", ["no_bias_correction", "no_decay", "swapped_betas",
