@@ -224,8 +224,12 @@ typedef struct {
  *   m <- beta1 * m + (1 - beta1) * grad,  v <- beta2 * v + (1 - beta2) * grad^2
  *   p <- p - lr / (1 - beta1^t) * m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
  * (PyTorch's AdamW) with lr = hp->lr_scale for sfp and hp->lr_coef for the
- * coefficients, in binary32, and writes the new moments.  The gradients are
- * not written to memory unless gcrs / gdgs / gsfp are given.
+ * coefficients, in binary32, and writes the new moments.  The moments are
+ * correctly rounded binary32 operations; the square root and the division of
+ * the last line are the hardware's approximate forms (within 2 ulp each), so
+ * the new parameters may differ from a correctly rounded evaluation by a few
+ * ulp.  The gradients are not written to memory unless gcrs / gdgs / gsfp
+ * are given.
  * crs, dgs, sfp  parameters as for focus_fq_bwd, updated in place; NULL: not
  *        learned (coefficient 1 / absmax scale).  sfp only with per-row
  *        coefficients.
