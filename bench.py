@@ -915,7 +915,8 @@ def gpu_arm(case, args, rank, world, device):
     for t in ts:
         t.host_in = t.in_buf.cpu().pin_memory()   # every batch's inputs
         t.host_out = torch.empty_like(t.out_buf, device="cpu").pin_memory()
-    if not case.adam and (case.fmt == "nvfp4" or case.shared):
+    staged_used = not case.adam and (case.fmt == "nvfp4" or case.shared)
+    if staged_used:
         # Steps without the fused optimizer are independent.  Where one step
         # cannot overlap its own input and output copies -- NVFP4, whose
         # outputs all wait for the whole of x (the per-tensor alpha), and
@@ -968,7 +969,11 @@ def gpu_arm(case, args, rank, world, device):
         barrier()
     e2e_ms = e0.elapsed_time(e1) / e2e_steps
     e2e_ms = max_over_ranks(e2e_ms, world, device)
-    res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
+    method = ("pinned host buffers, two device buffer sets: step k's inputs cross the host link while "
+              "step k-1's outputs return (input, compute and output graphs per step)" if staged_used else
+              "pinned host buffers, one device buffer set: one graph per step, H2D, compute and D2H "
+              "chains pipelined over tensors and row pieces")
+    res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h, e2e_method=method)
     return res
 
 
@@ -1502,6 +1507,7 @@ def device_line(case, r, args, world, default_case):
                           f"inputs larger than L2: x+g = {r['n_elem'] * 2 * r['esz'] / 2**20:.0f} MiB"
                           " per step"),
                    "parallelism": f"replicas x{world}",
+                   **({"e2e_method": r["e2e_method"]} if "e2e_method" in r else {}),
                    "phase_split": (f"each phase captured {r['phase_reps']} times in one graph (tensors joined "
                                    "between repetitions), timed per repetition" if r["phase_reps"] > 1 else
                                    "each phase graph timed per replay")},
