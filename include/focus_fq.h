@@ -290,7 +290,8 @@ size_t focus_mma_scale_bytes(const focus_desc_t* desc);
  * FOCUS_BF16 rounded to nearest even), overwritten.  The products are exact
  * and accumulate in fp32 inside the tensor core; alpha is applied to the
  * fp32 sum before the output rounding.
- * Requirements: K % 64 == 0 (FOCUS_ERR_UNSUPPORTED otherwise); codes and
+ * Requirements: K % 32 == 0 (FOCUS_ERR_UNSUPPORTED otherwise: code rows on
+ * 16-byte boundaries); codes and
  * scale tiles 16-byte aligned.  timeout_flag: optional device int32; a
  * kernel whose wait on its pipeline gives up sets it to 1 (the output is
  * then incomplete) instead of waiting for ever.  Enqueued on `stream`; the

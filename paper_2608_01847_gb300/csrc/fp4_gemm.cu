@@ -118,7 +118,7 @@ struct GemmParams {
     uint32_t tiles_k;      // scale tiles per 128-row tile row: ceil(K / block / 4)
     uint32_t tiles_m, tiles_n;   // pair tiles: ceil(M / 256), ceil(N / 256)
     uint32_t tile_rows_b;  // 128-row scale-tile rows of B: ceil(N / 128)
-    uint32_t n_steps;      // K / 64
+    uint32_t n_steps;      // ceil(K / 64)
     int d_bf16;
     int d_vec;             // rows of D start on 16-byte boundaries: TMA stores through tma_d
 };
@@ -636,7 +636,10 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
     if (fmt != FOCUS_MXFP4 && fmt != FOCUS_NVFP4) return FOCUS_ERR_INVALID_ARG;
     if (d_dtype != FOCUS_F32 && d_dtype != FOCUS_BF16) return FOCUS_ERR_INVALID_ARG;
     if (M < 0 || N < 0 || K < 0 || ldd < N) return FOCUS_ERR_INVALID_ARG;
-    if (K % 64 != 0) return FOCUS_ERR_UNSUPPORTED;
+    // rows of codes on 16-byte boundaries (the tensor maps' pitch); a last K
+    // step of 32 elements reads zero codes past K (the maps' fill) with the
+    // zeroed padding of the export's scale tiles
+    if (K % 32 != 0) return FOCUS_ERR_UNSUPPORTED;
     if (M > (int64_t(1) << 31) - kPairM || N > (int64_t(1) << 31) - kTileN || K > (int64_t(1) << 31))
         return FOCUS_ERR_UNSUPPORTED;
     if (M == 0 || N == 0) return FOCUS_OK;
@@ -673,7 +676,7 @@ FOCUS_API int focus_fp4_gemm(int32_t fmt, int64_t M, int64_t N, int64_t K, const
     p.tiles_m = static_cast<uint32_t>((M + kPairM - 1) / kPairM);
     p.tiles_n = static_cast<uint32_t>((N + kTileN - 1) / kTileN);
     p.tile_rows_b = static_cast<uint32_t>((N + kTile - 1) / kTile);
-    p.n_steps = static_cast<uint32_t>(K / 64);
+    p.n_steps = static_cast<uint32_t>((K + 63) / 64);
     p.d_bf16 = bf16;
     p.d_vec = !misaligned(d, 16) && (ldd * (bf16 ? 2 : 4)) % 16 == 0;
     std::memset(&md, 0, sizeof(md));

@@ -89,7 +89,10 @@ def check_gemm(fmt, M, N, K, seed=0, crs=True):
                                    # several 256 x 256 pair tiles both ways; the last tile row and
                                    # column leave the second CTA of the pair without rows of A / B;
                                    # K of 13 steps ends in a one-step chunk
-                                   (513, 770, 832)])
+                                   (513, 770, 832),
+                                   # K of 32, 96, 160: a last K step of 32 elements (zero codes
+                                   # past K, the export's zeroed scale padding)
+                                   (130, 260, 32), (129, 257, 96), (300, 520, 160)])
 def test_fp4_gemm_parity(fmt, M, N, K):
     check_gemm(FMT[fmt], M, N, K, seed=M + N + K)
 
@@ -110,9 +113,9 @@ def test_fp4_gemm_degenerate_sizes(fmt):
                          d=torch.full((3, 5), 7.0, device="cuda"))
     torch.cuda.synchronize()
     assert torch.equal(d, torch.zeros_like(d))                       # K = 0: empty sums
-    with pytest.raises(F.FocusError):
-        F.focus_fp4_gemm(f, torch.zeros((4, 16), dtype=torch.uint8, device="cuda"), z,
-                         torch.zeros((4, 16), dtype=torch.uint8, device="cuda"), z, one, one)  # K = 32
+    with pytest.raises(F.FocusError):   # K = 16: code rows off 16-byte boundaries, refused before launch
+        F.focus_fp4_gemm(f, torch.zeros((4, 8), dtype=torch.uint8, device="cuda"), z,
+                         torch.zeros((4, 8), dtype=torch.uint8, device="cuda"), z, one, one)
 
 
 @pytest.mark.parametrize("fmt", ["mx", "nv"])
