@@ -1287,6 +1287,20 @@ def gemm_arm(args, device):
         for (ac, at, aa), (wc, wt, wa), d in jobs:
             F.focus_fp4_gemm(fmt, ac, at, wc, wt, aa, wa, d=d, timeout_flag=flag)
 
+    # the projections are independent: in the captured step each GEMM runs on
+    # its own graph branch, so that one GEMM's last, partly filled wave of
+    # tiles overlaps the next one's first
+    side = [torch.cuda.Stream(device) for _ in jobs]
+
+    def step_branches():
+        main = torch.cuda.current_stream(device)
+        for st, ((ac, at, aa), (wc, wt, wa), d) in zip(side, jobs):
+            st.wait_stream(main)
+            with torch.cuda.stream(st):
+                F.focus_fp4_gemm(fmt, ac, at, wc, wt, aa, wa, d=d, timeout_flag=flag)
+        for st in side:
+            main.wait_stream(st)
+
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize(device)
@@ -1295,7 +1309,7 @@ def gemm_arm(args, device):
     cap = torch.cuda.Stream(device)
     cap.wait_stream(torch.cuda.current_stream(device))
     with torch.cuda.graph(graph, stream=cap):
-        step()
+        (step if args.serial else step_branches)()
     torch.cuda.current_stream(device).wait_stream(cap)
     graph.replay()
     torch.cuda.synchronize(device)
@@ -1359,6 +1373,9 @@ def gemm_arm(args, device):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "e2m1", "data": "synthetic",
         "config": {"workload": f"{args.workload} projections x {GEMM_TOKENS} tokens", "fmt": args.fmt,
                    "gemms": [[GEMM_TOKENS, t.rows, t.cols] for t in w.tensors], "out": "bf16",
+                   "launch": ("the GEMMs one after another in one captured graph (programmatic dependent "
+                              "launches)" if args.serial else
+                              "one captured graph, each GEMM on its own branch (independent projections)"),
                    "l2": "operands of one GEMM fit in L2 (weights <= 25 MB of codes); outputs stream"},
         "roofline": {"bound": "tensor", "kernel": f"fp4_gemm_kernel ({w.tensors[big].name})",
                      "achieved": round(big_tflops, 1), "peak": round(peak, 1), "peak_kind": peak_kind,
@@ -1390,6 +1407,8 @@ def main():
                          "tensor's phases chained on its own branch)")
     ap.add_argument("--group", action="store_true",
                     help="one group launch per phase for all tensors instead of per-tensor launches")
+    ap.add_argument("--serial", action="store_true",
+                    help="--gemm: the step's GEMMs one after another on one stream instead of on graph branches")
     ap.add_argument("--gemm", action="store_true",
                     help="time the W4A4 FP4 GEMMs of the workload's projections on their exports")
     ap.add_argument("--no-cpu-baseline", action="store_true")
