@@ -22,13 +22,14 @@ timed steps.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
                   [--workload NAME --fmt mxfp4|nvfp4 --shared --sfp --adam
                    --io f16 --sub B --staged --group --no-e2e --no-cpu-baseline]
-  python bench.py --gemm [--fmt mxfp4] [--workload NAME]
+  python bench.py --gemm [--fmt mxfp4] [--workload NAME] [--serial]
 
 Other workloads (the Qwen3-4B layer, the Llama-3-8B block, the 70B layer
 set, sweep tensors) are measured the same way with --workload.
 `--impl reference` times the CPU oracle on a bounded sample of the same
 workload.  `--gemm` times the W4A4 FP4 GEMMs of a layer's projections on
-their exports (default: the Qwen3-4B layer x 8192 tokens).
+their exports (default: the Qwen3-4B layer x 8192 tokens), the independent
+GEMMs of a step on parallel graph branches (--serial: one after another).
 
 Under torchrun (N > 1) every rank runs the same workload on its own GPU
 (replicas; no data-path collective), the step time is the max over ranks and
