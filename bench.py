@@ -99,9 +99,9 @@ def bytes_per_elem(case: Case, esz: int) -> dict:
 # was taken on.  Reported only while the sources are unchanged.
 TRAFFIC = {
     # fq_block_kernel<1,1,8,2> on [32768, 4096] of the activations: 637.6 MB
-    # read + 336.6 MB written for 134,217,728 elements
+    # read + 336.8 MB written for 134,217,728 elements
     # (profiles/fq_bwd_nvfp4_act_32768rows.txt)
-    ("act_262144x4096", "nvfp4", "bwd"): {"sources": "ca817502aaf8d410", "bytes_per_elem": 7.2588},
+    ("act_262144x4096", "nvfp4", "bwd"): {"sources": "42cba47e57d406a3", "bytes_per_elem": 7.2604},
 }
 
 # AdamW hyper-parameters of the fused optimizer: the paper's learning rates

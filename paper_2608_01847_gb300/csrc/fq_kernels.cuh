@@ -635,7 +635,10 @@ struct Span {
 // with AdamW on the coefficients takes the same counts (Llama-70B layer set,
 // NVFP4 6664 -> 6883 GB/s, MXFP4 6617 -> 6704; Qwen3-4B 6448 -> 6547, against
 // one CTA fewer); with S^fp learned as well its extra state spills too much
-// and keeps one fewer (at the backward's count: 70B NVFP4 6361 -> 6177).
+// and keeps one fewer (at the backward's count: 70B NVFP4 6361 -> 6177) --
+// except NVFP4 with 16-bit elements and sub-blocks of 8 or more since the
+// optimizer's square root and division are the approximate forms (70B: 6571
+// -> 6793 at 4 CTAs; MXFP4 at 3: 6297 -> 6154).
 // The MXFP4 backward with binary16 elements is the exception: its
 // conversions spill three times as much at 3 CTAs, and 2 CTAs per SM are
 // faster (Llama-70B layer set, fp16 I/O: backward 5927 -> 6413 GB/s).
@@ -651,7 +654,7 @@ struct MinCtas {
     // a thread of a pair kernel holds 16 elements, as an NVFP4 thread does
     static constexpr int FMT = PairBlocks<FMT_, DT, SUB, MODE>::value ? 1 : FMT_;
     static constexpr int bwd = FMT == 1 ? (DT != 0 ? 4 : 3) : (DT == 1 ? 3 : 2);
-    static constexpr int adam_sfp = FMT == 1 ? 3 : 2;
+    static constexpr int adam_sfp = FMT == 1 ? ((DT != 0 && SUB >= 8) ? 4 : 3) : 2;
     static constexpr int base =
         MODE == kBwdSA ? adam_sfp : (MODE >= kBwd) ? bwd : (MODE == kPack && FMT == 1) ? 5 : 4;
     static constexpr int value = base - ((SUB == 2 && !(FMT == 1 && DT != 0 && MODE == kBwd)) ? 1 : 0);
