@@ -1,0 +1,98 @@
+"""CPU: the oracle's pins catch plausible mistakes in the oracle.  Each case
+plants one mistake in a copy of oracle/focus_oracle.c (a swapped operand, a
+dropped term, a wrong sign, an off-by-one exponent, a wrong tie rule, a
+wrong nibble order, a wrong constant), builds it with the oracle's own
+flags, points the oracle module at that build, and runs a fast subset of
+the pins of test_oracle_pins.py: at least one of them must fail.  The same
+subset passes on the unmodified source built the same way."""
+import os
+import subprocess
+
+import pytest
+
+import oracle as O
+import test_oracle_pins as P
+
+SRC = os.path.join(os.path.dirname(O.__file__), "focus_oracle.c")
+
+# (name, text in focus_oracle.c, replacement, occurrences)
+MUTANTS = [
+    ("dequantized by the relaxed scale", "yv = focus_oracle_e2m1_value(code) * s_dq;",
+     "yv = focus_oracle_e2m1_value(code) * s_q;", 1),
+    ("dL/dc_i without the c_i^k factor", "ksum_add(&gc, G * (double)d);", "ksum_add(&gc, G);", 1),
+    ("coefficient gradient sign", "double G = -ksum_value(&T) / (ce * ce);",
+     "double G = ksum_value(&T) / (ce * ce);", 1),
+    ("coefficient gradient over c_eff, not c_eff^2", "double G = -ksum_value(&T) / (ce * ce);",
+     "double G = -ksum_value(&T) / ce;", 1),
+    ("E8M0 ceiling off by one at powers of two", "e = (f == 0.5) ? E - 1 : E;", "e = E;", 1),
+    ("E2M1 ties away from the even code", "(d == bestd && (c & 1) == 0)", "(d == bestd)", 2),
+    ("even element in the high nibble", "if ((col & 1) == 0) *p = (uint8_t)((*p & 0xF0) | code);",
+     "if ((col & 1) == 1) *p = (uint8_t)((*p & 0xF0) | code);", 1),
+    ("alpha constant", "*alpha_out = amax / 2688.0f;", "*alpha_out = amax / 2687.0f;", 1),
+    ("relaxed scale divided by the coefficients (Eq. 6 inverted)", "float s_q = s_dq * c_eff;",
+     "float s_q = s_dq / c_eff;", 2),
+    ("E4M3 exponent bias", "ldexp(1.0 + m / 8.0, e - 7)", "ldexp(1.0 + m / 8.0, e - 8)", 1),
+    ("STE ratio inverted", "float rho = dead ? 0.0f : s_dq / s_q;", "float rho = dead ? 0.0f : s_q / s_dq;", 1),
+]
+
+# fast pins (a few seconds together), with their parameters
+PINS = [
+    (P.test_hand_mxfp4_block_crs, ()),
+    (P.test_hand_gx_rounding_order, ()),
+    (P.test_hand_mxfp4_ties, ()),
+    (P.test_hand_nvfp4_blocks, ()),
+    (P.test_alpha_closed_form, ()),
+    (P.test_e4m3_decode_matches_torch, ()),
+    (P.test_e2m1_brute_force_grid, ()),
+    (P.test_e8m0_ceil_and_floor_rules, ()),
+    (P.test_crs_at_one_equals_rtn, (O.MXFP4,)),
+    (P.test_crs_at_one_equals_rtn, (O.NVFP4,)),
+    (P.test_dequant_of_export_equals_forward, (O.MXFP4, "f32")),
+    (P.test_dequant_of_export_equals_forward, (O.NVFP4, "bf16")),
+    (P.test_input_gradient_is_g_over_c, (O.MXFP4,)),
+    (P.test_coefficient_gradients_finite_difference, (O.NVFP4, 8)),
+    (P.test_autograd_restatement, (O.MXFP4,)),
+]
+
+
+def build_variant(tmp, name, text):
+    src = os.path.join(tmp, f"{name}.c")
+    lib = os.path.join(tmp, f"lib{name}.so")
+    with open(src, "w") as f:
+        f.write(text)
+    subprocess.check_call(["gcc", *O.CFLAGS, src, "-o", lib, "-lm"])
+    return lib
+
+
+def failing_pins(lib):
+    """Names of the pins in PINS that fail with the oracle loaded from lib."""
+    saved = (O._LIB, O._lib)
+    O._LIB, O._lib = lib, None
+    failed = []
+    try:
+        for fn, args in PINS:
+            try:
+                fn(*args)
+            except Exception as e:   # a failed assertion, or a mutant's exception
+                failed.append(f"{fn.__name__}{args}: {type(e).__name__}")
+    finally:
+        O._LIB, O._lib = saved
+    return failed
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(SRC) as f:
+        return f.read()
+
+
+def test_unmodified_source_passes_the_pins(tmp_path, source):
+    assert failing_pins(build_variant(str(tmp_path), "control", source)) == []
+
+
+@pytest.mark.parametrize("name,text,repl,count", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_planted_mistake_fails_a_pin(tmp_path, source, name, text, repl, count):
+    assert source.count(text) == count, (name, source.count(text))
+    lib = build_variant(str(tmp_path), "mutant", source.replace(text, repl))
+    failed = failing_pins(lib)
+    assert failed, f"no pin caught: {name}"
