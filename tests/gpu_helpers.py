@@ -164,3 +164,19 @@ def assert_adamw_close(got, p0, m0, v0, ref, floor, lr, hp, step, what):
                                  f"[{lo.reshape(-1)[i]!r}, {hi.reshape(-1)[i]!r}]")
     # the interval contains the oracle's exact step
     assert np.all((ref["p"] >= pl) & (ref["p"] <= ph)), f"{what}: oracle p outside its bound"
+
+
+def gemm_bound(K, mag, ref):
+    """Tolerance of the FP4 GEMM (R18): exact products, binary32 accumulation
+    inside the tensor core -- (K/16 + 8) 2^-23 sum|A B| + 2^-23 |D|."""
+    return (K / 16 + 8) * 2.0 ** -23 * np.asarray(mag) + 2.0 ** -23 * np.abs(ref) + 1e-30
+
+
+def assert_gemm_close(got, ref, mag, K, what="D"):
+    """got: the device's D (any float array); ref, mag: the oracle's D and
+    its sum of |products| (binary64)."""
+    got = np.asarray(got, np.float64)
+    err = np.abs(got - ref)
+    bad = np.argwhere(~(err <= gemm_bound(K, mag, ref)))
+    assert bad.size == 0, (f"{what}: {len(bad)} of {got.size} outside the bound; first {tuple(bad[0])}: "
+                           f"got {got[tuple(bad[0])]!r} ref {ref[tuple(bad[0])]!r}")

@@ -18,7 +18,7 @@ import oracle as O
 from paper_2608_01847_gb300 import build as B
 from paper_2608_01847_gb300 import focus as F
 from paper_2608_01847_gb300 import workloads as W
-from gpu_helpers import assert_bits_equal, dev, host
+from gpu_helpers import assert_bits_equal, assert_gemm_close, dev, gemm_bound, host
 
 pytestmark = pytest.mark.gpu
 
@@ -73,12 +73,7 @@ def check_gemm(fmt, M, N, K, seed=0, crs=True):
     assert int(flag.item()) == 0, "MMA wait gave up"
     ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], fmt, aa, ab)
     mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], fmt, aa, ab)
-    got = host(d).astype(np.float64)
-    bound = (K / 16 + 8) * 2.0 ** -23 * mag + 2.0 ** -23 * np.abs(ref) + 1e-30
-    err = np.abs(got - ref)
-    bad = np.argwhere(~(err <= bound))
-    assert bad.size == 0, (f"{len(bad)} of {got.size} outside the bound; first {tuple(bad[0])}: "
-                           f"gpu {got[tuple(bad[0])]!r} ref {ref[tuple(bad[0])]!r}")
+    assert_gemm_close(host(d), ref, mag, K)
     return d, ref
 
 
@@ -207,7 +202,7 @@ def test_fp4_gemm_full_size_sampled(fmt):
     assert torch.equal(ac, ac2) and torch.equal(bc, bc2)
     ref = O.fp4_gemm(ra["codes"], ra["scales"], rb["codes"], rb["scales"], f, aa, ab)
     mag = O.fp4_gemm(ra["codes"] & 0x77, ra["scales"], rb["codes"] & 0x77, rb["scales"], f, aa, ab)
-    bound = (K / 16 + 8) * 2.0 ** -23 * mag + 2.0 ** -23 * np.abs(ref) + 1e-30
+    bound = gemm_bound(K, mag, ref)
     ia, ib = torch.from_numpy(ma).cuda(), torch.from_numpy(nb).cuda()
     got32 = host(d32[ia][:, ib]).astype(np.float64)
     got16 = host(d16[ia][:, ib].float()).astype(np.float64)
