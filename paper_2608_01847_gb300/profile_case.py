@@ -57,6 +57,9 @@ def main():
     ap.add_argument("--pad", type=int, default=0,
                     help="row pitch cols + PAD elements (PAD = 8 bf16: rows on 16-byte, not 32-byte, "
                          "boundaries)")
+    ap.add_argument("--library", action="store_true",
+                    help="gemm, NVFP4: NVIDIA's block-scaled GEMM (cuBLASLt through torch._scaled_mm) on the "
+                         "same exports instead of fp4_gemm_kernel")
     ap.add_argument("--launches", type=int, default=3)
     a = ap.parse_args()
 
@@ -109,6 +112,11 @@ def main():
         wc, wt = F.focus_pack_mma(x, fmt, alpha=alpha)
         dmat = torch.empty((a.tokens, rows), dtype=torch.bfloat16, device="cuda")
         del act, g, gx, y
+        if a.library:
+            if fmt != F.FOCUS_NVFP4:
+                raise SystemExit("--library: NVFP4 only")
+            a4, w4 = ac.view(torch.float4_e2m1fn_x2), wc.view(torch.float4_e2m1fn_x2).t()
+            sa, sw = at.view(torch.float8_e4m3fn), wt.view(torch.float8_e4m3fn)
 
     if a.adam:
         # the paper's learning rates (Sec. 4.1), PyTorch's AdamW defaults
@@ -124,6 +132,8 @@ def main():
             F.focus_fq_bwd_adamw(x, g, fmt, step, hp, crs=crs, dgs=dgs, sfp=sfp, moments=moments,
                                  alpha=alpha, sub_block=a.sub, shared=a.shared, gx=gx,
                                  want_gx=not a.no_gx, ws=ws)
+        elif a.phase == "gemm" and a.library:
+            torch._scaled_mm(a4, w4, sa, sw, out_dtype=torch.bfloat16)
         elif a.phase == "gemm":
             F.focus_fp4_gemm(fmt, ac, at, wc, wt, act_alpha, alpha, d=dmat)
         elif a.phase == "alpha":
@@ -139,6 +149,9 @@ def main():
 
     torch.cuda.synchronize()
     times = []
+    # the timed launches inside one NVTX range, so that a profiler can take
+    # them alone (ncu --nvtx --nvtx-include "launches/")
+    torch.cuda.nvtx.range_push("launches")
     for _ in range(a.launches):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
@@ -146,10 +159,12 @@ def main():
         e1.record()
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1))
+    torch.cuda.nvtx.range_pop()
     if a.phase == "gemm":
         flops = 2 * a.tokens * rows * cols
         print(json.dumps({"phase": "gemm", "tensor": f"{a.workload}/{a.tensor}",
-                          "shape": [a.tokens, rows, cols], "fmt": a.fmt, "ms": times,
+                          "shape": [a.tokens, rows, cols], "fmt": a.fmt,
+                          "kernel": "cuBLASLt (torch._scaled_mm)" if a.library else "fp4_gemm_kernel", "ms": times,
                           "tflops_last": flops / (times[-1] * 1e-3) / 1e12}))
         return
     n = rows * cols
