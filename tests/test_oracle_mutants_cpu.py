@@ -1,10 +1,14 @@
 """CPU: the oracle's pins catch plausible mistakes in the oracle.  Each case
 plants one mistake in a copy of oracle/focus_oracle.c (a swapped operand, a
 dropped term, a wrong sign, an off-by-one exponent, a wrong tie rule, a
-wrong nibble order, a wrong constant), builds it with the oracle's own
-flags, points the oracle module at that build, and runs a fast subset of
-the pins of test_oracle_pins.py: at least one of them must fail.  The same
-subset passes on the unmodified source built the same way."""
+wrong nibble order, a wrong constant, a strict mask boundary, a factor of
+the wrong coefficient), builds it with the oracle's own flags, points the
+oracle module at that build, and runs a fast subset of the pins of
+test_oracle_pins.py: at least one of them must fail.  The same subset
+passes on the unmodified source built the same way.  The AdamW step, which
+the oracle states in Python, gets the same treatment on a copy of its
+source."""
+import inspect
 import os
 import subprocess
 
@@ -33,6 +37,21 @@ MUTANTS = [
      "float s_q = s_dq / c_eff;", 2),
     ("E4M3 exponent bias", "ldexp(1.0 + m / 8.0, e - 7)", "ldexp(1.0 + m / 8.0, e - 8)", 1),
     ("STE ratio inverted", "float rho = dead ? 0.0f : s_dq / s_q;", "float rho = dead ? 0.0f : s_q / s_dq;", 1),
+    ("clipped STE mask strict at |u| = 6", "if (ste == OR_STE_CLIPPED) mask = fabsf(u) <= 6.0f;",
+     "if (ste == OR_STE_CLIPPED) mask = fabsf(u) < 6.0f;", 1),
+    ("clipped STE mask never applied", "if (ste == OR_STE_CLIPPED) mask = fabsf(u) <= 6.0f;",
+     "if (ste == -1) mask = fabsf(u) <= 6.0f;", 1),
+    ("shared-row CRS gradient times c instead of c^k", "ksum_add(&acc_c[j], G * (double)d);",
+     "ksum_add(&acc_c[j], G * (double)c);", 1),
+    ("shared-row DGS gradient without c", "ksum_add(&acc_d[j * K + k], G * (double)c);",
+     "ksum_add(&acc_d[j * K + k], G);", 1),
+    ("S^fp gradient: sign of the x / S^q term", "ksum_add(&gs, gq - gu);", "ksum_add(&gs, gq + gu);", 1),
+    ("S^fp gradient: the STE term ignores the mask", "double gu = mask ? (double)gv * (double)xv / sq_exact : 0.0;",
+     "double gu = (double)gv * (double)xv / sq_exact;", 1),
+    ("S^fp gradient without alpha (NVFP4)", "double ds = (fmt == OR_NVFP4) ? (double)alpha : 1.0;",
+     "double ds = 1.0;", 1),
+    ("OCP floor rule off by one", "e = (E - 1) - 2;", "e = E - 2;", 1),
+    ("NVFP4 scale denominator without the 6", "float den = alpha * 6.0f;", "float den = alpha * 4.0f;", 1),
 ]
 
 # fast pins (a few seconds together), with their parameters
@@ -52,6 +71,28 @@ PINS = [
     (P.test_input_gradient_is_g_over_c, (O.MXFP4,)),
     (P.test_coefficient_gradients_finite_difference, (O.NVFP4, 8)),
     (P.test_autograd_restatement, (O.MXFP4,)),
+    (P.test_clipped_ste_masks_saturated, ()),
+    (P.test_clipped_ste_keeps_the_saturation_boundary, ()),
+    (P.test_shared_row_gradients_sum_over_rows, ()),
+    (P.test_hand_mxfp4_sfp_gradient, ()),
+    (P.test_hand_mxfp4_sfp_gradient_clipped_ste, ()),
+    (P.test_sfp_gradient_autograd, (O.NVFP4,)),
+]
+
+# (name, text in oracle.adamw's source, replacement)
+ADAMW_MUTANTS = [
+    ("weight decay skipped", "p = np.asarray(p, np.float64) * (1.0 - lr * weight_decay)", "p = np.asarray(p, np.float64)"),
+    ("second moment without bias correction", "vhat = v / (1.0 - beta2 ** t)", "vhat = v"),
+    ("epsilon inside the square root", "(np.sqrt(vhat) + eps)", "np.sqrt(vhat + eps)"),
+    ("first moment with the second moment's beta",
+     "m = beta1 * np.asarray(m, np.float64) + (1.0 - beta1) * g",
+     "m = beta2 * np.asarray(m, np.float64) + (1.0 - beta2) * g"),
+]
+
+ADAMW_PINS = [
+    (P.test_adamw_matches_torch, ()),
+    (P.test_adamw_first_step_closed_form, ()),
+    (P.test_bwd_adamw_equals_autograd_and_torch_adamw, (O.MXFP4,)),
 ]
 
 
@@ -64,20 +105,43 @@ def build_variant(tmp, name, text):
     return lib
 
 
+def run_pins(pins):
+    failed = []
+    for fn, args in pins:
+        try:
+            fn(*args)
+        except Exception as e:   # a failed assertion, or a mutant's exception
+            failed.append(f"{fn.__name__}{args}: {type(e).__name__}")
+    return failed
+
+
 def failing_pins(lib):
     """Names of the pins in PINS that fail with the oracle loaded from lib."""
     saved = (O._LIB, O._lib)
     O._LIB, O._lib = lib, None
-    failed = []
     try:
-        for fn, args in PINS:
-            try:
-                fn(*args)
-            except Exception as e:   # a failed assertion, or a mutant's exception
-                failed.append(f"{fn.__name__}{args}: {type(e).__name__}")
+        return run_pins(PINS)
     finally:
         O._LIB, O._lib = saved
-    return failed
+
+
+def adamw_variant(text, repl):
+    """oracle.adamw rebuilt from its source with one replacement, in the
+    oracle module's namespace."""
+    src = inspect.getsource(O.adamw)
+    assert src.count(text) == 1, text
+    ns = dict(vars(O))
+    exec(src.replace(text, repl), ns)
+    return ns["adamw"]
+
+
+def failing_adamw_pins(fn):
+    saved = O.adamw
+    O.adamw = fn
+    try:
+        return run_pins(ADAMW_PINS)
+    finally:
+        O.adamw = saved
 
 
 @pytest.fixture(scope="module")
@@ -96,3 +160,12 @@ def test_planted_mistake_fails_a_pin(tmp_path, source, name, text, repl, count):
     lib = build_variant(str(tmp_path), "mutant", source.replace(text, repl))
     failed = failing_pins(lib)
     assert failed, f"no pin caught: {name}"
+
+
+def test_unmodified_adamw_passes_its_pins():
+    assert failing_adamw_pins(adamw_variant("np.sqrt(vhat)", "np.sqrt(vhat)")) == []
+
+
+@pytest.mark.parametrize("name,text,repl", ADAMW_MUTANTS, ids=[m[0] for m in ADAMW_MUTANTS])
+def test_planted_adamw_mistake_fails_a_pin(name, text, repl):
+    assert failing_adamw_pins(adamw_variant(text, repl)), f"no pin caught: {name}"

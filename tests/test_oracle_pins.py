@@ -592,6 +592,22 @@ def test_clipped_ste_masks_saturated():
     assert b["gcrs"][0, 0] == pytest.approx(-float(np.float32(0.1)) / 0.81, rel=1e-6)
 
 
+def test_clipped_ste_keeps_the_saturation_boundary():
+    """Clipped STE mask [|u| <= 6] (Sec. 3.2 with the clamp convention): an
+    element exactly at |u| = 6 keeps its gradient.  MXFP4 block max 1.5 ->
+    S^dq = 0.25 (ceiling rule), c = 1: x = 1.5 and -1.5 give u = +-6, x = 0.75
+    gives u = 3; at c = 1 the ratio is 1, so gx = g on all three, and the CRS
+    gradient is -(sum g x) / c^2 = -(1.5 * 1 + (-1.5) * 2 + 0.75 * 4)."""
+    x = np.zeros((1, 32), np.float32)
+    x[0, :3] = [1.5, -1.5, 0.75]
+    g = np.zeros_like(x)
+    g[0, :3] = [1.0, 2.0, 4.0]
+    crs = np.ones((1, 1), np.float32)
+    b = O.bwd(x, g, O.MXFP4, crs=crs, ste=O.STE_CLIPPED)
+    assert list(b["gx"][0, :3]) == [1.0, 2.0, 4.0]
+    assert b["gcrs"][0, 0] == pytest.approx(-1.5, rel=1e-12)
+
+
 def test_nvfp4_all_zero_tensor_is_dead():
     x = np.zeros((4, 32), np.float32)
     g = np.ones_like(x)
@@ -668,6 +684,31 @@ def test_hand_mxfp4_sfp_gradient():
     expect = float(np.sum(np.array([2.0, -1.0, 0.5, 4.0]) - u))
     assert b["gsfp"][0, 0] == pytest.approx(expect, rel=1e-7)
     assert expect == pytest.approx(-1.124, abs=1e-6)
+
+
+def test_hand_mxfp4_sfp_gradient_clipped_ste():
+    """dL/dS^dq = sum g (q - mask x / S^q) with the clipped mask [|u| <= 6]
+    applied to the STE term only (q is the forward's value): block
+    [1.5, 1.45, 0.1, 0...], S^fp = 0.25 -> S^dq = 0.25, c = 0.9 (S^q = 0.225),
+    u = [6.67, 6.44, 0.44] -> q = [6, 6, 0.5], g = 1 on the three:
+    clipped (6 - 0) + (6 - 0) + (0.5 - 0.1 / 0.225) = 12.0556;
+    identity (6 - 6.667) + (6 - 6.444) + (0.5 - 0.444) = -1.0556."""
+    x = np.zeros((1, 32), np.float32)
+    x[0, :3] = [1.5, 1.45, 0.1]
+    g = np.zeros_like(x)
+    g[0, :3] = 1
+    crs = np.array([[0.9]], np.float32)
+    sfp = np.array([[0.25]], np.float32)
+    sq = 0.25 * float(np.float32(0.9))
+    xs = x[0, :3].astype(np.float64)
+    q = np.array([6.0, 6.0, 0.5])
+    expect = {O.STE_CLIPPED: float(np.sum(q - np.array([0.0, 0.0, 1.0]) * xs / sq)),
+              O.STE_IDENTITY: float(np.sum(q - xs / sq))}
+    assert expect[O.STE_CLIPPED] == pytest.approx(12.0556, abs=1e-4)
+    assert expect[O.STE_IDENTITY] == pytest.approx(-1.0556, abs=1e-4)
+    for ste, e in expect.items():
+        b = O.bwd(x, g, O.MXFP4, crs=crs, sfp=sfp, ste=ste, want_gsfp=True)
+        assert b["gsfp"][0, 0] == pytest.approx(e, rel=1e-7)
 
 
 def test_sfp_rounding_rules():
