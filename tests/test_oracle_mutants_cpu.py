@@ -5,9 +5,10 @@ wrong nibble order, a wrong constant, a strict mask boundary, a factor of
 the wrong coefficient), builds it with the oracle's own flags, points the
 oracle module at that build, and runs a fast subset of the pins of
 test_oracle_pins.py: at least one of them must fail.  The same subset
-passes on the unmodified source built the same way.  The AdamW step, which
-the oracle states in Python, gets the same treatment on a copy of its
-source."""
+passes on the unmodified source built the same way.  The oracle's Python
+functions (the AdamW step, the MMA scale-tile layout, the GEMM on an
+export) get the same treatment on copies of their source, each against
+its own pins."""
 import inspect
 import os
 import subprocess
@@ -52,6 +53,15 @@ MUTANTS = [
      "double ds = 1.0;", 1),
     ("OCP floor rule off by one", "e = (E - 1) - 2;", "e = E - 2;", 1),
     ("NVFP4 scale denominator without the 6", "float den = alpha * 6.0f;", "float den = alpha * 4.0f;", 1),
+    ("bf16 rounding ties away from even", "return (uint16_t)((b + 0x7FFFu + lsb) >> 16);",
+     "return (uint16_t)((b + 0x8000u) >> 16);", 1),
+    ("binary16 rounding ties up", "return fmod(f, 2.0) != 0.0 ? f + 1.0 : f;", "return f + 1.0;", 1),
+    ("binary16 subnormals one binade off", "if (e == 0) v = ldexpf((float)m, -24);",
+     "if (e == 0) v = ldexpf((float)m, -25);", 1),
+    ("dequantization with swapped nibbles", "int code = (col & 1) ? (byte >> 4) : (byte & 15);",
+     "int code = (col & 1) ? (byte & 15) : (byte >> 4);", 1),
+    ("NVFP4 dequantization without alpha", ": focus_oracle_e4m3_decode(sb) * alpha;",
+     ": focus_oracle_e4m3_decode(sb);", 1),
 ]
 
 # fast pins (a few seconds together), with their parameters
@@ -77,23 +87,39 @@ PINS = [
     (P.test_hand_mxfp4_sfp_gradient, ()),
     (P.test_hand_mxfp4_sfp_gradient_clipped_ste, ()),
     (P.test_sfp_gradient_autograd, (O.NVFP4,)),
+    (P.test_bf16_rne_matches_torch, ()),
+    (P.test_f16_decode_all_patterns_matches_numpy, ()),
+    (P.test_f16_rne_matches_numpy, ()),
 ]
 
-# (name, text in oracle.adamw's source, replacement)
-ADAMW_MUTANTS = [
-    ("weight decay skipped", "p = np.asarray(p, np.float64) * (1.0 - lr * weight_decay)", "p = np.asarray(p, np.float64)"),
-    ("second moment without bias correction", "vhat = v / (1.0 - beta2 ** t)", "vhat = v"),
-    ("epsilon inside the square root", "(np.sqrt(vhat) + eps)", "np.sqrt(vhat + eps)"),
-    ("first moment with the second moment's beta",
+# planted mistakes in the oracle's Python functions:
+# (name, function, text in its source, replacement)
+PY_MUTANTS = [
+    ("AdamW: weight decay skipped", "adamw", "p = np.asarray(p, np.float64) * (1.0 - lr * weight_decay)",
+     "p = np.asarray(p, np.float64)"),
+    ("AdamW: second moment without bias correction", "adamw", "vhat = v / (1.0 - beta2 ** t)", "vhat = v"),
+    ("AdamW: epsilon inside the square root", "adamw", "(np.sqrt(vhat) + eps)", "np.sqrt(vhat + eps)"),
+    ("AdamW: first moment with the second moment's beta", "adamw",
      "m = beta1 * np.asarray(m, np.float64) + (1.0 - beta1) * g",
      "m = beta2 * np.asarray(m, np.float64) + (1.0 - beta2) * g"),
+    ("MMA scale tiles: row and column offsets swapped in a line", "mma_scale_tiles",
+     "(rr % 32) * 16 + (rr // 32) * 4 + cc", "(rr % 32) * 16 + (rr // 32) + cc * 4"),
+    ("GEMM: NVFP4 without the per-tensor scales", "fp4_gemm",
+     "d = d * (float(np.float32(alpha_a)) * float(np.float32(alpha_b)))", "d = d"),
+    ("GEMM: even element from the high nibble", "fp4_gemm", "nib[:, 0::2] = codes & 15", "nib[:, 0::2] = codes >> 4"),
+    ("GEMM: E8M0 bias off by one", "fp4_gemm", "s = np.ldexp(1.0, sb.astype(np.int64) - 127)",
+     "s = np.ldexp(1.0, sb.astype(np.int64) - 126)"),
 ]
 
-ADAMW_PINS = [
-    (P.test_adamw_matches_torch, ()),
-    (P.test_adamw_first_step_closed_form, ()),
-    (P.test_bwd_adamw_equals_autograd_and_torch_adamw, (O.MXFP4,)),
-]
+# the pins each Python function is held to
+PY_PINS = {
+    "adamw": [(P.test_adamw_matches_torch, ()), (P.test_adamw_first_step_closed_form, ()),
+              (P.test_bwd_adamw_equals_autograd_and_torch_adamw, (O.MXFP4,))],
+    "mma_scale_tiles": [(P.test_mma_scale_tiles_hand_offsets, ()), (P.test_mma_scale_tiles_is_a_permutation, ())],
+    "fp4_gemm": [(P.test_fp4_gemm_matches_independent_dequant, (O.MXFP4,)),
+                 (P.test_fp4_gemm_matches_independent_dequant, (O.NVFP4,)),
+                 (P.test_fp4_gemm_is_the_product_of_fake_quantized_operands, (O.NVFP4,))],
+}
 
 
 def build_variant(tmp, name, text):
@@ -125,23 +151,23 @@ def failing_pins(lib):
         O._LIB, O._lib = saved
 
 
-def adamw_variant(text, repl):
-    """oracle.adamw rebuilt from its source with one replacement, in the
-    oracle module's namespace."""
-    src = inspect.getsource(O.adamw)
+def py_variant(name, text, repl):
+    """Oracle function `name` rebuilt from its source with one replacement,
+    in the oracle module's namespace."""
+    src = inspect.getsource(getattr(O, name))
     assert src.count(text) == 1, text
     ns = dict(vars(O))
     exec(src.replace(text, repl), ns)
-    return ns["adamw"]
+    return ns[name]
 
 
-def failing_adamw_pins(fn):
-    saved = O.adamw
-    O.adamw = fn
+def failing_py_pins(name, fn):
+    saved = getattr(O, name)
+    setattr(O, name, fn)
     try:
-        return run_pins(ADAMW_PINS)
+        return run_pins(PY_PINS[name])
     finally:
-        O.adamw = saved
+        setattr(O, name, saved)
 
 
 @pytest.fixture(scope="module")
@@ -162,10 +188,11 @@ def test_planted_mistake_fails_a_pin(tmp_path, source, name, text, repl, count):
     assert failed, f"no pin caught: {name}"
 
 
-def test_unmodified_adamw_passes_its_pins():
-    assert failing_adamw_pins(adamw_variant("np.sqrt(vhat)", "np.sqrt(vhat)")) == []
+@pytest.mark.parametrize("name", sorted(PY_PINS))
+def test_unmodified_python_functions_pass_their_pins(name):
+    assert failing_py_pins(name, py_variant(name, f"def {name}(", f"def {name}(")) == []
 
 
-@pytest.mark.parametrize("name,text,repl", ADAMW_MUTANTS, ids=[m[0] for m in ADAMW_MUTANTS])
-def test_planted_adamw_mistake_fails_a_pin(name, text, repl):
-    assert failing_adamw_pins(adamw_variant(text, repl)), f"no pin caught: {name}"
+@pytest.mark.parametrize("name,fn,text,repl", PY_MUTANTS, ids=[m[0] for m in PY_MUTANTS])
+def test_planted_python_mistake_fails_a_pin(name, fn, text, repl):
+    assert failing_py_pins(fn, py_variant(fn, text, repl)), f"no pin caught: {name}"
